@@ -1,0 +1,377 @@
+#!/usr/bin/env python3
+"""Benchmark: batched complex64 DFT on GB300 tensor cores.
+
+Default workload: n = 65536 (= 16^4, sqrt_m = 16), batch = 1024, N(0,1)
+inputs from seed 1, forward, 3xTF32.  One "step" is one complete forward
+transform of the whole batch (every stage of every pass), inputs resident in
+HBM (512 MiB, larger than the 129 MB L2, so no flush is needed between
+steps).
+
+Prints ONE JSON line on stdout (rank 0).  Logs go to stderr.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl reference]
+
+For N > 1 launch under torchrun: each rank transforms its own batch (weak
+scaling, no collective on the data path; one all-reduce of the timings).
+``--impl reference`` times the fp64 CPU oracle on the host cores on bounded
+samples of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+import numpy as np  # noqa: E402
+
+import inputs  # noqa: E402
+
+METRIC = ("DFT GFLOP/s (5n·log2n) & % of roofline, n=2^16 ×1024 "
+          "complex64, 1×GB300")
+UNIT = "GFLOP/s"
+# nominal dense tensor rates (PFLOP/s): ratio used to scale the measured bf16
+# peak to tf32
+NOMINAL_BF16 = 2.25
+NOMINAL_TF32 = 1.1
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0,
+                  "bf16_tflops_sustained": 1700.0}
+
+
+def log(*a):
+    print(*a, file=sys.stderr, flush=True)
+
+
+def dft_flops(n, batch):
+    return 5.0 * n * math.log2(n) * batch
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return d, "measured"
+    except Exception:
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+class ClockSampler:
+    """nvidia-smi clocks/throttle sampling during the timed region."""
+
+    Q = ("index,clocks.sm,clocks.max.sm,power.draw,"
+         "clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+         "clocks_event_reasons.hw_thermal_slowdown,"
+         "clocks_event_reasons.sw_thermal_slowdown,"
+         "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index):
+        self.gpu = gpu_index
+        self.proc = None
+        self.lines = []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.gpu), "--query-gpu=" + self.Q,
+                 "--format=csv,noheader,nounits", "-lms", "50"],
+                stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+            self.t = threading.Thread(target=self._read, daemon=True)
+            self.t.start()
+        except Exception:
+            self.proc = None
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.t.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown",
+                 "sw_power_cap"]
+        for ln in self.lines:
+            f = [x.strip() for x in ln.split(",")]
+            if len(f) < 9:
+                continue
+            try:
+                sm.append(float(f[1]))
+                mx.append(float(f[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, f[5:9]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": [],
+                    "samples": 0}
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx),
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup():
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return world, rank, local
+
+
+def cpu_baseline(wl, seconds=10.0, sample=32):
+    """The fp64 oracle (radix-2 FFT) on a bounded sample of the workload,
+    using every host core; returns the metric in GFLOP/s."""
+    import oracle
+    n = wl["n"]
+    x = inputs.make(wl["kind"], n, wl["batch"], wl["seed"], first=0,
+                    count=sample)
+    threads = oracle.default_threads()
+    done, used, t0 = 0, 1, time.perf_counter()
+    while True:
+        _, used = oracle.fft_radix2_timed(x, threads=threads)
+        done += sample
+        el = time.perf_counter() - t0
+        if el >= seconds:
+            break
+    return {"value": dft_flops(n, done) / el / 1e9, "unit": UNIT,
+            "cores": used, "kind": "oracle",
+            "sample": "%d transforms (first %d of the workload, repeated) of "
+                      "n=%d through the fp64 recursive radix-2 FFT, %.1f s "
+                      "wall" % (done, sample, n, el)}
+
+
+def run_reference(args, wl):
+    world, rank, _ = dist_setup()
+    if rank != 0:
+        return 0
+    import oracle
+    n = wl["n"]
+    sample = args.ref_sample
+    x = inputs.make(wl["kind"], n, wl["batch"], wl["seed"], first=0,
+                    count=sample)
+    threads = oracle.default_threads()
+    used = 1
+    for _ in range(args.warmup):
+        _, used = oracle.fft_radix2_timed(x, threads=threads)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        _, used = oracle.fft_radix2_timed(x, threads=threads)
+    el = time.perf_counter() - t0
+    value = dft_flops(n, sample) * args.steps / el / 1e9
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": UNIT,
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": el / args.steps * 1e3, "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+        "data": "synthetic", "config": workload_config(wl, args),
+        "cpu_baseline": {"value": value, "unit": UNIT, "cores": used,
+                         "kind": "oracle",
+                         "sample": "%d transforms of n=%d per step (first %d "
+                                   "of the workload), fp64 recursive radix-2 "
+                                   "FFT" % (sample, n, sample)},
+        "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+def workload_config(wl, args):
+    return {"workload": "batched complex64 forward DFT n=%d (=%d^%d) x batch "
+                        "%d, %s inputs seed %d, %s" % (
+                            wl["n"], wl["sqrt_m"],
+                            round(math.log(wl["n"], wl["sqrt_m"])),
+                            wl["batch"], wl["kind"], wl["seed"],
+                            "3xTF32" if args.precision == 3 else "TF32"),
+            "n": wl["n"], "batch": wl["batch"], "sqrt_m": wl["sqrt_m"],
+            "precision": "3xTF32" if args.precision == 3 else "TF32",
+            "l2": "inputs larger than L2 (%d MiB per buffer), no flush"
+                  % (wl["n"] * wl["batch"] * 8 >> 20),
+            "parallelism": "replica/batch shard x%d" % args.gpus}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=200)
+    ap.add_argument("--warmup", type=int, default=10)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="n65536_b1024",
+                    choices=sorted(inputs.WORKLOADS))
+    ap.add_argument("--precision", type=int, default=3, choices=[1, 3])
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    ap.add_argument("--ref-sample", type=int, default=16)
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--e2e-steps", type=int, default=20)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        args.warmup = 3
+    wl = dict(inputs.WORKLOADS[args.workload])
+    if args.impl == "reference":
+        return run_reference(args, wl)
+
+    import torch
+    world, rank, local = dist_setup()
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl")
+    else:
+        dist = None
+    dev = torch.device("cuda", torch.cuda.current_device())
+
+    from paper_1908_06649_gb300 import _build
+    if rank == 0 or world == 1:
+        _build.build()
+    if dist is not None:
+        dist.barrier()
+    import paper_1908_06649_gb300 as pkg
+
+    n, batch, r = wl["n"], wl["batch"], wl["sqrt_m"]
+    log("rank %d: generating %s inputs n=%d batch=%d" % (rank, wl["kind"], n,
+                                                       batch))
+    x_host = inputs.make(wl["kind"], n, batch, wl["seed"] + 1000 * rank)
+    x = torch.from_numpy(x_host).to(dev)
+    y = torch.empty_like(x)
+    plan = pkg.Plan(n, batch, r, args.precision)
+    npass = len(plan.passes())
+    stream = torch.cuda.current_stream()
+
+    for _ in range(args.warmup):
+        plan.forward(x, y)
+    plan.check()
+
+    K = args.steps
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(npass + 1)]
+          for _ in range(K)]
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    # torch creates the CUDA event lazily on its first record
+    for row in ev:
+        for e in row:
+            e.record(stream)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(torch.cuda.current_device()) if rank == 0 else None
+    if clocks:
+        clocks.start()
+        time.sleep(0.2)
+    if dist is not None:
+        dist.barrier()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    for i in range(K):
+        plan.exec_timed(x, y, ev[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if dist is not None:
+        dist.barrier()
+    clk = clocks.stop() if clocks else None
+    plan.check()
+    elapsed_ms = t_start.elapsed_time(t_end)
+    pass_ms = [[ev[i][p].elapsed_time(ev[i][p + 1]) for i in range(K)]
+               for p in range(npass)]
+    if dist is not None:
+        t = torch.tensor([elapsed_ms], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        elapsed_ms = float(t.item())
+
+    ms_per_step = elapsed_ms / K
+    value = dft_flops(n, batch) * world * K / (elapsed_ms * 1e-3) / 1e9
+
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    # per-launch algorithmic bytes: every complex64 point read once and
+    # written once by each pass kernel
+    bytes_launch = 16.0 * n * batch
+    avg = [sum(p) / len(p) for p in pass_ms]
+    dom = max(range(npass), key=lambda i: avg[i])
+    achieved = bytes_launch / (avg[dom] * 1e-3) / 1e9
+    stages = plan.passes()
+    # whole-step roofline: min HBM bytes vs tensor flops at tf32 peak
+    p_tf32 = float(peaks["bf16_tflops"]) * NOMINAL_TF32 / NOMINAL_BF16
+    k = sum(stages)
+    tensor_flops = 8.0 * r * n * batch * k * args.precision
+    t_roof = max(bytes_launch / (hbm * 1e9), tensor_flops / (p_tf32 * 1e12))
+    frac_step = t_roof / (ms_per_step * 1e-3)
+
+    e2e = None
+    if args.e2e_steps > 0:
+        h_in = torch.from_numpy(x_host).pin_memory()
+        h_out = torch.empty_like(h_in).pin_memory()
+        work = torch.empty_like(x)
+        plan.exec_host(h_in, h_out, work)
+        torch.cuda.synchronize()
+        e0 = torch.cuda.Event(enable_timing=True)
+        e1 = torch.cuda.Event(enable_timing=True)
+        if dist is not None:
+            dist.barrier()
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(args.e2e_steps):
+            plan.exec_host(h_in, h_out, work)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        e2e_ms = e0.elapsed_time(e1)
+        if dist is not None:
+            t = torch.tensor([e2e_ms], device=dev, dtype=torch.float64)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            e2e_ms = float(t.item())
+        e2e = {"value": dft_flops(n, batch) * world * args.e2e_steps
+                        / (e2e_ms * 1e-3) / 1e9,
+               "unit": UNIT, "h2d_bytes_per_step": n * batch * 8,
+               "d2h_bytes_per_step": n * batch * 8,
+               "steps": args.e2e_steps}
+
+    plan.destroy()
+    cpu = None
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        cpu = cpu_baseline(wl, seconds=args.cpu_seconds)
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": K, "warmup": args.warmup, "ms_per_step": ms_per_step,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "tf32x3" if args.precision == 3 else "tf32",
+            "data": "synthetic", "config": workload_config(wl, args),
+            "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm,
+                         "unit": "GB/s", "frac": achieved / hbm,
+                         "traffic": None,
+                         "kernel": "dft_pass_kernel pass %d of %d (%d stages)"
+                                   % (dom + 1, npass, stages[dom]),
+                         "peak_source": peak_kind,
+                         "pass_ms": avg},
+            "roofline_step": {"t_roof_ms": t_roof * 1e3, "frac": frac_step,
+                              "hbm_bytes_min": bytes_launch,
+                              "tensor_flops": tensor_flops,
+                              "tf32_peak_tflops": p_tf32,
+                              "tf32_peak_source": "%s bf16 x %.2f/%.2f nominal"
+                                                  % (peak_kind, NOMINAL_TF32,
+                                                     NOMINAL_BF16)},
+            "cpu_baseline": cpu, "e2e": e2e,
+            "gpu_launches": K * npass,
+            "clocks": clk,
+        }
+        print(json.dumps(line), flush=True)
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+    return 0
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,126 @@
+/*
+ * tcu_dft.h -- C ABI of the GB300 (sm_103a) batched complex DFT.
+ *
+ * The operation (arXiv 1908.06649, Sec. 4.5): the DFT of an n-vector x is
+ * y = x^T W with the symmetric Fourier matrix W[r][c] = exp(-(2 pi i/n) r c).
+ * It is computed with the paper's Cooley-Tukey scheme for the (m, l)-TCU
+ * (Sec. 4.5, Theorem 7): with sqrt(m) = r and n = r^k, each of the k stages is
+ * one tall-left product of the (batch*n/r) x r data matrix with the r x r DFT
+ * matrix F_r (X^T W_sqrt(m)), followed by the element-wise twiddle multiply
+ * w_n^{rc} and the transposition that feeds the next stage.  A complex r x r
+ * product is done as real arithmetic (Sec. 4.5: four real products and two
+ * sums), here as one real (2r x 2r) block operand [[Re, Im], [-Im, Re]] on the
+ * tensor cores (tcgen05, kind::tf32, accumulating in tensor memory).
+ *
+ * Conventions
+ *   forward : y_k = sum_j x_j exp(-2 pi i j k / n), unscaled.
+ *   inverse : x_j = (1/n) sum_k y_k exp(+2 pi i j k / n) (the paper defines
+ *             only the forward transform; this is the numpy/torch
+ *             "backward" normalisation).
+ *   Output is in natural order.
+ *
+ * Data layout (all entry points): `batch` transforms of length n, stored
+ * contiguously, transform-major, as interleaved complex64 (float re, float
+ * im): element j of transform b is at ((float2*)ptr)[b*n + j].  Device
+ * pointers must be 16-byte aligned.
+ *
+ * Threading: plans are independent objects; one plan must not be executed
+ * concurrently on two streams (its scratch is shared).  tcu_dft_last_error()
+ * is thread-local.
+ */
+#ifndef TCU_DFT_H
+#define TCU_DFT_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct tcu_dft_plan_s *tcu_dft_plan_t;
+
+/* precision: number of TF32 products per complex MMA term.
+ *   TCU_DFT_TF32   -- one product, operands rounded to TF32 (~1e-3 rel. L2)
+ *   TCU_DFT_3XTF32 -- hi*hi + lo*hi + hi*lo split products (fp32-level) */
+enum { TCU_DFT_TF32 = 1, TCU_DFT_3XTF32 = 3 };
+
+/* direction = sign of the exponent */
+enum { TCU_DFT_FORWARD = -1, TCU_DFT_INVERSE = +1 };
+
+/* status codes */
+enum {
+  TCU_DFT_OK = 0,
+  TCU_DFT_ERR_INVALID = 1,     /* bad argument (null, size, alignment, overlap) */
+  TCU_DFT_ERR_UNSUPPORTED = 2, /* valid but not supported (radix, n not r^k, n too large) */
+  TCU_DFT_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed, or no sm_103 device */
+  TCU_DFT_ERR_OOM = 4,         /* device allocation failed */
+  TCU_DFT_ERR_TIMEOUT = 5      /* a device-side wait hit its iteration limit */
+};
+
+/* Build a plan for `batch` forward/inverse DFTs of length n with radix
+ * sqrt_m (the TCU side length sqrt(m) of Sec. 3; one of 8, 16, 32) and the
+ * given precision.  n must equal sqrt_m^k for some k >= 1 (Theorem 7 assumes
+ * all of n, n/sqrt(m), ... are integers).
+ * Allocates the device tables (F_r operand images, twiddles) and, when n
+ * needs two passes, a scratch buffer of batch*n complex64 values; uses the
+ * current CUDA device.  This is the only call that allocates.
+ * Returns NULL on error and sets tcu_dft_last_error():
+ *   ERR_INVALID (n < 1, batch < 1, precision not 1 or 3),
+ *   ERR_UNSUPPORTED (sqrt_m not in {8,16,32}, n not a power of sqrt_m, or
+ *   n beyond two on-chip passes), ERR_CUDA (no sm_103 device), ERR_OOM. */
+tcu_dft_plan_t tcu_dft_plan(int64_t n, int64_t batch, int32_t sqrt_m,
+                            int32_t precision);
+
+/* Forward transform: equivalent to tcu_dft_exec_dir(p, in, out,
+ * TCU_DFT_FORWARD, stream). */
+int tcu_dft_exec(tcu_dft_plan_t p, const void *in, void *out, void *stream);
+
+/* Run the plan on `stream` (a cudaStream_t; NULL = legacy default stream).
+ * in, out: device pointers to batch*n complex64 values (caller-owned,
+ * 16-byte aligned).  in == out (full overlap) is allowed; partial overlap is
+ * rejected with ERR_INVALID.  Asynchronous: no allocation and no host
+ * synchronisation.  On an argument error nothing is launched.  Returns OK,
+ * ERR_INVALID, or ERR_CUDA if a launch failed. */
+int tcu_dft_exec_dir(tcu_dft_plan_t p, const void *in, void *out, int dir,
+                     void *stream);
+
+/* Same as tcu_dft_exec_dir, and records `events[i]` (cudaEvent_t handles,
+ * caller-created) on `stream` just before pass i and events[npasses] after
+ * the last pass, so the caller can time each pass kernel on the stream it
+ * runs on.  `events` must hold tcu_dft_num_passes(p) + 1 entries. */
+int tcu_dft_exec_timed(tcu_dft_plan_t p, const void *in, void *out, int dir,
+                       void *stream, void *const *events);
+
+/* End-to-end variant for host data: copies h_in (host, batch*n complex64;
+ * pinned memory makes the copy asynchronous) into the caller-owned device
+ * buffer d_work (batch*n complex64, 16-byte aligned), transforms it in place,
+ * and copies the result to h_out (host).  All on `stream`; the call returns
+ * after enqueuing (synchronise the stream before reading h_out).  Returns
+ * OK, ERR_INVALID or ERR_CUDA. */
+int tcu_dft_exec_host(tcu_dft_plan_t p, const void *h_in, void *h_out,
+                      void *d_work, int dir, void *stream);
+
+/* Synchronise `stream` and report whether any device-side wait of this
+ * plan's kernels gave up (ERR_TIMEOUT), then clear the flag.  OK otherwise;
+ * ERR_CUDA if the synchronisation itself failed. */
+int tcu_dft_check(tcu_dft_plan_t p, void *stream);
+
+/* Free the plan's device memory (cudaFree synchronises the device).
+ * Destroying NULL is a no-op returning OK. */
+int tcu_dft_destroy(tcu_dft_plan_t p);
+
+/* Plan introspection: number of HBM passes, and stages in pass i (0-based);
+ * -1 for a NULL plan or an index out of range. */
+int tcu_dft_num_passes(tcu_dft_plan_t p);
+int tcu_dft_pass_stages(tcu_dft_plan_t p, int i);
+
+/* Status of the last tcu_dft_plan call on this thread. */
+int tcu_dft_last_error(void);
+
+/* Static, human-readable name of a status code. */
+const char *tcu_dft_strerror(int status);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* TCU_DFT_H */

@@ -1,0 +1,208 @@
+"""Python binding of the GB300 batched complex DFT (C ABI in include/tcu_dft.h).
+
+Argument marshalling only: every step of the transform runs in the CUDA
+library ``libtcu_dft.so`` built from ``csrc/tcu_dft.cu``.  There is no CPU or
+PyTorch fallback: if the library is missing this module raises on import of
+the library (``lib()``), and a transform on a machine without the library
+fails loudly.
+
+The transform is the paper's (arXiv 1908.06649, Sec. 4.5): y = x^T W,
+W[r][c] = exp(-(2 pi i/n) r c), computed as n = r^k radix-r stages, each a
+tall-left tensor-core product with F_r (Theorem 7).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+from . import _build
+
+TF32 = 1
+X3TF32 = 3
+FORWARD = -1
+INVERSE = 1
+
+OK = 0
+ERR_INVALID = 1
+ERR_UNSUPPORTED = 2
+ERR_CUDA = 3
+ERR_OOM = 4
+ERR_TIMEOUT = 5
+
+SYMBOLS = (
+    "tcu_dft_plan", "tcu_dft_exec", "tcu_dft_exec_dir", "tcu_dft_exec_timed",
+    "tcu_dft_exec_host",
+    "tcu_dft_check", "tcu_dft_destroy", "tcu_dft_num_passes",
+    "tcu_dft_pass_stages", "tcu_dft_last_error", "tcu_dft_strerror",
+)
+
+_lib = None
+
+
+class TcuDftError(RuntimeError):
+    def __init__(self, status, what):
+        self.status = status
+        super().__init__("%s: %s (status %d)" % (what, strerror(status), status))
+
+
+def lib_path() -> str:
+    return _build.LIB_PATH
+
+
+def lib():
+    """Load libtcu_dft.so (built in-tree by ``_build.build()``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    path = _build.LIB_PATH
+    if not os.path.exists(path):
+        raise ImportError(
+            "libtcu_dft.so is not built (%s); run "
+            "paper_1908_06649_gb300._build.build() first" % path)
+    L = ctypes.CDLL(path)
+    vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
+    L.tcu_dft_plan.argtypes = [i64, i64, i32, i32]
+    L.tcu_dft_plan.restype = vp
+    L.tcu_dft_exec.argtypes = [vp, vp, vp, vp]
+    L.tcu_dft_exec.restype = ctypes.c_int
+    L.tcu_dft_exec_dir.argtypes = [vp, vp, vp, ctypes.c_int, vp]
+    L.tcu_dft_exec_dir.restype = ctypes.c_int
+    L.tcu_dft_exec_timed.argtypes = [vp, vp, vp, ctypes.c_int, vp,
+                                     ctypes.POINTER(vp)]
+    L.tcu_dft_exec_timed.restype = ctypes.c_int
+    L.tcu_dft_exec_host.argtypes = [vp, vp, vp, vp, ctypes.c_int, vp]
+    L.tcu_dft_exec_host.restype = ctypes.c_int
+    L.tcu_dft_check.argtypes = [vp, vp]
+    L.tcu_dft_check.restype = ctypes.c_int
+    L.tcu_dft_destroy.argtypes = [vp]
+    L.tcu_dft_destroy.restype = ctypes.c_int
+    L.tcu_dft_num_passes.argtypes = [vp]
+    L.tcu_dft_num_passes.restype = ctypes.c_int
+    L.tcu_dft_pass_stages.argtypes = [vp, ctypes.c_int]
+    L.tcu_dft_pass_stages.restype = ctypes.c_int
+    L.tcu_dft_last_error.argtypes = []
+    L.tcu_dft_last_error.restype = ctypes.c_int
+    L.tcu_dft_strerror.argtypes = [ctypes.c_int]
+    L.tcu_dft_strerror.restype = ctypes.c_char_p
+    _lib = L
+    return L
+
+
+def strerror(status: int) -> str:
+    try:
+        return lib().tcu_dft_strerror(int(status)).decode()
+    except ImportError:
+        return "status %d" % status
+
+
+def _stream_handle(stream):
+    import torch
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+class Plan:
+    """tcu_dft_plan(n, batch, sqrt_m, precision) and its executions.
+
+    ``forward(x)`` / ``inverse(x)`` take a contiguous complex64 CUDA tensor of
+    shape (batch, n) (or batch*n elements) and return the transform in a new
+    tensor (or in ``out``).  They run on torch's current stream.
+    """
+
+    def __init__(self, n: int, batch: int, sqrt_m: int = 16,
+                 precision: int = X3TF32):
+        L = lib()
+        h = L.tcu_dft_plan(int(n), int(batch), int(sqrt_m), int(precision))
+        if not h:
+            raise TcuDftError(L.tcu_dft_last_error(), "tcu_dft_plan")
+        self._h = h
+        self.n, self.batch, self.sqrt_m, self.precision = (
+            int(n), int(batch), int(sqrt_m), int(precision))
+
+    @property
+    def handle(self):
+        return self._h
+
+    def passes(self):
+        L = lib()
+        return [L.tcu_dft_pass_stages(self._h, i)
+                for i in range(L.tcu_dft_num_passes(self._h))]
+
+    def _check_tensor(self, t, name):
+        import torch
+        if not isinstance(t, torch.Tensor) or t.dtype != torch.complex64:
+            raise TypeError("%s must be a complex64 torch tensor" % name)
+        if not t.is_cuda or not t.is_contiguous():
+            raise ValueError("%s must be a contiguous CUDA tensor" % name)
+        if t.numel() != self.n * self.batch:
+            raise ValueError("%s must hold batch*n = %d elements"
+                             % (name, self.n * self.batch))
+
+    def exec(self, x, out=None, direction: int = FORWARD, stream=None):
+        import torch
+        self._check_tensor(x, "x")
+        if out is None:
+            out = torch.empty_like(x)
+        self._check_tensor(out, "out")
+        rc = lib().tcu_dft_exec_dir(self._h, ctypes.c_void_p(x.data_ptr()),
+                                    ctypes.c_void_p(out.data_ptr()),
+                                    int(direction), _stream_handle(stream))
+        if rc != OK:
+            raise TcuDftError(rc, "tcu_dft_exec_dir")
+        return out
+
+    def exec_timed(self, x, out, events, direction: int = FORWARD,
+                   stream=None):
+        """exec() that records torch.cuda.Event objects ``events`` (one per
+        pass plus one) around the pass kernels on the stream."""
+        self._check_tensor(x, "x")
+        self._check_tensor(out, "out")
+        arr = (ctypes.c_void_p * len(events))(
+            *[ctypes.c_void_p(e.cuda_event) for e in events])
+        rc = lib().tcu_dft_exec_timed(self._h, ctypes.c_void_p(x.data_ptr()),
+                                      ctypes.c_void_p(out.data_ptr()),
+                                      int(direction), _stream_handle(stream),
+                                      arr)
+        if rc != OK:
+            raise TcuDftError(rc, "tcu_dft_exec_timed")
+        return out
+
+    def forward(self, x, out=None, stream=None):
+        return self.exec(x, out, FORWARD, stream)
+
+    def inverse(self, x, out=None, stream=None):
+        return self.exec(x, out, INVERSE, stream)
+
+    def exec_host(self, h_in, h_out, d_work, direction: int = FORWARD,
+                  stream=None):
+        """Host in -> device work buffer -> host out, all enqueued on the
+        stream (synchronise before reading h_out)."""
+        self._check_tensor(d_work, "d_work")
+        for t, nm in ((h_in, "h_in"), (h_out, "h_out")):
+            if t.is_cuda or t.numel() != self.n * self.batch:
+                raise ValueError("%s must be a host tensor of batch*n" % nm)
+        rc = lib().tcu_dft_exec_host(
+            self._h, ctypes.c_void_p(h_in.data_ptr()),
+            ctypes.c_void_p(h_out.data_ptr()),
+            ctypes.c_void_p(d_work.data_ptr()), int(direction),
+            _stream_handle(stream))
+        if rc != OK:
+            raise TcuDftError(rc, "tcu_dft_exec_host")
+
+    def check(self, stream=None):
+        """Synchronise and raise if a device-side wait timed out."""
+        rc = lib().tcu_dft_check(self._h, _stream_handle(stream))
+        if rc != OK:
+            raise TcuDftError(rc, "tcu_dft_check")
+
+    def destroy(self):
+        if getattr(self, "_h", None):
+            lib().tcu_dft_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass

@@ -1,0 +1,93 @@
+"""The C ABI on the CPU: the library builds, loads, exports every symbol that
+include/tcu_dft.h declares, and rejects bad arguments before touching CUDA."""
+import ctypes
+import os
+import re
+import subprocess
+
+import pytest
+
+from paper_1908_06649_gb300 import _build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "tcu_dft.h")
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(tcu_dft_[a-z_]+)\s*\(", src)))
+
+
+@pytest.fixture(scope="module")
+def lib():
+    _build.build()
+    import paper_1908_06649_gb300 as pkg
+    return pkg.lib()
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("tcu_dft_plan", "tcu_dft_exec", "tcu_dft_exec_dir",
+                     "tcu_dft_destroy", "tcu_dft_last_error",
+                     "tcu_dft_strerror"):
+        assert required in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    out = subprocess.run(["nm", "-D", "--defined-only", _build.LIB_PATH],
+                         capture_output=True, text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (\w+)", out))
+    for name in declared_functions():
+        assert name in exported, name
+        assert getattr(lib, name) is not None
+
+
+def test_binding_lists_every_symbol():
+    import paper_1908_06649_gb300 as pkg
+    assert sorted(pkg.SYMBOLS) == declared_functions()
+
+
+def test_strerror_and_null_handling(lib):
+    import paper_1908_06649_gb300 as pkg
+    assert lib.tcu_dft_strerror(0) == b"ok"
+    assert lib.tcu_dft_strerror(pkg.ERR_TIMEOUT) == b"device wait timed out"
+    assert lib.tcu_dft_destroy(None) == pkg.OK
+    assert lib.tcu_dft_exec(None, None, None, None) == pkg.ERR_INVALID
+    assert lib.tcu_dft_exec_dir(None, None, None, -1, None) == pkg.ERR_INVALID
+    assert lib.tcu_dft_exec_host(None, None, None, None, -1, None) == pkg.ERR_INVALID
+    assert lib.tcu_dft_check(None, None) == pkg.ERR_INVALID
+    assert lib.tcu_dft_num_passes(None) == -1
+    assert lib.tcu_dft_pass_stages(None, 0) == -1
+
+
+@pytest.mark.parametrize("n,batch,r,prec,status", [
+    (0, 1, 16, 3, 1),        # n < 1
+    (16, 0, 16, 3, 1),       # batch < 1
+    (16, 1, 16, 2, 1),       # precision not 1 or 3
+    (16, 1, 4, 3, 2),        # radix not in {8, 16, 32}
+    (16, 1, 64, 3, 2),
+    (48, 1, 16, 3, 2),       # not a power of the radix
+    (128, 1, 16, 3, 2),      # power of two but not of 16
+    (16 ** 7, 1, 16, 3, 2),  # beyond two on-chip passes
+    (32 ** 5, 1, 32, 3, 2),
+])
+def test_plan_rejects_before_cuda(lib, n, batch, r, prec, status):
+    h = lib.tcu_dft_plan(n, batch, r, prec)
+    assert not h
+    assert lib.tcu_dft_last_error() == status
+
+
+def test_plan_without_gpu_reports_cuda_error(lib):
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    assert not lib.tcu_dft_plan(256, 4, 16, 3)
+    assert lib.tcu_dft_last_error() == 3
+
+
+def test_python_plan_raises(lib):
+    import paper_1908_06649_gb300 as pkg
+    with pytest.raises(pkg.TcuDftError) as e:
+        pkg.Plan(48, 1, 16)
+    assert e.value.status == pkg.ERR_UNSUPPORTED
