@@ -217,10 +217,14 @@ def main():
     ap.add_argument("--ref-sample", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=20)
+    ap.add_argument("--batch", type=int, default=0,
+                    help="override the workload's batch (profiling cases)")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
     wl = dict(inputs.WORKLOADS[args.workload])
+    if args.batch > 0:
+        wl["batch"] = args.batch
     if args.impl == "reference":
         return run_reference(args, wl)
 

@@ -463,14 +463,368 @@ __global__ void __launch_bounds__(kThreads, 1) dft_pass_kernel(const PassArgs a)
   }
 }
 
+// ------------------------------------------------------------ group kernel
+// Persistent kernel for passes of L = r^S <= 128 r points per sub-transform.
+// A CTA holds NWG independent warpgroups.  A warpgroup owns one TMEM slot
+// (A_hi | A_lo | D for 128 rows), one SMEM transpose buffer and one mbarrier,
+// and walks a strided list of work items; an item is GG = 128 r / L
+// consecutive sub-transforms, i.e. exactly 128 data rows per stage, so every
+// stage of an item is one M=128 tcgen05 product and the transposes between
+// stages stay inside the warpgroup.  Stage-1 rows are loaded from global
+// memory straight into registers (the row-to-lane map makes the loads
+// coalesced), the next item's rows are prefetched while the current item's
+// products run, and the last stage's rows are stored straight from registers.
+
+enum RowMode { kQF = 0, kUF = 1, kRQF = 2 };
+
+struct GroupArgs {
+  const float2 *in;
+  float2 *out;
+  const float *bimg;   // hi | lo B images of F_r for this direction
+  const float2 *twL;   // w_L^e, e in [0, L)
+  const float2 *twA;   // inter-pass twiddle, high part: w_N^{i 2^h}
+  const float2 *twB;   // inter-pass twiddle, low part:  w_N^{j}
+  int *err;
+  long long U;         // sub-transforms in the pass
+  long long n;         // transform length
+  long long in_vstride, in_stride, out_vstride, out_stride;
+  int log2Uper;        // log2(sub-transforms per transform)
+  int tw_log2N;        // inter-pass twiddle period log2 (0: none)
+  int tw_h;            // low-part bits of the two-level twiddle
+  int mode_first, mode_mid, mode_last;  // RowMode of the first/middle/last stage
+  unsigned long long swz_tab;           // 16 nibbles: SMEM swizzle per (ul & 15)
+  float scale;         // output scale (1 or 1/n)
+};
+
+template <int R, int S>
+struct GCfg {
+  static constexpr int LOG2R = (R == 8) ? 3 : (R == 16) ? 4 : 5;
+  static constexpr int NWG = (R == 32) ? 2 : 4;
+  static constexpr int THREADS = 128 * NWG;
+  static constexpr int GPTS = 128 * R;               // points per item
+  static constexpr int LOG2GPTS = 7 + LOG2R;
+  static constexpr int LOG2L = LOG2R * S;
+  static constexpr int L = 1 << LOG2L;
+  static constexpr int LOG2RPS = LOG2L - LOG2R;      // rows per sub-transform
+  static constexpr int LOG2GG = LOG2GPTS - LOG2L;    // sub-transforms per item
+  static constexpr int GG = 1 << LOG2GG;
+  static constexpr int Q = (2 * R > 32) ? 2 * R : 32;
+  static constexpr int GCOLS = 3 * Q;
+  static constexpr int IMG_BYTES = 16 * R * R;
+  static constexpr int LBO = 128, SBO = 64 * R, KSTEPS = 2 * R / 8;
+  static constexpr size_t OFF_TW = 2 * IMG_BYTES;
+  static constexpr size_t OFF_BUF = OFF_TW + (size_t)L * 8;
+  static constexpr size_t OFF_BAR =
+      OFF_BUF + (S > 1 ? (size_t)NWG * GPTS * 8 : 0);
+  static constexpr size_t SMEM_BYTES = OFF_BAR + 8 * NWG + 16;
+  static_assert(LOG2GG >= 0, "sub-transform longer than one item");
+  static_assert(NWG * GCOLS <= 512, "TMEM budget");
+};
+
+// bar.sync on a named barrier that also ORs a predicate across the threads
+__device__ __forceinline__ bool named_bar_or(int id, int count, bool v) {
+  uint32_t out;
+  asm volatile(
+      "{\n\t.reg .pred p, q;\n\t"
+      "setp.ne.u32 q, %1, 0;\n\t"
+      "bar.red.or.pred p, %2, %3, q;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(out)
+      : "r"((uint32_t)v), "r"(id), "r"(count)
+      : "memory");
+  return out != 0;
+}
+
+template <int R, int S>
+__device__ __forceinline__ void row_of(int mode, int rho, int &ul, int &q) {
+  using C = GCfg<R, S>;
+  if (mode == kUF) {
+    ul = rho & (C::GG - 1);
+    q = rho >> C::LOG2GG;
+  } else {
+    ul = rho >> C::LOG2RPS;
+    q = rho & ((1 << C::LOG2RPS) - 1);
+    if (mode == kRQF) {  // digit-reversed q over S-1 digits
+      int rq = 0, v = q;
+#pragma unroll
+      for (int i = 0; i < S - 1; ++i) {
+        rq = (rq << C::LOG2R) | (v & (R - 1));
+        v >>= C::LOG2R;
+      }
+      q = rq;
+    }
+  }
+}
+
+__device__ __forceinline__ int gswz(int p, uint32_t tabv) {
+  return p ^ (int)((tabv ^ (uint32_t)(p >> 4)) & 15u);
+}
+
+// Split a complex row into TF32 hi / lo parts and store them as the A
+// operand rows of this thread's TMEM lane.
+template <int R, int PREC>
+__device__ __forceinline__ void split_store(const float2 *x, uint32_t col_hi,
+                                            uint32_t col_lo) {
+#pragma unroll
+  for (int c = 0; c < R; c += 8) {
+    float vh[16], vl[16];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const float hx = tf32_rna(x[c + j].x), hy = tf32_rna(x[c + j].y);
+      vh[2 * j] = hx;
+      vh[2 * j + 1] = hy;
+      if (PREC == 3) {
+        vl[2 * j] = tf32_rna(x[c + j].x - hx);
+        vl[2 * j + 1] = tf32_rna(x[c + j].y - hy);
+      }
+    }
+    tmem_st16(col_hi + 2 * c, vh);
+    if (PREC == 3) tmem_st16(col_lo + 2 * c, vl);
+  }
+}
+
+template <int R, int PREC>
+__device__ __forceinline__ void issue_stage_mma(uint32_t slot, uint32_t img_addr) {
+  constexpr int Q = (2 * R > 32) ? 2 * R : 32;
+  constexpr int IMG = 16 * R * R, LBO = 128, SBO = 64 * R, KSTEPS = 2 * R / 8;
+  constexpr uint32_t idesc = idesc_tf32(128, 2 * R);
+  const uint32_t ahi = slot, alo = slot + Q, d = slot + 2 * Q;
+  const uint32_t ihi = img_addr, ilo = img_addr + IMG;
+  uint32_t acc = 0;
+  if (PREC == 3) {
+#pragma unroll
+    for (int kk = 0; kk < KSTEPS; ++kk) {
+      mma_tf32_ts(d, alo + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO),
+                  idesc, acc);
+      acc = 1;
+    }
+#pragma unroll
+    for (int kk = 0; kk < KSTEPS; ++kk)
+      mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(ilo + kk * 2 * LBO, LBO, SBO),
+                  idesc, 1);
+  }
+#pragma unroll
+  for (int kk = 0; kk < KSTEPS; ++kk) {
+    mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO),
+                idesc, acc);
+    acc = 1;
+  }
+}
+
+template <int R, int S>
+__device__ __forceinline__ void load_row(const GroupArgs &a, long long item,
+                                         long long nitems, int ul, int q,
+                                         float2 *x) {
+  using C = GCfg<R, S>;
+  const long long u = (item << C::LOG2GG) + ul;
+  if (item < nitems && u < a.U) {
+    const long long beta = u >> a.log2Uper;
+    const long long vv = u & ((1ll << a.log2Uper) - 1);
+    const float2 *src = a.in + beta * a.n + vv * a.in_vstride + (long long)q * a.in_stride;
+    const long long js = a.in_stride << (C::LOG2R * (S - 1));
+#pragma unroll
+    for (int j = 0; j < R; ++j) x[j] = __ldg(src + j * js);
+  } else {
+#pragma unroll
+    for (int j = 0; j < R; ++j) x[j] = make_float2(0.f, 0.f);
+  }
+}
+
+template <int R, int PREC, int S>
+__global__ void __launch_bounds__(GCfg<R, S>::THREADS, 1)
+    dft_group_kernel(const GroupArgs a) {
+  using C = GCfg<R, S>;
+  constexpr int LOG2R = C::LOG2R;
+  extern __shared__ __align__(1024) unsigned char smem[];
+  float *img = reinterpret_cast<float *>(smem);
+  float2 *tw = reinterpret_cast<float2 *>(smem + C::OFF_TW);
+  uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + C::OFF_BAR);
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + C::NWG);
+
+  const int tid = threadIdx.x;
+  const int warp = tid >> 5, lane = tid & 31;
+  const int wg = warp >> 2, wq = warp & 3;
+  const int rho = wq * 32 + lane;
+  float2 *buf = reinterpret_cast<float2 *>(smem + C::OFF_BUF) + wg * C::GPTS;
+
+  // ---- set-up
+  {
+    const float4 *src = reinterpret_cast<const float4 *>(a.bimg);
+    float4 *dst = reinterpret_cast<float4 *>(img);
+    const int n4 = (PREC == 3 ? 2 : 1) * C::IMG_BYTES / 16;
+    for (int i = tid; i < n4; i += C::THREADS) dst[i] = __ldg(src + i);
+    if (S > 1)
+      for (int i = tid; i < C::L; i += C::THREADS) tw[i] = __ldg(a.twL + i);
+  }
+  if (tid == 0) {
+    for (int w = 0; w < C::NWG; ++w) mbar_init(smem_u32(mbar + w), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  if (warp == 0) tmem_alloc(smem_u32(tmem_slot), 512);
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tbase = *tmem_slot;
+  const uint32_t slot = tbase + wg * C::GCOLS;
+  const uint32_t lane_off = (uint32_t)(wq * 32) << 16;
+  const uint32_t img_addr = smem_u32(img);
+  const uint32_t bar_addr = smem_u32(mbar + wg);
+  const int bar_id = 1 + wg;
+
+  const long long nitems = (a.U + C::GG - 1) >> C::LOG2GG;
+  const long long istride = (long long)gridDim.x * C::NWG;
+  long long item = (long long)blockIdx.x * C::NWG + wg;
+  uint32_t phase = 0;
+  bool fail = false;
+
+  int ul1, q1;
+  row_of<R, S>(a.mode_first, rho, ul1, q1);
+  float2 x[R];
+  load_row<R, S>(a, item, nitems, ul1, q1, x);
+
+  while (item < nitems) {
+    // ---- stage 1 operand
+    split_store<R, PREC>(x, slot + lane_off, slot + C::Q + lane_off);
+    tmem_wait_st();
+    fence_before_sync();
+    if (named_bar_or(bar_id, 128, fail)) break;
+    if (rho == 0) {
+      fence_after_sync();
+      issue_stage_mma<R, PREC>(slot, img_addr);
+      mma_commit(bar_addr);
+    }
+    const long long next = item + istride;
+    load_row<R, S>(a, next, nitems, ul1, q1, x);  // prefetch
+    if (!mbar_wait_bounded(bar_addr, phase)) fail = true;
+    phase ^= 1;
+    fence_after_sync();
+
+#pragma unroll 1
+    for (int t = 1; t <= S; ++t) {
+      if (t < S) {
+        // epilogue of stage t, 8 outputs at a time: TMEM -> registers,
+        // twiddle w_{L_t}^{k_t c_t} = w_L^{k_t * lo * r^(t-1)}, transposed
+        // write to the SMEM buffer
+        const int mode = (t == 1) ? a.mode_first : a.mode_mid;
+        int ul, q;
+        row_of<R, S>(mode, rho, ul, q);
+        const int shift_lo = LOG2R * (S - t);
+        const int hi = q >> shift_lo, lo = q & ((1 << shift_lo) - 1);
+        const int base = (ul << C::LOG2L) + (hi << (shift_lo + LOG2R)) + lo;
+        const uint32_t tabv = (uint32_t)(a.swz_tab >> (4 * (ul & 15))) & 15u;
+        const int estep = lo << (LOG2R * (t - 1));
+#pragma unroll
+        for (int c = 0; c < R; c += 8) {
+          float d[16];
+          tmem_ld16(slot + 2 * C::Q + lane_off + 2 * c, d);
+#pragma unroll
+          for (int jj = 0; jj < 8; ++jj) {
+            const int j = c + jj;
+            const float2 y = cmul(make_float2(d[2 * jj], d[2 * jj + 1]),
+                                  tw[(j * estep) & (C::L - 1)]);
+            buf[gswz(base + (j << shift_lo), tabv)] = y;
+          }
+        }
+        fence_before_sync();
+        named_bar_or(bar_id, 128, false);
+        // rows of stage t+1, 8 elements at a time: SMEM -> split -> TMEM
+        const int mode2 = (t + 1 == S) ? a.mode_last : a.mode_mid;
+        row_of<R, S>(mode2, rho, ul, q);
+        const int shift2 = LOG2R * (S - t - 1);
+        const int hi2 = q >> shift2, lo2 = q & ((1 << shift2) - 1);
+        const int base2 = (ul << C::LOG2L) + (hi2 << (shift2 + LOG2R)) + lo2;
+        const uint32_t tabv2 = (uint32_t)(a.swz_tab >> (4 * (ul & 15))) & 15u;
+#pragma unroll
+        for (int c = 0; c < R; c += 8) {
+          float2 row[8];
+#pragma unroll
+          for (int jj = 0; jj < 8; ++jj)
+            row[jj] = buf[gswz(base2 + ((c + jj) << shift2), tabv2)];
+          split_store<8, PREC>(row, slot + lane_off + 2 * c, slot + C::Q + lane_off + 2 * c);
+        }
+        tmem_wait_st();
+        fence_before_sync();
+        if (named_bar_or(bar_id, 128, fail)) {
+          fail = true;
+          break;
+        }
+        if (rho == 0) {
+          fence_after_sync();
+          issue_stage_mma<R, PREC>(slot, img_addr);
+          mma_commit(bar_addr);
+        }
+        if (!mbar_wait_bounded(bar_addr, phase)) fail = true;
+        phase ^= 1;
+        fence_after_sync();
+      } else {
+        // last stage: natural-order output straight from registers
+        float d[2 * R];
+#pragma unroll
+        for (int c = 0; c < 2 * R; c += 16) tmem_ld16(slot + 2 * C::Q + lane_off + c, d + c);
+        int ul, q;
+        row_of<R, S>(a.mode_last, rho, ul, q);
+        const long long u = (item << C::LOG2GG) + ul;
+        if (u < a.U) {
+          int klow = 0, v = q;
+#pragma unroll
+          for (int i = 0; i < S - 1; ++i) {
+            klow = (klow << LOG2R) | (v & (R - 1));
+            v >>= LOG2R;
+          }
+          const long long beta = u >> a.log2Uper;
+          const long long vv = u & ((1ll << a.log2Uper) - 1);
+          float2 *dst = a.out + beta * a.n + vv * a.out_vstride + klow * a.out_stride;
+          const long long jstep = a.out_stride << (LOG2R * (S - 1));
+          // twiddle exponent (vv * k) mod 2^tw_log2N, tw_log2N <= 32: exact in
+          // wrap-around 32-bit arithmetic
+          const uint32_t Nmask = (uint32_t)((1ull << a.tw_log2N) - 1);
+          const uint32_t hmask = (1u << a.tw_h) - 1;
+          const uint32_t e0 = (uint32_t)vv * (uint32_t)klow;
+          const uint32_t estep = (uint32_t)vv << (LOG2R * (S - 1));
+#pragma unroll
+          for (int j = 0; j < R; ++j) {
+            float2 y = make_float2(d[2 * j], d[2 * j + 1]);
+            if (a.tw_log2N) {
+              const uint32_t e = (e0 + (uint32_t)j * estep) & Nmask;
+              y = cmul(y, cmul(__ldg(a.twA + (e >> a.tw_h)), __ldg(a.twB + (e & hmask))));
+            }
+            y.x *= a.scale;
+            y.y *= a.scale;
+            dst[j * jstep] = y;
+          }
+        }
+      }
+    }
+    // a failed wait is acted on at the next barrier, where the flag is
+    // reduced over the warpgroup so that every thread leaves together
+    item = next;
+  }
+  if (fail && rho == 0) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);
+
+  // ---- teardown
+  fence_before_sync();
+  __syncthreads();
+  if (warp == 0) {
+    fence_after_sync();
+    tmem_dealloc(tbase, 512);
+  }
+}
+
 // ------------------------------------------------------------------ host side
+enum PassKind { kTilePass = 0, kGroupPass = 1 };
+
 struct PassPlan {
+  int kind;        // kTilePass or kGroupPass
   int s;
   int log2L;
-  int log2G;
+  int log2G;       // tile kernel: sub-transforms per tile
   long long U, Uper;
+  int log2Uper;
   long long in_vstride, in_stride, out_vstride, out_stride;
   int tw_log2N, tw_h;
+  int modes[3];    // group kernel: row map of first / middle / last stage
+  unsigned long long swz_tab;
   bool last;
   float2 *twL[2];  // [dir index] w_L^e
 };
@@ -489,6 +843,7 @@ struct tcu_dft_plan_s {
   long long n, batch;
   int r, log2r, k, precision;
   int npasses;
+  int num_sms;
   PassPlan pass[2];
   float *bimg[2];      // [dir index] hi | lo images
   float2 *twA[2], *twB[2];
@@ -552,7 +907,94 @@ std::vector<float2> twiddle_table(long long period, long long count, long long s
   return t;
 }
 
-int max_stages(int r) { return r == 8 ? 4 : (r == 16 ? 3 : 2); }
+// Largest stage count per pass: tile kernel (a sub-transform fills at most one
+// SMEM tile) and group kernel (a sub-transform fits 128 rows).
+int max_tile_stages(int r) { return r == 8 ? 4 : (r == 16 ? 3 : 2); }
+int max_group_stages(int r) { return r == 8 ? 3 : 2; }
+
+int stage_mode(const int modes[3], int t, int S) {
+  return t == 1 ? modes[0] : (t == S ? modes[2] : modes[1]);
+}
+
+// Shared-memory wavefronts per warp-wide 8-byte access of the group kernel's
+// transposes (1.0 = conflict free), for swizzle table `tab`:
+// phys(P) = P ^ ((tab[ul & 15] ^ (P >> 4)) & 15).
+double swizzle_cost(int r, int S, const int modes[3], unsigned long long tab) {
+  const int log2r = ilog2(r);
+  const int L = 1 << (log2r * S);
+  const int rps = L / r, gg = 128 * r / L;
+  long long waves = 0, accesses = 0;
+  for (int t = 1; t < S; ++t) {
+    for (int side = 0; side < 2; ++side) {  // epilogue write of t, read of t+1
+      const int tt = t + side;
+      const int mode = stage_mode(modes, tt, S);
+      const int sl = log2r * (S - tt);
+      for (int w = 0; w < 4; ++w)
+        for (int j = 0; j < r; ++j)
+          for (int h = 0; h < 2; ++h) {
+            int seen = 0;  // bitmask of the 16 eight-byte bank slots
+            int count = 0;
+            for (int l = 16 * h; l < 16 * h + 16; ++l) {
+              const int rho = 32 * w + l;
+              int ul, q;
+              if (mode == kUF) {
+                ul = rho % gg;
+                q = rho / gg;
+              } else {
+                ul = rho / rps;
+                q = rho % rps;
+                if (mode == kRQF) {
+                  int rq = 0, v = q;
+                  for (int i = 0; i < S - 1; ++i) {
+                    rq = rq * r + v % r;
+                    v /= r;
+                  }
+                  q = rq;
+                }
+              }
+              const int hi = q >> sl, lo = q & ((1 << sl) - 1);
+              const int P = ul * L + (hi << (sl + log2r)) + (j << sl) + lo;
+              const unsigned tv = (unsigned)(tab >> (4 * (ul & 15))) & 15u;
+              const int ph = P ^ (int)((tv ^ (unsigned)(P >> 4)) & 15u);
+              const int slot = ph & 15;
+              if (!(seen & (1 << slot))) {
+                seen |= 1 << slot;
+                ++count;
+              }
+            }
+            waves += (16 + count - 1) / count;
+            ++accesses;
+          }
+    }
+  }
+  return accesses ? (double)waves / (double)accesses : 1.0;
+}
+
+unsigned long long choose_swizzle(int r, int S, const int modes[3]) {
+  std::vector<unsigned long long> cands;
+  for (int c = 0; c < 4; ++c) {
+    unsigned long long t = 0;
+    for (int u = 0; u < 16; ++u) t |= (unsigned long long)((u << c) & 15) << (4 * u);
+    cands.push_back(t);
+  }
+  for (int c = 1; c < 4; ++c) {
+    unsigned long long t = 0;
+    for (int u = 0; u < 16; ++u) t |= (unsigned long long)((u ^ (u << c)) & 15) << (4 * u);
+    cands.push_back(t);
+  }
+  cands.push_back(0ull);
+  cands.push_back(0x7fe70d6c0000a378ull);  // found by an offline search
+  unsigned long long best = cands[0];
+  double bc = 1e30;
+  for (unsigned long long t : cands) {
+    const double c = swizzle_cost(r, S, modes, t);
+    if (c < bc - 1e-9) {
+      bc = c;
+      best = t;
+    }
+  }
+  return best;
+}
 
 template <typename T>
 int upload(T **dst, const std::vector<T> &src) {
@@ -606,6 +1048,43 @@ cudaError_t launch_dispatch(int r, int prec, const PassArgs &a, long long grid,
   return prec == 3 ? launch_pass<32, 3>(a, grid, st) : launch_pass<32, 1>(a, grid, st);
 }
 
+template <int R, int PREC, int S>
+cudaError_t launch_group(const GroupArgs &a, int num_sms, cudaStream_t st) {
+  using C = GCfg<R, S>;
+  const size_t sm = C::SMEM_BYTES;
+  cudaError_t e = cudaFuncSetAttribute(dft_group_kernel<R, PREC, S>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)sm);
+  if (e != cudaSuccess) return e;
+  const long long nitems = (a.U + C::GG - 1) >> C::LOG2GG;
+  long long grid = (nitems + C::NWG - 1) / C::NWG;
+  if (grid > num_sms) grid = num_sms;
+  dft_group_kernel<R, PREC, S><<<(unsigned)grid, C::THREADS, sm, st>>>(a);
+  return cudaGetLastError();
+}
+
+template <int R, int PREC>
+cudaError_t launch_group_s(int s, const GroupArgs &a, int num_sms, cudaStream_t st) {
+  if (s == 1) return launch_group<R, PREC, 1>(a, num_sms, st);
+  if (s == 2) return launch_group<R, PREC, 2>(a, num_sms, st);
+  if constexpr (R == 8) {
+    if (s == 3) return launch_group<R, PREC, 3>(a, num_sms, st);
+  }
+  return cudaErrorInvalidValue;
+}
+
+cudaError_t launch_group_dispatch(int r, int prec, int s, const GroupArgs &a,
+                                  int num_sms, cudaStream_t st) {
+  if (r == 8)
+    return prec == 3 ? launch_group_s<8, 3>(s, a, num_sms, st)
+                     : launch_group_s<8, 1>(s, a, num_sms, st);
+  if (r == 16)
+    return prec == 3 ? launch_group_s<16, 3>(s, a, num_sms, st)
+                     : launch_group_s<16, 1>(s, a, num_sms, st);
+  return prec == 3 ? launch_group_s<32, 3>(s, a, num_sms, st)
+                   : launch_group_s<32, 1>(s, a, num_sms, st);
+}
+
 int tile_points(int r) { return r == 8 ? 4096 : 8192; }
 
 bool overlaps(const void *a, const void *b, size_t bytes) {
@@ -653,15 +1132,27 @@ tcu_dft_plan_t tcu_dft_plan(int64_t n, int64_t batch, int32_t sqrt_m,
     g_last_error = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
   }
-  const int smax = max_stages(r);
-  int stages[2] = {0, 0}, npasses;
-  if (k <= smax) {
+  // Pass grouping: prefer the group kernel (sub-transforms of <= 128 rows),
+  // fall back to the tile kernel for longer sub-transforms.
+  const int sg = max_group_stages(r), stl = max_tile_stages(r);
+  int stages[2] = {0, 0}, kinds[2] = {kGroupPass, kGroupPass}, npasses;
+  if (k <= sg) {
     npasses = 1;
     stages[0] = k;
-  } else if (k <= 2 * smax) {
+  } else if (k <= 2 * sg) {
     npasses = 2;
     stages[0] = (k + 1) / 2;
     stages[1] = k - stages[0];
+  } else if (k <= stl + sg) {
+    npasses = 2;
+    stages[0] = k - sg;
+    kinds[0] = kTilePass;
+    stages[1] = sg;
+  } else if (k <= 2 * stl) {
+    npasses = 2;
+    stages[0] = (k + 1) / 2;
+    stages[1] = k - stages[0];
+    kinds[0] = kinds[1] = kTilePass;
   } else {
     g_last_error = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
@@ -690,10 +1181,12 @@ tcu_dft_plan_t tcu_dft_plan(int64_t n, int64_t batch, int32_t sqrt_m,
   p->precision = precision;
   p->npasses = npasses;
   p->device = dev;
+  p->num_sms = prop.multiProcessorCount;
   const int log2n = ilog2(n);
   int rc = TCU_DFT_OK;
   for (int pi = 0; pi < npasses && rc == TCU_DFT_OK; ++pi) {
     PassPlan &pp = p->pass[pi];
+    pp.kind = kinds[pi];
     pp.s = stages[pi];
     pp.log2L = log2r * pp.s;
     pp.log2G = ilog2(tile_points(r)) - pp.log2L;
@@ -727,6 +1220,11 @@ tcu_dft_plan_t tcu_dft_plan(int64_t n, int64_t batch, int32_t sqrt_m,
       pp.out_stride = n1;
       pp.tw_log2N = 0;
     }
+    pp.log2Uper = ilog2(pp.Uper);
+    pp.modes[0] = pp.in_stride == 1 ? kQF : kUF;
+    pp.modes[1] = kUF;
+    pp.modes[2] = pp.out_stride == 1 ? kRQF : kUF;
+    pp.swz_tab = choose_swizzle(r, pp.s, pp.modes);
     for (int d = 0; d < 2 && rc == TCU_DFT_OK; ++d) {
       const int sign = d == 0 ? -1 : 1;
       rc = upload(&pp.twL[d], twiddle_table(L, L, 1, sign));
@@ -776,6 +1274,37 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
   const int di = dir_index(dir);
   for (int pi = 0; pi < p->npasses; ++pi) {
     const PassPlan &pp = p->pass[pi];
+    if (pp.kind == kGroupPass) {
+      GroupArgs g;
+      memset(&g, 0, sizeof(g));
+      g.in = (pi == 0) ? (const float2 *)in : p->scratch;
+      g.out = pp.last ? (float2 *)out : p->scratch;
+      g.bimg = p->bimg[di];
+      g.twL = pp.twL[di];
+      g.twA = p->twA[di];
+      g.twB = p->twB[di];
+      g.err = p->err;
+      g.U = pp.U;
+      g.n = p->n;
+      g.in_vstride = pp.in_vstride;
+      g.in_stride = pp.in_stride;
+      g.out_vstride = pp.out_vstride;
+      g.out_stride = pp.out_stride;
+      g.log2Uper = pp.log2Uper;
+      g.tw_log2N = pp.tw_log2N;
+      g.tw_h = pp.tw_h;
+      g.mode_first = pp.modes[0];
+      g.mode_mid = pp.modes[1];
+      g.mode_last = pp.modes[2];
+      g.swz_tab = pp.swz_tab;
+      g.scale = (pp.last && dir == TCU_DFT_INVERSE) ? (float)(1.0 / (double)p->n) : 1.0f;
+      if (events && cudaEventRecord((cudaEvent_t)events[pi], st) != cudaSuccess)
+        return TCU_DFT_ERR_CUDA;
+      if (launch_group_dispatch(p->r, p->precision, pp.s, g, p->num_sms, st) !=
+          cudaSuccess)
+        return TCU_DFT_ERR_CUDA;
+      continue;
+    }
     PassArgs a;
     memset(&a, 0, sizeof(a));
     a.in = (pi == 0) ? (const float2 *)in : p->scratch;
