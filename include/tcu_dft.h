@@ -71,6 +71,24 @@ enum {
 tcu_dft_plan_t tcu_dft_plan(int64_t n, int64_t batch, int32_t sqrt_m,
                             int32_t precision);
 
+/* Plan flags for tcu_dft_plan_ex. */
+enum {
+  TCU_DFT_PLAN_DEFAULT = 0,
+  /* Run a two-pass transform as two separate kernel launches with a full
+   * batch*n intermediate in HBM, instead of the single fused launch whose
+   * intermediate is a small ring kept in L2. */
+  TCU_DFT_PLAN_NO_FUSE = 1
+};
+
+/* tcu_dft_plan with scheduling flags (TCU_DFT_PLAN_*); unknown bits are
+ * rejected with ERR_INVALID.  Same results either way. */
+tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
+                               int32_t precision, uint32_t flags);
+
+/* 1 if the plan runs its two passes as one fused launch, 0 if not, -1 for a
+ * NULL plan. */
+int tcu_dft_is_fused(tcu_dft_plan_t p);
+
 /* Forward transform: equivalent to tcu_dft_exec_dir(p, in, out,
  * TCU_DFT_FORWARD, stream). */
 int tcu_dft_exec(tcu_dft_plan_t p, const void *in, void *out, void *stream);

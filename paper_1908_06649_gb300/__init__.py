@@ -29,8 +29,12 @@ ERR_CUDA = 3
 ERR_OOM = 4
 ERR_TIMEOUT = 5
 
+PLAN_DEFAULT = 0
+PLAN_NO_FUSE = 1
+
 SYMBOLS = (
-    "tcu_dft_plan", "tcu_dft_exec", "tcu_dft_exec_dir", "tcu_dft_exec_timed",
+    "tcu_dft_plan", "tcu_dft_plan_ex", "tcu_dft_is_fused", "tcu_dft_exec",
+    "tcu_dft_exec_dir", "tcu_dft_exec_timed",
     "tcu_dft_exec_host",
     "tcu_dft_check", "tcu_dft_destroy", "tcu_dft_num_passes",
     "tcu_dft_pass_stages", "tcu_dft_last_error", "tcu_dft_strerror",
@@ -63,6 +67,10 @@ def lib():
     vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
     L.tcu_dft_plan.argtypes = [i64, i64, i32, i32]
     L.tcu_dft_plan.restype = vp
+    L.tcu_dft_plan_ex.argtypes = [i64, i64, i32, i32, ctypes.c_uint32]
+    L.tcu_dft_plan_ex.restype = vp
+    L.tcu_dft_is_fused.argtypes = [vp]
+    L.tcu_dft_is_fused.restype = ctypes.c_int
     L.tcu_dft_exec.argtypes = [vp, vp, vp, vp]
     L.tcu_dft_exec.restype = ctypes.c_int
     L.tcu_dft_exec_dir.argtypes = [vp, vp, vp, ctypes.c_int, vp]
@@ -111,9 +119,10 @@ class Plan:
     """
 
     def __init__(self, n: int, batch: int, sqrt_m: int = 16,
-                 precision: int = X3TF32):
+                 precision: int = X3TF32, flags: int = PLAN_DEFAULT):
         L = lib()
-        h = L.tcu_dft_plan(int(n), int(batch), int(sqrt_m), int(precision))
+        h = L.tcu_dft_plan_ex(int(n), int(batch), int(sqrt_m), int(precision),
+                              int(flags))
         if not h:
             raise TcuDftError(L.tcu_dft_last_error(), "tcu_dft_plan")
         self._h = h
@@ -123,6 +132,10 @@ class Plan:
     @property
     def handle(self):
         return self._h
+
+    @property
+    def fused(self) -> bool:
+        return lib().tcu_dft_is_fused(self._h) == 1
 
     def passes(self):
         L = lib()

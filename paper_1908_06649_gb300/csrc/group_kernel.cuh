@@ -1,0 +1,725 @@
+// group_kernel.cuh -- warpgroup kernels for passes whose sub-transforms fit
+// in 128 data rows (L = r^S <= 128 r).
+//
+// A CTA (one per SM, persistent) holds NWG independent warpgroups.  A
+// warpgroup owns one TMEM slot (A_hi | A_lo | D for 128 rows), one SMEM
+// transpose buffer and one mbarrier, and processes work items; an item is
+// GG = 128 r / L consecutive sub-transforms, i.e. exactly 128 data rows per
+// stage, so every stage of an item is ONE M=128 tall-left tcgen05 product
+// with F_r (the (m,l)-TCU call of Sec. 3 / Theorem 7) and the transposition
+// between stages stays inside the warpgroup.
+//
+// Per item: the stage-1 rows come from global memory straight into
+// registers (the row-to-lane map makes the loads coalesced), are split into
+// TF32 hi/lo parts and stored into TMEM as the A operand; one thread issues
+// the products; the epilogue reads D from TMEM, multiplies by the stage
+// twiddles w_L^{k_t c_t} and writes the transposed rows of the next stage to
+// SMEM; the last stage's outputs go straight from registers to global memory
+// in natural order, with the inter-pass twiddle w_n^{b k} of the four-step
+// split applied on the way (the inverse's 1/n is folded, exactly, into a
+// 2^-log2(n)-scaled copy of F_r used by the last stage).  The next item's
+// rows are prefetched into registers while the current item's products run.
+//
+// The whole geometry of a pass (radix, stage counts of both passes, role) is
+// a template parameter, so every stride is a compile-time constant and the
+// element addresses are immediate offsets from one per-row base pointer.
+//
+// Two kernels share the item routine:
+//   dft_pass_kernel   -- one pass, items assigned round-robin;
+//   dft_fused_kernel  -- both passes of a two-pass (four-step) transform in
+//     ONE launch: a work queue interleaves the passes by chunks of C
+//     transforms, pass-1 items write their output to a small ring of chunks
+//     that stays resident in L2, and pass-2 items read it back once all
+//     pass-1 items of their transform have signalled (release/acquire
+//     counters).  HBM then sees each point read once and written once.
+#pragma once
+#include "../../include/tcu_dft.h"
+#include "tcgen05.cuh"
+
+namespace tcu {
+
+enum RowMode { kQF = 0, kUF = 1, kRQF = 2 };
+enum Role { kSingle = 0, kFirst = 1, kSecond = 2 };
+
+constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 16 ? 4 : 5); }
+constexpr int nwg_of(int R) { return R == 32 ? 2 : 4; }
+
+// Compile-time geometry of one pass: S stages of radix R; the other pass (if
+// any) has SO stages.  Sub-transform u = b * Uper + v of transform b.
+//   kSingle: x[b n + a]                      -> y[b n + k]
+//   kFirst : x[b n + a n2 + v] (n2 = R^SO)   -> T[b n + k n2 + v] * w_n^{v k}
+//   kSecond: T[b n + v L + a]                -> y[b n + v + k n1] (n1 = R^SO)
+template <int R, int S, int SO, int ROLE>
+struct Geo {
+  static constexpr int LOG2R = log2_radix(R);
+  static constexpr int NWG = nwg_of(R);
+  static constexpr int THREADS = 128 * NWG;
+  static constexpr int LOG2GPTS = 7 + LOG2R;   // 128 rows of R points
+  static constexpr int GPTS = 1 << LOG2GPTS;
+  static constexpr int LOG2L = LOG2R * S;
+  static constexpr int L = 1 << LOG2L;
+  static constexpr int LOG2N = LOG2R * (S + SO);
+  static constexpr int LOG2RPS = LOG2L - LOG2R;   // rows per sub-transform
+  static constexpr int LOG2GG = LOG2GPTS - LOG2L; // sub-transforms per item
+  static constexpr int GG = 1 << LOG2GG;
+  static constexpr int LOG2O = LOG2R * SO;
+  static constexpr int LOG2UPER = ROLE == kSingle ? 0 : LOG2O;
+  static constexpr long long IN_STRIDE = ROLE == kFirst ? (1ll << LOG2O) : 1;
+  static constexpr long long IN_VSTRIDE = ROLE == kFirst ? 1 : (ROLE == kSecond ? L : 0);
+  static constexpr long long OUT_STRIDE = ROLE == kSingle ? 1 : (1ll << LOG2O);
+  static constexpr long long OUT_VSTRIDE = ROLE == kSingle ? 0 : 1;
+  static constexpr int MODE_FIRST = ROLE == kFirst ? kUF : kQF;
+  static constexpr int MODE_MID = kUF;
+  static constexpr int MODE_LAST = ROLE == kSingle ? kRQF : kUF;
+  static constexpr bool TW_OUT = ROLE == kFirst;
+  static constexpr int Q = (2 * R > 32) ? 2 * R : 32;
+  static constexpr int GCOLS = 3 * Q;
+  static constexpr int IMG_BYTES = 16 * R * R;
+  // entries of the stage twiddle tables: sum over t < S of R * R^(S-t)
+  static constexpr int TW_ENTRIES = S == 1 ? 0 : (S == 2 ? R * R : R * R * R + R * R);
+  static_assert(LOG2GG >= 0, "sub-transform longer than one item");
+  static_assert(NWG * GCOLS <= 512, "TMEM budget");
+};
+
+// Runtime part of a pass.
+struct PRun {
+  const float2 *in;
+  float2 *out;
+  long long in_bmask, out_bmask;  // transform index mask (ring) or ~0
+  long long U;                    // sub-transforms in the pass
+  const float2 *tw_out;           // kFirst: w_n^{v k} as [k][v]
+  const float2 *tw_stage;         // stage twiddles [t][j][lo]
+  unsigned long long swz_tab;     // SMEM swizzle nibble per (ul & 15)
+  int last_img;                   // byte offset of the last stage's F images
+};
+
+struct GArgs {
+  PRun p[2];
+  const float *bimg;    // F_r images: hi, lo, hi*2^-log2n, lo*2^-log2n
+  int *err;
+  // fused schedule
+  int *counters;        // [0] queue head, [1, 1+batch) done1, then done2
+  long long batch;
+  int nchunks, lag, ring_chunks;
+  int items1_per_tf;    // pass-1 items per transform
+  int items1_per_chunk, items2_per_chunk;
+};
+
+// Offset of stage t's block [j][lo] in the stage twiddle table.
+template <int R, int S>
+__host__ __device__ constexpr int tw_stage_offset(int t) {
+  int off = 0, p = 1;
+  for (int i = 0; i < S - 1; ++i) p *= R;  // R^(S-1)
+  for (int u = 1; u < t; ++u) {
+    off += R * p;  // block u holds R * R^(S-u) entries
+    p /= R;
+  }
+  return off;
+}
+
+// Shared memory: 4 F images | stage twiddles (two passes) | NWG transpose
+// buffers | NWG mbarriers | TMEM slot | NWG scheduler mailboxes.
+template <int R, int TW1, int TW2>
+struct SmemLayout {
+  static constexpr int NWG = nwg_of(R);
+  static constexpr size_t IMG = 4 * 16 * R * R;
+  static constexpr size_t OFF_TW1 = IMG;
+  static constexpr size_t OFF_TW2 = OFF_TW1 + (size_t)TW1 * 8;
+  static constexpr size_t OFF_BUF = OFF_TW2 + (size_t)TW2 * 8;
+  static constexpr size_t BUF_PTS = 128 * R;
+  static constexpr size_t OFF_BAR = OFF_BUF + (size_t)NWG * BUF_PTS * 8;
+  static constexpr size_t OFF_SCHED = OFF_BAR + 8 * NWG + 8;
+  static constexpr size_t BYTES = OFF_SCHED + 32 * NWG;
+};
+
+// Per-warpgroup state.
+struct WG {
+  uint32_t slot;      // TMEM column base of this warpgroup's slot
+  uint32_t lane_off;  // this warp's TMEM lane quarter
+  uint32_t img_addr;  // SMEM address of the F images
+  uint32_t bar_addr;  // this warpgroup's mbarrier
+  int bar_id;         // named barrier id
+  int rho;            // this thread's row within the item (0..127)
+  float2 *buf;        // SMEM transpose buffer
+  uint32_t phase;
+  bool fail;
+};
+
+template <class G>
+__device__ __forceinline__ void row_of(int mode, int rho, int &ul, int &q) {
+  if (mode == kUF) {
+    ul = rho & (G::GG - 1);
+    q = rho >> G::LOG2GG;
+  } else {
+    ul = rho >> G::LOG2RPS;
+    q = rho & ((1 << G::LOG2RPS) - 1);
+    if (mode == kRQF) {  // digit-reversed q over S-1 digits
+      int rq = 0, v = q;
+#pragma unroll
+      for (int i = 0; i < G::LOG2RPS / G::LOG2R; ++i) {
+        rq = (rq << G::LOG2R) | (v & ((1 << G::LOG2R) - 1));
+        v >>= G::LOG2R;
+      }
+      q = rq;
+    }
+  }
+}
+
+__device__ __forceinline__ int gswz(int p, uint32_t tabv) {
+  return p ^ (int)((tabv ^ (uint32_t)(p >> 4)) & 15u);
+}
+
+// TF32 split of 8 complex values, stored as A operand columns of this
+// thread's TMEM lane.  3xTF32: hi keeps the top 10 explicit mantissa bits
+// (exactly representable in TF32) and lo = v - hi is exact in fp32.  TF32:
+// hi rounded to nearest.
+template <int PREC>
+__device__ __forceinline__ void split_store8(const float2 *x, uint32_t col_hi,
+                                             uint32_t col_lo) {
+  float vh[16], vl[16];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    if (PREC == 3) {
+      const float hx = __uint_as_float(__float_as_uint(x[j].x) & 0xFFFFE000u);
+      const float hy = __uint_as_float(__float_as_uint(x[j].y) & 0xFFFFE000u);
+      vh[2 * j] = hx;
+      vh[2 * j + 1] = hy;
+      vl[2 * j] = x[j].x - hx;
+      vl[2 * j + 1] = x[j].y - hy;
+    } else {
+      vh[2 * j] = tf32_rna(x[j].x);
+      vh[2 * j + 1] = tf32_rna(x[j].y);
+    }
+  }
+  tmem_st16(col_hi, vh);
+  if (PREC == 3) tmem_st16(col_lo, vl);
+}
+
+// One stage: D = A * Bf for the 128 rows of this warpgroup's slot.
+template <int R, int PREC>
+__device__ __forceinline__ void issue_stage_mma(uint32_t slot, uint32_t img_addr) {
+  constexpr int Q = (2 * R > 32) ? 2 * R : 32;
+  constexpr int IMG = 16 * R * R, LBO = 128, SBO = 64 * R, KSTEPS = 2 * R / 8;
+  constexpr uint32_t idesc = idesc_tf32(128, 2 * R);
+  const uint32_t ahi = slot, alo = slot + Q, d = slot + 2 * Q;
+  const uint32_t ihi = img_addr, ilo = img_addr + IMG;
+  uint32_t acc = 0;
+  if (PREC == 3) {
+    // small terms first: lo*Bhi, hi*Blo, then hi*Bhi
+#pragma unroll
+    for (int kk = 0; kk < KSTEPS; ++kk) {
+      mma_tf32_ts(d, alo + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO),
+                  idesc, acc);
+      acc = 1;
+    }
+#pragma unroll
+    for (int kk = 0; kk < KSTEPS; ++kk)
+      mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(ilo + kk * 2 * LBO, LBO, SBO),
+                  idesc, 1);
+  }
+#pragma unroll
+  for (int kk = 0; kk < KSTEPS; ++kk) {
+    mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO),
+                idesc, acc);
+    acc = 1;
+  }
+}
+
+// The stage-1 row of this thread for `item` (zeros past the end), via L2.
+template <class G>
+__device__ __forceinline__ void load_row(const PRun &P, long long item, bool valid,
+                                         int ul, int q, float2 *x) {
+  constexpr int R = 1 << G::LOG2R;
+  const long long u = (item << G::LOG2GG) + ul;
+  if (valid && u < P.U) {
+    const long long b = u >> G::LOG2UPER;
+    const long long v = u & ((1ll << G::LOG2UPER) - 1);
+    const float2 *src = P.in + ((b & P.in_bmask) << G::LOG2N) + v * G::IN_VSTRIDE +
+                        q * G::IN_STRIDE;
+    constexpr long long JS = G::IN_STRIDE << (G::LOG2L - G::LOG2R);
+#pragma unroll
+    for (int j = 0; j < R; ++j) x[j] = __ldcg(src + j * JS);
+  } else {
+#pragma unroll
+    for (int j = 0; j < R; ++j) x[j] = make_float2(0.f, 0.f);
+  }
+}
+
+// Epilogue of stage T < S: D -> registers, stage twiddle, transposed write.
+template <class G, int T>
+__device__ __forceinline__ void stage_epilogue(const PRun &P, const float2 *tws,
+                                               const WG &w) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  constexpr int SH = G::LOG2R * (S - T);  // digits below the current one
+  constexpr int TWOFF = tw_stage_offset<R, S>(T);
+  int ul, q;
+  row_of<G>(T == 1 ? G::MODE_FIRST : G::MODE_MID, w.rho, ul, q);
+  const int hi = q >> SH, lo = q & ((1 << SH) - 1);
+  const int base = (ul << G::LOG2L) + (hi << (SH + G::LOG2R)) + lo;
+  const uint32_t tabv = (uint32_t)(P.swz_tab >> (4 * (ul & 15))) & 15u;
+  const float2 *twrow = tws + TWOFF + lo;  // [j][lo], row length R^(S-T)
+#pragma unroll
+  for (int c = 0; c < R; c += 8) {
+    float d[16];
+    tmem_ld16(w.slot + 2 * G::Q + w.lane_off + 2 * c, d);
+#pragma unroll
+    for (int jj = 0; jj < 8; ++jj) {
+      const int j = c + jj;
+      const float2 y = cmul(make_float2(d[2 * jj], d[2 * jj + 1]), twrow[j << SH]);
+      w.buf[gswz(base + (j << SH), tabv)] = y;
+    }
+  }
+}
+
+// Rows of stage T >= 2 from the SMEM buffer into TMEM.
+template <class G, int PREC, int T>
+__device__ __forceinline__ void stage_rows(const PRun &P, const WG &w) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  constexpr int SH = G::LOG2R * (S - T);
+  int ul, q;
+  row_of<G>(T == S ? G::MODE_LAST : G::MODE_MID, w.rho, ul, q);
+  const int hi = q >> SH, lo = q & ((1 << SH) - 1);
+  const int base = (ul << G::LOG2L) + (hi << (SH + G::LOG2R)) + lo;
+  const uint32_t tabv = (uint32_t)(P.swz_tab >> (4 * (ul & 15))) & 15u;
+#pragma unroll
+  for (int c = 0; c < R; c += 8) {
+    float2 row[8];
+#pragma unroll
+    for (int jj = 0; jj < 8; ++jj) row[jj] = w.buf[gswz(base + ((c + jj) << SH), tabv)];
+    split_store8<PREC>(row, w.slot + w.lane_off + 2 * c, w.slot + G::Q + w.lane_off + 2 * c);
+  }
+}
+
+// Last stage: D -> registers -> natural-order output.
+template <class G, bool OUT_L2>
+__device__ __forceinline__ void last_stage_store(const PRun &P, long long item,
+                                                 const WG &w) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  int ul, q;
+  row_of<G>(G::MODE_LAST, w.rho, ul, q);
+  const long long u = (item << G::LOG2GG) + ul;
+  float d[2 * R];
+#pragma unroll
+  for (int c = 0; c < 2 * R; c += 16) tmem_ld16(w.slot + 2 * G::Q + w.lane_off + c, d + c);
+  if (u >= P.U) return;
+  int klow = 0, vq = q;
+#pragma unroll
+  for (int i = 0; i < S - 1; ++i) {
+    klow = (klow << G::LOG2R) | (vq & (R - 1));
+    vq >>= G::LOG2R;
+  }
+  const long long b = u >> G::LOG2UPER;
+  const long long v = u & ((1ll << G::LOG2UPER) - 1);
+  float2 *dst = P.out + ((b & P.out_bmask) << G::LOG2N) + v * G::OUT_VSTRIDE +
+                klow * G::OUT_STRIDE;
+  constexpr long long JS = G::OUT_STRIDE << (G::LOG2L - G::LOG2R);
+  const float2 *twp = P.tw_out + ((long long)klow << G::LOG2UPER) + v;
+  constexpr long long TWS = 1ll << (G::LOG2UPER + G::LOG2L - G::LOG2R);
+#pragma unroll
+  for (int j = 0; j < R; ++j) {
+    float2 y = make_float2(d[2 * j], d[2 * j + 1]);
+    if (G::TW_OUT) y = cmul(y, __ldg(twp + j * TWS));
+    if (OUT_L2)
+      __stcg(dst + j * JS, y);
+    else
+      __stcs(dst + j * JS, y);
+  }
+}
+
+// The whole item.  `mid` supplies the next-item logic:
+//   mid.claim()    -- thread rho==0, right after the stage-1 products issue
+//   mid.publish()  -- thread rho==0, just before the first epilogue barrier
+//   mid.prefetch() -- every thread, after the first stage's SMEM barrier
+//                     (for S == 1: right after claim, no barrier in between)
+template <class G, int PREC, bool OUT_L2, class Mid>
+__device__ __forceinline__ void process_item(const PRun &P, const float2 *tws,
+                                             long long item, float2 *x, WG &w,
+                                             Mid &mid) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr int S = G::LOG2L / G::LOG2R;
+#pragma unroll
+  for (int c = 0; c < R; c += 8)
+    split_store8<PREC>(x + c, w.slot + w.lane_off + 2 * c, w.slot + G::Q + w.lane_off + 2 * c);
+  tmem_wait_st();
+  fence_before_sync();
+  if (named_bar_or(w.bar_id, 128, w.fail)) {
+    w.fail = true;
+    return;
+  }
+  if (w.rho == 0) {
+    fence_after_sync();
+    issue_stage_mma<R, PREC>(w.slot, w.img_addr + (S == 1 ? P.last_img : 0));
+    mma_commit(w.bar_addr);
+    mid.claim();
+  }
+  if (S == 1) mid.prefetch();
+  if (!mbar_wait_bounded(w.bar_addr, w.phase)) w.fail = true;
+  w.phase ^= 1;
+  fence_after_sync();
+  constexpr int S2 = S >= 2 ? 2 : S, S3 = S >= 3 ? 3 : S2;
+#pragma unroll
+  for (int t = 1; t < S; ++t) {
+    if (t == 1) stage_epilogue<G, 1>(P, tws, w);
+    if (t == 2) stage_epilogue<G, S2>(P, tws, w);
+    if (t == 1 && w.rho == 0) mid.publish();
+    fence_before_sync();
+    named_bar_or(w.bar_id, 128, false);
+    if (t == 1) mid.prefetch();
+    if (t == 1) stage_rows<G, PREC, S2>(P, w);
+    if (t == 2) stage_rows<G, PREC, S3>(P, w);
+    tmem_wait_st();
+    fence_before_sync();
+    if (named_bar_or(w.bar_id, 128, w.fail)) {
+      w.fail = true;
+      return;
+    }
+    if (w.rho == 0) {
+      fence_after_sync();
+      issue_stage_mma<R, PREC>(w.slot, w.img_addr + (t + 1 == S ? P.last_img : 0));
+      mma_commit(w.bar_addr);
+    }
+    if (!mbar_wait_bounded(w.bar_addr, w.phase)) w.fail = true;
+    w.phase ^= 1;
+    fence_after_sync();
+  }
+  last_stage_store<G, OUT_L2>(P, item, w);
+}
+
+// Common set-up: F images and stage twiddles into SMEM, mbarriers, TMEM.
+template <int NWG, int THREADS>
+__device__ __forceinline__ uint32_t kernel_setup(const float *bimg, int img_floats,
+                                                 float *img, const float2 *tw_src0,
+                                                 float2 *tw_dst0, int tw_n0,
+                                                 const float2 *tw_src1, float2 *tw_dst1,
+                                                 int tw_n1, uint64_t *mbar,
+                                                 uint32_t *tmem_slot) {
+  const int tid = threadIdx.x;
+  {
+    const float4 *src = reinterpret_cast<const float4 *>(bimg);
+    float4 *dst = reinterpret_cast<float4 *>(img);
+    for (int i = tid; i < img_floats / 4; i += THREADS) dst[i] = __ldg(src + i);
+    for (int i = tid; i < tw_n0; i += THREADS) tw_dst0[i] = __ldg(tw_src0 + i);
+    for (int i = tid; i < tw_n1; i += THREADS) tw_dst1[i] = __ldg(tw_src1 + i);
+  }
+  if (tid == 0) {
+    for (int w = 0; w < NWG; ++w) mbar_init(smem_u32(mbar + w), 1);
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+  if ((tid >> 5) == 0) tmem_alloc(smem_u32(tmem_slot), 512);
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  return *tmem_slot;
+}
+
+__device__ __forceinline__ void kernel_teardown(uint32_t tbase) {
+  fence_before_sync();
+  __syncthreads();
+  if ((threadIdx.x >> 5) == 0) {
+    fence_after_sync();
+    tmem_dealloc(tbase, 512);
+  }
+}
+
+template <int NWG, int GCOLS>
+__device__ __forceinline__ void init_wg(WG &w, uint32_t tbase, unsigned char *smem,
+                                        size_t off_bar, size_t off_buf, size_t buf_pts) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int wg = warp >> 2;
+  uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + off_bar);
+  w.rho = (warp & 3) * 32 + lane;
+  w.slot = tbase + wg * GCOLS;
+  w.lane_off = (uint32_t)((warp & 3) * 32) << 16;
+  w.img_addr = smem_u32(smem);
+  w.bar_addr = smem_u32(mbar + wg);
+  w.bar_id = 1 + wg;
+  w.buf = reinterpret_cast<float2 *>(smem + off_buf) + wg * buf_pts;
+  w.phase = 0;
+  w.fail = false;
+}
+
+// ---------------------------------------------------------------- one pass
+template <class G>
+struct StaticNext {
+  const PRun &P;
+  long long next, nitems;
+  int ul, q;
+  float2 *x;
+  __device__ void claim() {}
+  __device__ void publish() {}
+  __device__ void prefetch() { load_row<G>(P, next, next < nitems, ul, q, x); }
+};
+
+template <int R, int PREC, int S, int SO, int ROLE>
+__global__ void __launch_bounds__(Geo<R, S, SO, ROLE>::THREADS, 1)
+    dft_pass_kernel(const GArgs a) {
+  using G = Geo<R, S, SO, ROLE>;
+  using SM = SmemLayout<R, G::TW_ENTRIES, 0>;
+  extern __shared__ __align__(1024) unsigned char smem[];
+  float2 *tw = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
+  uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + SM::OFF_BAR);
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + G::NWG);
+  const PRun &P = a.p[0];
+  const uint32_t tbase = kernel_setup<G::NWG, G::THREADS>(
+      a.bimg, (int)(SM::IMG / 4), reinterpret_cast<float *>(smem), P.tw_stage, tw,
+      G::TW_ENTRIES, P.tw_stage, tw, 0, mbar, tmem_slot);
+  WG w;
+  init_wg<G::NWG, G::GCOLS>(w, tbase, smem, SM::OFF_BAR, SM::OFF_BUF, SM::BUF_PTS);
+
+  const int wg = threadIdx.x >> 7;
+  const long long nitems = (P.U + G::GG - 1) >> G::LOG2GG;
+  const long long istride = (long long)gridDim.x * G::NWG;
+  long long item = (long long)blockIdx.x * G::NWG + wg;
+  int ul1, q1;
+  row_of<G>(G::MODE_FIRST, w.rho, ul1, q1);
+  float2 x[R];
+  load_row<G>(P, item, item < nitems, ul1, q1, x);
+  StaticNext<G> nx{P, item + istride, nitems, ul1, q1, x};
+  while (item < nitems && !w.fail) {
+    nx.next = item + istride;
+    process_item<G, PREC, false>(P, tw, item, x, w, nx);
+    item += istride;
+  }
+  if (w.fail && w.rho == 0) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);
+  kernel_teardown(tbase);
+}
+
+// ------------------------------------------------------- fused two passes
+__device__ __forceinline__ int ld_acquire(const int *p) {
+  int v;
+  asm volatile("ld.acquire.gpu.global.b32 %0, [%1];" : "=r"(v) : "l"(p) : "memory");
+  return v;
+}
+
+__device__ __forceinline__ void red_release_add(int *p, int v) {
+  asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
+}
+
+// Queue position -> (pass, item).  Order: P1(0) .. P1(lag-1), then for
+// c >= lag: P1(c), P2(c - lag); then the remaining P2 chunks.  Returns false
+// past the end.
+__device__ __forceinline__ bool decode_queue(const GArgs &a, long long pos, int &pass,
+                                             long long &item, int &chunk) {
+  const long long A = a.items1_per_chunk, B = a.items2_per_chunk;
+  const int lag = a.lag, nc = a.nchunks;
+  if (pos < (long long)lag * A) {
+    pass = 0;
+    chunk = (int)(pos / A);
+    item = chunk * A + pos % A;
+    return true;
+  }
+  const long long p2 = pos - (long long)lag * A;
+  const long long mid = (long long)(nc - lag) * (A + B);
+  if (p2 < mid) {
+    const long long step = p2 / (A + B), off = p2 % (A + B);
+    if (off < A) {
+      pass = 0;
+      chunk = (int)(lag + step);
+      item = chunk * A + off;
+    } else {
+      pass = 1;
+      chunk = (int)step;
+      item = chunk * B + (off - A);
+    }
+    return true;
+  }
+  const long long p3 = p2 - mid;
+  if (p3 < (long long)lag * B) {
+    pass = 1;
+    chunk = (int)(nc - lag + p3 / B);
+    item = chunk * B + p3 % B;
+    return true;
+  }
+  return false;
+}
+
+struct __align__(8) FusedSched {  // per-warpgroup mailbox for the next item
+  long long item;
+  int pass;         // 0, 1, or -1 (queue exhausted)
+  int chunk;
+  int ready;        // its dependencies were satisfied when checked
+  int pad;
+};
+
+// Next-item logic of the fused schedule.  The queue position of the item
+// after next is claimed (atomicAdd) and the dependency flag of the next item
+// is read (ld.acquire) right after the current item's first products are
+// issued; both results are consumed only at the end of the first epilogue, so
+// their latency hides behind the item's own work.  The completion of an
+// item is published (red.release, ordered after every thread's stores by the
+// warpgroup barriers in between) at the end of the following item's first
+// epilogue.
+template <class G1, class G2>
+struct FusedNext {
+  const GArgs &a;
+  FusedSched *box;
+  int ul1[2], q1[2];
+  float2 *x;
+  // every thread, filled by prefetch()
+  int npass, nchunk;
+  long long nitem;
+  bool loaded;
+  // thread rho == 0 only
+  bool c_valid;
+  int c_pass, c_chunk;
+  long long c_item;
+  int dep_val, dep_target;
+  int pos2;
+  int *pend_flag;
+
+  // A pass-1 item waits until the ring slot it overwrites has been drained
+  // by pass 2; a pass-2 item until every pass-1 item of its transform has
+  // been written.  Null flag: no dependency.
+  __device__ const int *dep_flag(int pass, long long item, int chunk, int &target) const {
+    if (pass == 0) {
+      if (chunk < a.ring_chunks) return nullptr;
+      target = a.items2_per_chunk;
+      return a.counters + 1 + a.batch + (chunk - a.ring_chunks);
+    }
+    target = a.items1_per_tf;
+    const long long u0 = item << G2::LOG2GG;
+    return a.counters + 1 + (u0 >> G2::LOG2UPER);
+  }
+
+  __device__ bool wait_deps(int pass, long long item, int chunk) const {
+    int target = 0;
+    const int *flag = dep_flag(pass, item, chunk, target);
+    if (!flag || ld_acquire(flag) >= target) return true;
+    const unsigned long long t0 = global_ns();
+    while (ld_acquire(flag) < target) {
+      if (global_ns() - t0 > kWaitNs) return false;
+      __nanosleep(100);
+    }
+    return true;
+  }
+
+  __device__ void take_claim(int pos) { c_valid = decode_queue(a, pos, c_pass, c_item, c_chunk); }
+
+  __device__ void publish_pending() {
+    if (pend_flag) {
+      red_release_add(pend_flag, 1);
+      pend_flag = nullptr;
+    }
+  }
+
+  __device__ void claim() {  // thread rho == 0, after the first products issue
+    dep_val = 1;
+    dep_target = 0;
+    if (c_valid) {
+      const int *flag = dep_flag(c_pass, c_item, c_chunk, dep_target);
+      if (flag) dep_val = ld_acquire(flag);
+    }
+    pos2 = atomicAdd(a.counters, 1);
+  }
+
+  __device__ void publish() {  // thread rho == 0, before the first epilogue barrier
+    publish_pending();  // the previous item's stores were issued long ago
+    box->pass = c_valid ? c_pass : -1;
+    box->item = c_item;
+    box->chunk = c_chunk;
+    box->ready = (dep_val >= dep_target) ? 1 : 0;
+    take_claim(pos2);
+  }
+
+  __device__ void load(int pass, long long item) {
+    if (pass == 0)
+      load_row<G1>(a.p[0], item, true, ul1[0], q1[0], x);
+    else
+      load_row<G2>(a.p[1], item, true, ul1[1], q1[1], x);
+  }
+
+  __device__ void prefetch() {  // every thread, after the barrier following publish()
+    npass = box->pass;
+    nitem = box->item;
+    nchunk = box->chunk;
+    loaded = false;
+    if (npass >= 0 && box->ready) {
+      load(npass, nitem);
+      loaded = true;
+    }
+  }
+};
+
+template <int R, int PREC, int S1, int S2>
+__global__ void __launch_bounds__(Geo<R, S1, S2, kFirst>::THREADS, 1)
+    dft_fused_kernel(const GArgs a) {
+  static_assert(S1 >= 2 && S2 >= 2, "the fused schedule needs an SMEM barrier per item");
+  using G1 = Geo<R, S1, S2, kFirst>;
+  using G2 = Geo<R, S2, S1, kSecond>;
+  using SM = SmemLayout<R, G1::TW_ENTRIES, G2::TW_ENTRIES>;
+  constexpr int NWG = G1::NWG;
+  extern __shared__ __align__(1024) unsigned char smem[];
+  float2 *tw1 = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
+  float2 *tw2 = reinterpret_cast<float2 *>(smem + SM::OFF_TW2);
+  uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + SM::OFF_BAR);
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + NWG);
+  FusedSched *boxes = reinterpret_cast<FusedSched *>(smem + SM::OFF_SCHED);
+  const uint32_t tbase = kernel_setup<NWG, G1::THREADS>(
+      a.bimg, (int)(SM::IMG / 4), reinterpret_cast<float *>(smem), a.p[0].tw_stage, tw1,
+      G1::TW_ENTRIES, a.p[1].tw_stage, tw2, G2::TW_ENTRIES, mbar, tmem_slot);
+  WG w;
+  init_wg<NWG, G1::GCOLS>(w, tbase, smem, SM::OFF_BAR, SM::OFF_BUF, SM::BUF_PTS);
+  const int wg = threadIdx.x >> 7;
+
+  float2 x[R];
+  FusedNext<G1, G2> nx{a, boxes + wg};
+  nx.x = x;
+  nx.pend_flag = nullptr;
+  row_of<G1>(G1::MODE_FIRST, w.rho, nx.ul1[0], nx.q1[0]);
+  row_of<G2>(G2::MODE_FIRST, w.rho, nx.ul1[1], nx.q1[1]);
+
+  // first item: claim it and the one after, wait for its dependencies
+  bool f = false;
+  if (w.rho == 0) {
+    nx.take_claim(atomicAdd(a.counters, 1));
+    nx.dep_val = 1;
+    nx.dep_target = 0;
+    if (nx.c_valid && !nx.wait_deps(nx.c_pass, nx.c_item, nx.c_chunk)) f = true;
+    nx.pos2 = atomicAdd(a.counters, 1);
+    nx.publish();
+  }
+  if (named_bar_or(w.bar_id, 128, f)) w.fail = true;
+  if (!w.fail) nx.prefetch();
+
+  while (!w.fail && nx.npass >= 0) {
+    const int pass = nx.npass, chunk = nx.nchunk;
+    const long long item = nx.nitem;
+    if (pass == 0)
+      process_item<G1, PREC, true>(a.p[0], tw1, item, x, w, nx);
+    else
+      process_item<G2, PREC, false>(a.p[1], tw2, item, x, w, nx);
+    if (w.fail) break;
+    // completion is published during the next item (after its first
+    // barrier), or below
+    if (w.rho == 0)
+      nx.pend_flag = (pass == 0) ? a.counters + 1 + ((item << G1::LOG2GG) >> G1::LOG2UPER)
+                                 : a.counters + 1 + a.batch + chunk;
+    if (nx.npass >= 0 && !nx.loaded) {
+      bool ff = false;
+      // publish our own completion first: the item we wait for may need it
+      if (named_bar_or(w.bar_id, 128, false)) ff = true;
+      if (w.rho == 0) {
+        nx.publish_pending();
+        if (!nx.wait_deps(nx.npass, nx.nitem, nx.nchunk)) ff = true;
+      }
+      if (named_bar_or(w.bar_id, 128, ff)) {
+        w.fail = true;
+        break;
+      }
+      nx.load(nx.npass, nx.nitem);
+    }
+  }
+  // all stores of this warpgroup are issued: publish the last completion
+  named_bar_or(w.bar_id, 128, false);
+  if (w.rho == 0) {
+    nx.publish_pending();
+    if (w.fail) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);
+  }
+  kernel_teardown(tbase);
+}
+
+}  // namespace tcu

@@ -77,7 +77,8 @@ def test_single_pass(pkg, r, k, prec):
 
 @pytest.mark.parametrize("r,k,batch", [(16, 4, 5), (8, 5, 3), (32, 3, 3),
                                        (16, 5, 2), (8, 6, 2), (32, 4, 1),
-                                       (16, 6, 1), (8, 7, 1)])
+                                       (16, 6, 1), (8, 7, 1),
+                                       (16, 4, 40), (8, 5, 48), (8, 6, 12)])
 @pytest.mark.parametrize("prec", [3, 1])
 def test_two_pass(pkg, r, k, batch, prec):
     n = r ** k
