@@ -2,27 +2,27 @@
 // in 128 data rows (L = r^S <= 128 r).
 //
 // A CTA (one per SM, persistent) holds NWG independent warpgroups.  A
-// warpgroup owns one TMEM slot (A_hi | A_lo | D for 128 rows), one SMEM
-// transpose buffer and one mbarrier, and processes work items; an item is
-// GG = 128 r / L consecutive sub-transforms, i.e. exactly 128 data rows per
+// warpgroup owns one TMEM slot (A_hi | A_lo | D for 128 rows), SMEM staging
+// and transpose buffers and its mbarriers, and processes work items; an item
+// is GG = 128 r / L consecutive sub-transforms, i.e. exactly 128 data rows per
 // stage, so every stage of an item is ONE M=128 tall-left tcgen05 product
 // with F_r (the (m,l)-TCU call of Sec. 3 / Theorem 7) and the transposition
 // between stages stays inside the warpgroup.
 //
-// Per item: the stage-1 rows come from global memory straight into
-// registers (the row-to-lane map makes the loads coalesced), are split into
-// TF32 hi/lo parts and stored into TMEM as the A operand; one thread issues
-// the products; the epilogue reads D from TMEM, multiplies by the stage
-// twiddles w_L^{k_t c_t} and writes the transposed rows of the next stage to
-// SMEM; the last stage's outputs go straight from registers to global memory
-// in natural order, with the inter-pass twiddle w_n^{b k} of the four-step
-// split applied on the way (the inverse's 1/n is folded, exactly, into a
-// 2^-log2(n)-scaled copy of F_r used by the last stage).  The next item's
-// rows are prefetched into registers while the current item's products run.
+// Per item: the item's input block arrives in SMEM by TMA (a 1-D bulk copy
+// when it is contiguous, a 3-D tensor box for the strided first pass of a
+// four-step split), issued by one thread a whole item ahead; every thread
+// reads its stage-1 row from there, splits it into TF32 hi/lo parts and
+// stores them into TMEM as the A operand; one thread issues the products; the
+// epilogue reads D from TMEM, multiplies by the stage twiddles w_L^{k_t c_t}
+// and writes the transposed rows of the next stage to SMEM; the last stage's
+// outputs go straight from registers to global memory in natural order, with
+// the inter-pass twiddle w_n^{b k} of the four-step split (also staged by
+// TMA) applied on the way.  The inverse's 1/n is folded, exactly, into a
+// 2^-log2(n)-scaled copy of F_r used by the last stage.
 //
 // The whole geometry of a pass (radix, stage counts of both passes, role) is
-// a template parameter, so every stride is a compile-time constant and the
-// element addresses are immediate offsets from one per-row base pointer.
+// a template parameter, so every stride is a compile-time constant.
 //
 // Two kernels share the item routine:
 //   dft_pass_kernel   -- one pass, items assigned round-robin;
@@ -33,6 +33,8 @@
 //     pass-1 items of their transform have signalled (release/acquire
 //     counters).  HBM then sees each point read once and written once.
 #pragma once
+#include <cuda.h>
+
 #include "../../include/tcu_dft.h"
 #include "tcgen05.cuh"
 
@@ -64,14 +66,14 @@ struct Geo {
   static constexpr int GG = 1 << LOG2GG;
   static constexpr int LOG2O = LOG2R * SO;
   static constexpr int LOG2UPER = ROLE == kSingle ? 0 : LOG2O;
-  static constexpr long long IN_STRIDE = ROLE == kFirst ? (1ll << LOG2O) : 1;
-  static constexpr long long IN_VSTRIDE = ROLE == kFirst ? 1 : (ROLE == kSecond ? L : 0);
   static constexpr long long OUT_STRIDE = ROLE == kSingle ? 1 : (1ll << LOG2O);
   static constexpr long long OUT_VSTRIDE = ROLE == kSingle ? 0 : 1;
   static constexpr int MODE_FIRST = ROLE == kFirst ? kUF : kQF;
   static constexpr int MODE_MID = kUF;
   static constexpr int MODE_LAST = ROLE == kSingle ? kRQF : kUF;
   static constexpr bool TW_OUT = ROLE == kFirst;
+  static constexpr bool TW_SMEM = TW_OUT && R != 32;  // twiddles staged by TMA
+  static constexpr int TMA_ROWS = L < 256 ? L : 256;  // tensor box height
   static constexpr int Q = (2 * R > 32) ? 2 * R : 32;
   static constexpr int GCOLS = 3 * Q;
   static constexpr int IMG_BYTES = 16 * R * R;
@@ -95,6 +97,8 @@ struct PRun {
 
 struct GArgs {
   PRun p[2];
+  CUtensorMap tm_in;    // kFirst input  x as [b][a][2 v + re/im] floats
+  CUtensorMap tm_tw;    // kFirst twiddles tw_out as [1][k][2 v + re/im]
   const float *bimg;    // F_r images: hi, lo, hi*2^-log2n, lo*2^-log2n
   int *err;
   // fused schedule
@@ -117,19 +121,25 @@ __host__ __device__ constexpr int tw_stage_offset(int t) {
   return off;
 }
 
-// Shared memory: 4 F images | stage twiddles (two passes) | NWG transpose
-// buffers | NWG mbarriers | TMEM slot | NWG scheduler mailboxes.
+// Shared memory: 4 F images | stage twiddles of two passes | per warpgroup
+// transpose buffer, input staging and twiddle staging | mbarriers (3 per
+// warpgroup: products, input staging, twiddle staging) | TMEM slot |
+// scheduler mailboxes.
 template <int R, int TW1, int TW2>
 struct SmemLayout {
   static constexpr int NWG = nwg_of(R);
   static constexpr size_t IMG = 4 * 16 * R * R;
   static constexpr size_t OFF_TW1 = IMG;
   static constexpr size_t OFF_TW2 = OFF_TW1 + (size_t)TW1 * 8;
-  static constexpr size_t OFF_BUF = OFF_TW2 + (size_t)TW2 * 8;
-  static constexpr size_t BUF_PTS = 128 * R;
-  static constexpr size_t OFF_BAR = OFF_BUF + (size_t)NWG * BUF_PTS * 8;
-  static constexpr size_t OFF_SCHED = OFF_BAR + 8 * NWG + 8;
+  static constexpr size_t PTS = 128 * R;  // points per item
+  static constexpr size_t OFF_BUF = (OFF_TW2 + (size_t)TW2 * 8 + 127) / 128 * 128;
+  static constexpr size_t OFF_STG = OFF_BUF + (size_t)NWG * PTS * 8;
+  static constexpr size_t OFF_TWS = OFF_STG + (size_t)NWG * PTS * 8;
+  static constexpr size_t TWS_BYTES = (R == 32) ? 0 : (size_t)NWG * PTS * 8;
+  static constexpr size_t OFF_BAR = OFF_TWS + TWS_BYTES;
+  static constexpr size_t OFF_SCHED = OFF_BAR + 8 * 3 * NWG + 8;
   static constexpr size_t BYTES = OFF_SCHED + 32 * NWG;
+  static_assert(BYTES <= 227 * 1024, "shared memory budget");
 };
 
 // Per-warpgroup state.
@@ -137,12 +147,17 @@ struct WG {
   uint32_t slot;      // TMEM column base of this warpgroup's slot
   uint32_t lane_off;  // this warp's TMEM lane quarter
   uint32_t img_addr;  // SMEM address of the F images
-  uint32_t bar_addr;  // this warpgroup's mbarrier
+  uint32_t bar_mma;   // mbarrier: products done
+  uint32_t bar_stg;   // mbarrier: input staging full
+  uint32_t bar_tws;   // mbarrier: twiddle staging full
   int bar_id;         // named barrier id
   int rho;            // this thread's row within the item (0..127)
   float2 *buf;        // SMEM transpose buffer
-  uint32_t phase;
+  float2 *stg;        // SMEM input staging (one item)
+  float2 *tws;        // SMEM twiddle staging (one item)
+  uint32_t ph_mma, ph_stg, ph_tws;
   bool fail;
+  bool tws_inflight;  // thread rho == 0: a twiddle copy has not been waited on
 };
 
 template <class G>
@@ -225,23 +240,63 @@ __device__ __forceinline__ void issue_stage_mma(uint32_t slot, uint32_t img_addr
   }
 }
 
-// The stage-1 row of this thread for `item` (zeros past the end), via L2.
+// ---- TMA issue (one thread): the input block of `item` into staging
 template <class G>
-__device__ __forceinline__ void load_row(const PRun &P, long long item, bool valid,
-                                         int ul, int q, float2 *x) {
-  constexpr int R = 1 << G::LOG2R;
-  const long long u = (item << G::LOG2GG) + ul;
-  if (valid && u < P.U) {
-    const long long b = u >> G::LOG2UPER;
-    const long long v = u & ((1ll << G::LOG2UPER) - 1);
-    const float2 *src = P.in + ((b & P.in_bmask) << G::LOG2N) + v * G::IN_VSTRIDE +
-                        q * G::IN_STRIDE;
-    constexpr long long JS = G::IN_STRIDE << (G::LOG2L - G::LOG2R);
+__device__ __forceinline__ void issue_input(const PRun &P, const CUtensorMap *tm,
+                                            long long item, const WG &w) {
+  const long long u0 = item << G::LOG2GG;
+  const uint32_t dst = smem_u32(w.stg);
+  if (G::MODE_FIRST == kUF) {
+    // strided first pass: box of GG sub-transforms x L points
+    const long long b = u0 >> G::LOG2UPER;
+    const int v0 = (int)(u0 & ((1ll << G::LOG2UPER) - 1));
+    mbar_expect_tx(w.bar_stg, G::GPTS * 8);
 #pragma unroll
-    for (int j = 0; j < R; ++j) x[j] = __ldcg(src + j * JS);
+    for (int a0 = 0; a0 < G::L; a0 += G::TMA_ROWS)
+      tma_load_3d(dst + a0 * G::GG * 8, tm, 2 * v0, a0, (int)b, w.bar_stg);
   } else {
+    // contiguous block of GG sub-transforms (the last item may be short)
+    long long rem = P.U - u0;
+    if (rem > G::GG) rem = G::GG;
+    const uint32_t bytes = (uint32_t)(rem << G::LOG2L) * 8u;
+    const long long b = u0 >> G::LOG2UPER;
+    const long long v = u0 & ((1ll << G::LOG2UPER) - 1);
+    const float2 *src = P.in + ((b & P.in_bmask) << G::LOG2N) + (v << G::LOG2L);
+    mbar_expect_tx(w.bar_stg, bytes);
+    tma_load_1d(dst, src, bytes, w.bar_stg);
+  }
+}
+
+// ---- TMA issue (one thread): the inter-pass twiddles of a first-pass item
+template <class G>
+__device__ __forceinline__ void issue_twiddles(const CUtensorMap *tm, long long item,
+                                               const WG &w) {
+  if constexpr (G::TW_SMEM) {
+    const long long u0 = item << G::LOG2GG;
+    const int v0 = (int)(u0 & ((1ll << G::LOG2UPER) - 1));
+    const uint32_t dst = smem_u32(w.tws);
+    mbar_expect_tx(w.bar_tws, G::GPTS * 8);
 #pragma unroll
-    for (int j = 0; j < R; ++j) x[j] = make_float2(0.f, 0.f);
+    for (int k0 = 0; k0 < G::L; k0 += G::TMA_ROWS)
+      tma_load_3d(dst + k0 * G::GG * 8, tm, 2 * v0, k0, 0, w.bar_tws);
+  }
+}
+
+// This thread's stage-1 row, from the staged input block.
+template <class G>
+__device__ __forceinline__ void staged_row(const WG &w, float2 *x) {
+  constexpr int R = 1 << G::LOG2R;
+  int ul, q;
+  row_of<G>(G::MODE_FIRST, w.rho, ul, q);
+  constexpr int JS = 1 << (G::LOG2L - G::LOG2R);  // a = j * R^(S-1) + q
+  if (G::MODE_FIRST == kUF) {
+    const float2 *p = w.stg + q * G::GG + ul;  // staging [a][ul]
+#pragma unroll
+    for (int j = 0; j < R; ++j) x[j] = p[j * JS * G::GG];
+  } else {
+    const float2 *p = w.stg + (ul << G::LOG2L) + q;  // staging [ul][a]
+#pragma unroll
+    for (int j = 0; j < R; ++j) x[j] = p[j * JS];
   }
 }
 
@@ -294,8 +349,7 @@ __device__ __forceinline__ void stage_rows(const PRun &P, const WG &w) {
 
 // Last stage: D -> registers -> natural-order output.
 template <class G, bool OUT_L2>
-__device__ __forceinline__ void last_stage_store(const PRun &P, long long item,
-                                                 const WG &w) {
+__device__ __forceinline__ void last_stage_store(const PRun &P, long long item, WG &w) {
   constexpr int R = 1 << G::LOG2R;
   constexpr int S = G::LOG2L / G::LOG2R;
   int ul, q;
@@ -304,6 +358,13 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item,
   float d[2 * R];
 #pragma unroll
   for (int c = 0; c < 2 * R; c += 16) tmem_ld16(w.slot + 2 * G::Q + w.lane_off + c, d + c);
+  if constexpr (G::TW_SMEM) {
+    if (mbar_wait_bounded(w.bar_tws, w.ph_tws))
+      w.tws_inflight = false;
+    else
+      w.fail = true;
+    w.ph_tws ^= 1;
+  }
   if (u >= P.U) return;
   int klow = 0, vq = q;
 #pragma unroll
@@ -316,12 +377,16 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item,
   float2 *dst = P.out + ((b & P.out_bmask) << G::LOG2N) + v * G::OUT_VSTRIDE +
                 klow * G::OUT_STRIDE;
   constexpr long long JS = G::OUT_STRIDE << (G::LOG2L - G::LOG2R);
-  const float2 *twp = P.tw_out + ((long long)klow << G::LOG2UPER) + v;
-  constexpr long long TWS = 1ll << (G::LOG2UPER + G::LOG2L - G::LOG2R);
+  // twiddle of output k = klow + j r^(S-1): SMEM staging [k][ul], or global
+  const float2 *tws = w.tws + klow * G::GG + ul;
+  constexpr int TJS = G::GG << (G::LOG2L - G::LOG2R);
+  const float2 *twg = P.tw_out + ((long long)klow << G::LOG2UPER) + v;
+  constexpr long long TWG = 1ll << (G::LOG2UPER + G::LOG2L - G::LOG2R);
 #pragma unroll
   for (int j = 0; j < R; ++j) {
     float2 y = make_float2(d[2 * j], d[2 * j + 1]);
-    if (G::TW_OUT) y = cmul(y, __ldg(twp + j * TWS));
+    if (G::TW_SMEM) y = cmul(y, tws[j * TJS]);
+    else if (G::TW_OUT) y = cmul(y, __ldg(twg + j * TWG));
     if (OUT_L2)
       __stcg(dst + j * JS, y);
     else
@@ -329,35 +394,43 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item,
   }
 }
 
-// The whole item.  `mid` supplies the next-item logic:
-//   mid.claim()    -- thread rho==0, right after the stage-1 products issue
-//   mid.publish()  -- thread rho==0, just before the first epilogue barrier
-//   mid.prefetch() -- every thread, after the first stage's SMEM barrier
-//                     (for S == 1: right after claim, no barrier in between)
+// The whole item.  `mid` supplies the next-item logic (thread rho == 0 runs
+// issue() right after the stage-1 products and publish() just before the
+// first epilogue barrier).  On entry the item's input copy has been issued.
 template <class G, int PREC, bool OUT_L2, class Mid>
-__device__ __forceinline__ void process_item(const PRun &P, const float2 *tws,
-                                             long long item, float2 *x, WG &w,
+__device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *tm_tw,
+                                             const float2 *tws, long long item, WG &w,
                                              Mid &mid) {
   constexpr int R = 1 << G::LOG2R;
   constexpr int S = G::LOG2L / G::LOG2R;
+  if (!mbar_wait_bounded(w.bar_stg, w.ph_stg)) w.fail = true;
+  w.ph_stg ^= 1;
+  {
+    float2 x[R];
+    staged_row<G>(w, x);
 #pragma unroll
-  for (int c = 0; c < R; c += 8)
-    split_store8<PREC>(x + c, w.slot + w.lane_off + 2 * c, w.slot + G::Q + w.lane_off + 2 * c);
+    for (int c = 0; c < R; c += 8)
+      split_store8<PREC>(x + c, w.slot + w.lane_off + 2 * c, w.slot + G::Q + w.lane_off + 2 * c);
+  }
   tmem_wait_st();
   fence_before_sync();
   if (named_bar_or(w.bar_id, 128, w.fail)) {
     w.fail = true;
     return;
   }
+  // staging is free again: the next item's copy may land there
   if (w.rho == 0) {
     fence_after_sync();
     issue_stage_mma<R, PREC>(w.slot, w.img_addr + (S == 1 ? P.last_img : 0));
-    mma_commit(w.bar_addr);
-    mid.claim();
+    mma_commit(w.bar_mma);
+    if (G::TW_SMEM) {
+      issue_twiddles<G>(tm_tw, item, w);
+      w.tws_inflight = true;
+    }
+    mid.issue(w);
   }
-  if (S == 1) mid.prefetch();
-  if (!mbar_wait_bounded(w.bar_addr, w.phase)) w.fail = true;
-  w.phase ^= 1;
+  if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
+  w.ph_mma ^= 1;
   fence_after_sync();
   constexpr int S2 = S >= 2 ? 2 : S, S3 = S >= 3 ? 3 : S2;
 #pragma unroll
@@ -367,7 +440,6 @@ __device__ __forceinline__ void process_item(const PRun &P, const float2 *tws,
     if (t == 1 && w.rho == 0) mid.publish();
     fence_before_sync();
     named_bar_or(w.bar_id, 128, false);
-    if (t == 1) mid.prefetch();
     if (t == 1) stage_rows<G, PREC, S2>(P, w);
     if (t == 2) stage_rows<G, PREC, S3>(P, w);
     tmem_wait_st();
@@ -379,12 +451,13 @@ __device__ __forceinline__ void process_item(const PRun &P, const float2 *tws,
     if (w.rho == 0) {
       fence_after_sync();
       issue_stage_mma<R, PREC>(w.slot, w.img_addr + (t + 1 == S ? P.last_img : 0));
-      mma_commit(w.bar_addr);
+      mma_commit(w.bar_mma);
     }
-    if (!mbar_wait_bounded(w.bar_addr, w.phase)) w.fail = true;
-    w.phase ^= 1;
+    if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
+    w.ph_mma ^= 1;
     fence_after_sync();
   }
+  if (S == 1 && w.rho == 0) mid.publish();
   last_stage_store<G, OUT_L2>(P, item, w);
 }
 
@@ -405,7 +478,7 @@ __device__ __forceinline__ uint32_t kernel_setup(const float *bimg, int img_floa
     for (int i = tid; i < tw_n1; i += THREADS) tw_dst1[i] = __ldg(tw_src1 + i);
   }
   if (tid == 0) {
-    for (int w = 0; w < NWG; ++w) mbar_init(smem_u32(mbar + w), 1);
+    for (int w = 0; w < 3 * NWG; ++w) mbar_init(smem_u32(mbar + w), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
@@ -416,7 +489,14 @@ __device__ __forceinline__ uint32_t kernel_setup(const float *bimg, int img_floa
   return *tmem_slot;
 }
 
-__device__ __forceinline__ void kernel_teardown(uint32_t tbase) {
+// Leave: wait (bounded) for any copy still landing in this warpgroup's
+// staging, then free TMEM.
+__device__ __forceinline__ void kernel_teardown(uint32_t tbase, const WG &w, bool stg_pending,
+                                                bool tws_pending) {
+  if (w.rho == 0) {
+    if (stg_pending) mbar_wait_bounded(w.bar_stg, w.ph_stg);
+    if (tws_pending) mbar_wait_bounded(w.bar_tws, w.ph_tws);
+  }
   fence_before_sync();
   __syncthreads();
   if ((threadIdx.x >> 5) == 0) {
@@ -425,67 +505,71 @@ __device__ __forceinline__ void kernel_teardown(uint32_t tbase) {
   }
 }
 
-template <int NWG, int GCOLS>
-__device__ __forceinline__ void init_wg(WG &w, uint32_t tbase, unsigned char *smem,
-                                        size_t off_bar, size_t off_buf, size_t buf_pts) {
+template <int R, class SM, int GCOLS>
+__device__ __forceinline__ void init_wg(WG &w, uint32_t tbase, unsigned char *smem) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int wg = warp >> 2;
-  uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + off_bar);
+  uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + SM::OFF_BAR);
   w.rho = (warp & 3) * 32 + lane;
   w.slot = tbase + wg * GCOLS;
   w.lane_off = (uint32_t)((warp & 3) * 32) << 16;
   w.img_addr = smem_u32(smem);
-  w.bar_addr = smem_u32(mbar + wg);
+  w.bar_mma = smem_u32(mbar + 3 * wg);
+  w.bar_stg = smem_u32(mbar + 3 * wg + 1);
+  w.bar_tws = smem_u32(mbar + 3 * wg + 2);
   w.bar_id = 1 + wg;
-  w.buf = reinterpret_cast<float2 *>(smem + off_buf) + wg * buf_pts;
-  w.phase = 0;
+  w.buf = reinterpret_cast<float2 *>(smem + SM::OFF_BUF) + wg * SM::PTS;
+  w.stg = reinterpret_cast<float2 *>(smem + SM::OFF_STG) + wg * SM::PTS;
+  w.tws = reinterpret_cast<float2 *>(smem + SM::OFF_TWS) + (SM::TWS_BYTES ? wg * SM::PTS : 0);
+  w.ph_mma = w.ph_stg = w.ph_tws = 0;
   w.fail = false;
+  w.tws_inflight = false;
 }
 
 // ---------------------------------------------------------------- one pass
 template <class G>
 struct StaticNext {
   const PRun &P;
+  const CUtensorMap *tm;
   long long next, nitems;
-  int ul, q;
-  float2 *x;
-  __device__ void claim() {}
+  bool issued;  // a copy for `next` is in flight
+  __device__ void issue(const WG &w) {
+    issued = next < nitems;
+    if (issued) issue_input<G>(P, tm, next, w);
+  }
   __device__ void publish() {}
-  __device__ void prefetch() { load_row<G>(P, next, next < nitems, ul, q, x); }
 };
 
 template <int R, int PREC, int S, int SO, int ROLE>
 __global__ void __launch_bounds__(Geo<R, S, SO, ROLE>::THREADS, 1)
-    dft_pass_kernel(const GArgs a) {
+    dft_pass_kernel(const __grid_constant__ GArgs a) {
   using G = Geo<R, S, SO, ROLE>;
   using SM = SmemLayout<R, G::TW_ENTRIES, 0>;
   extern __shared__ __align__(1024) unsigned char smem[];
   float2 *tw = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
   uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + SM::OFF_BAR);
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + G::NWG);
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 3 * G::NWG);
   const PRun &P = a.p[0];
   const uint32_t tbase = kernel_setup<G::NWG, G::THREADS>(
       a.bimg, (int)(SM::IMG / 4), reinterpret_cast<float *>(smem), P.tw_stage, tw,
       G::TW_ENTRIES, P.tw_stage, tw, 0, mbar, tmem_slot);
   WG w;
-  init_wg<G::NWG, G::GCOLS>(w, tbase, smem, SM::OFF_BAR, SM::OFF_BUF, SM::BUF_PTS);
+  init_wg<R, SM, G::GCOLS>(w, tbase, smem);
 
   const int wg = threadIdx.x >> 7;
   const long long nitems = (P.U + G::GG - 1) >> G::LOG2GG;
   const long long istride = (long long)gridDim.x * G::NWG;
   long long item = (long long)blockIdx.x * G::NWG + wg;
-  int ul1, q1;
-  row_of<G>(G::MODE_FIRST, w.rho, ul1, q1);
-  float2 x[R];
-  load_row<G>(P, item, item < nitems, ul1, q1, x);
-  StaticNext<G> nx{P, item + istride, nitems, ul1, q1, x};
+  StaticNext<G> nx{P, &a.tm_in, item, nitems, false};
+  if (w.rho == 0 && item < nitems) issue_input<G>(P, &a.tm_in, item, w);
   while (item < nitems && !w.fail) {
     nx.next = item + istride;
-    process_item<G, PREC, false>(P, tw, item, x, w, nx);
+    process_item<G, PREC, false>(P, &a.tm_tw, tw, item, w, nx);
     item += istride;
   }
   if (w.fail && w.rho == 0) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);
-  kernel_teardown(tbase);
+  // on failure a copy issued for the next item may still be landing
+  kernel_teardown(tbase, w, w.fail && nx.issued, w.fail && w.tws_inflight);
 }
 
 // ------------------------------------------------------- fused two passes
@@ -537,57 +621,67 @@ __device__ __forceinline__ bool decode_queue(const GArgs &a, long long pos, int 
   return false;
 }
 
-struct __align__(8) FusedSched {  // per-warpgroup mailbox for the next item
+struct __align__(8) FusedSched {  // per-warpgroup mailbox: the next item
   long long item;
   int pass;         // 0, 1, or -1 (queue exhausted)
   int chunk;
-  int ready;        // its dependencies were satisfied when checked
+  int issued;       // its input copy is already in flight
   int pad;
 };
 
-// Next-item logic of the fused schedule.  The queue position of the item
-// after next is claimed (atomicAdd) and the dependency flag of the next item
-// is read (ld.acquire) right after the current item's first products are
-// issued; both results are consumed only at the end of the first epilogue, so
-// their latency hides behind the item's own work.  The completion of an
-// item is published (red.release, ordered after every thread's stores by the
-// warpgroup barriers in between) at the end of the following item's first
-// epilogue.
+struct QItem {
+  long long item;
+  int pass, chunk;
+  bool valid;
+};
+
+// Next-item logic of the fused schedule, run by one thread per warpgroup.
+// Items: cur (being processed), n1 (next), n2 (the one after).  During cur:
+//   issue()   -- right after cur's first products: if n1's dependency value
+//                (read one item earlier) says ready, issue n1's input copy;
+//                claim the queue position of the item after n1 (atomicAdd,
+//                its result is used only in publish());
+//   publish() -- before cur's first epilogue barrier: publish the completion
+//                of the previous item (red.release; every thread's stores of
+//                it are ordered before by the barriers in between), tell the
+//                warpgroup about n1, then decode n2 and start reading its
+//                dependency flag (ld.acquire, used in the next issue()).
+// So the latency of every atomic and flag read hides behind an item's work.
 template <class G1, class G2>
 struct FusedNext {
   const GArgs &a;
   FusedSched *box;
-  int ul1[2], q1[2];
-  float2 *x;
-  // every thread, filled by prefetch()
-  int npass, nchunk;
-  long long nitem;
-  bool loaded;
-  // thread rho == 0 only
-  bool c_valid;
-  int c_pass, c_chunk;
-  long long c_item;
+  QItem n1, n2;
   int dep_val, dep_target;
   int pos2;
+  bool n1_issued;
   int *pend_flag;
 
   // A pass-1 item waits until the ring slot it overwrites has been drained
   // by pass 2; a pass-2 item until every pass-1 item of its transform has
   // been written.  Null flag: no dependency.
-  __device__ const int *dep_flag(int pass, long long item, int chunk, int &target) const {
-    if (pass == 0) {
-      if (chunk < a.ring_chunks) return nullptr;
+  __device__ const int *dep_flag(const QItem &q, int &target) const {
+    if (q.pass == 0) {
+      if (q.chunk < a.ring_chunks) return nullptr;
       target = a.items2_per_chunk;
-      return a.counters + 1 + a.batch + (chunk - a.ring_chunks);
+      return a.counters + 1 + a.batch + (q.chunk - a.ring_chunks);
     }
     target = a.items1_per_tf;
-    const long long u0 = item << G2::LOG2GG;
+    const long long u0 = q.item << G2::LOG2GG;
     return a.counters + 1 + (u0 >> G2::LOG2UPER);
   }
 
-  __device__ bool wait_deps(int pass, long long item, int chunk) const {
+  __device__ void read_dep(const QItem &q) {
+    dep_val = 1;
+    dep_target = 0;
+    if (!q.valid) return;
+    const int *flag = dep_flag(q, dep_target);
+    if (flag) dep_val = ld_acquire(flag);
+  }
+
+  __device__ bool wait_deps(const QItem &q) const {
     int target = 0;
-    const int *flag = dep_flag(pass, item, chunk, target);
+    const int *flag = dep_flag(q, target);
     if (!flag || ld_acquire(flag) >= target) return true;
     const unsigned long long t0 = global_ns();
     while (ld_acquire(flag) < target) {
@@ -597,7 +691,19 @@ struct FusedNext {
     return true;
   }
 
-  __device__ void take_claim(int pos) { c_valid = decode_queue(a, pos, c_pass, c_item, c_chunk); }
+  __device__ QItem decode(int pos) const {
+    QItem q;
+    q.valid = decode_queue(a, pos, q.pass, q.item, q.chunk);
+    return q;
+  }
+
+  __device__ void issue_copy(const QItem &q, const WG &w) {
+    fence_proxy_async_global();  // the acquire of its flag comes first
+    if (q.pass == 0)
+      issue_input<G1>(a.p[0], &a.tm_in, q.item, w);
+    else
+      issue_input<G2>(a.p[1], &a.tm_in, q.item, w);
+  }
 
   __device__ void publish_pending() {
     if (pend_flag) {
@@ -606,47 +712,29 @@ struct FusedNext {
     }
   }
 
-  __device__ void claim() {  // thread rho == 0, after the first products issue
-    dep_val = 1;
-    dep_target = 0;
-    if (c_valid) {
-      const int *flag = dep_flag(c_pass, c_item, c_chunk, dep_target);
-      if (flag) dep_val = ld_acquire(flag);
+  __device__ void issue(const WG &w) {
+    n1_issued = false;
+    if (n1.valid && dep_val >= dep_target) {
+      issue_copy(n1, w);
+      n1_issued = true;
     }
     pos2 = atomicAdd(a.counters, 1);
   }
 
-  __device__ void publish() {  // thread rho == 0, before the first epilogue barrier
-    publish_pending();  // the previous item's stores were issued long ago
-    box->pass = c_valid ? c_pass : -1;
-    box->item = c_item;
-    box->chunk = c_chunk;
-    box->ready = (dep_val >= dep_target) ? 1 : 0;
-    take_claim(pos2);
-  }
-
-  __device__ void load(int pass, long long item) {
-    if (pass == 0)
-      load_row<G1>(a.p[0], item, true, ul1[0], q1[0], x);
-    else
-      load_row<G2>(a.p[1], item, true, ul1[1], q1[1], x);
-  }
-
-  __device__ void prefetch() {  // every thread, after the barrier following publish()
-    npass = box->pass;
-    nitem = box->item;
-    nchunk = box->chunk;
-    loaded = false;
-    if (npass >= 0 && box->ready) {
-      load(npass, nitem);
-      loaded = true;
-    }
+  __device__ void publish() {
+    publish_pending();
+    box->item = n1.item;
+    box->pass = n1.valid ? n1.pass : -1;
+    box->chunk = n1.chunk;
+    box->issued = n1_issued ? 1 : 0;
+    n1 = decode(pos2);
+    read_dep(n1);
   }
 };
 
 template <int R, int PREC, int S1, int S2>
 __global__ void __launch_bounds__(Geo<R, S1, S2, kFirst>::THREADS, 1)
-    dft_fused_kernel(const GArgs a) {
+    dft_fused_kernel(const __grid_constant__ GArgs a) {
   static_assert(S1 >= 2 && S2 >= 2, "the fused schedule needs an SMEM barrier per item");
   using G1 = Geo<R, S1, S2, kFirst>;
   using G2 = Geo<R, S2, S1, kSecond>;
@@ -656,62 +744,71 @@ __global__ void __launch_bounds__(Geo<R, S1, S2, kFirst>::THREADS, 1)
   float2 *tw1 = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
   float2 *tw2 = reinterpret_cast<float2 *>(smem + SM::OFF_TW2);
   uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + SM::OFF_BAR);
-  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + NWG);
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 3 * NWG);
   FusedSched *boxes = reinterpret_cast<FusedSched *>(smem + SM::OFF_SCHED);
   const uint32_t tbase = kernel_setup<NWG, G1::THREADS>(
       a.bimg, (int)(SM::IMG / 4), reinterpret_cast<float *>(smem), a.p[0].tw_stage, tw1,
       G1::TW_ENTRIES, a.p[1].tw_stage, tw2, G2::TW_ENTRIES, mbar, tmem_slot);
   WG w;
-  init_wg<NWG, G1::GCOLS>(w, tbase, smem, SM::OFF_BAR, SM::OFF_BUF, SM::BUF_PTS);
+  init_wg<R, SM, G1::GCOLS>(w, tbase, smem);
   const int wg = threadIdx.x >> 7;
+  FusedSched *box = boxes + wg;
 
-  float2 x[R];
-  FusedNext<G1, G2> nx{a, boxes + wg};
-  nx.x = x;
+  FusedNext<G1, G2> nx{a, box};
   nx.pend_flag = nullptr;
-  row_of<G1>(G1::MODE_FIRST, w.rho, nx.ul1[0], nx.q1[0]);
-  row_of<G2>(G2::MODE_FIRST, w.rho, nx.ul1[1], nx.q1[1]);
+  nx.n1_issued = false;
 
-  // first item: claim it and the one after, wait for its dependencies
+  // first item: claim it, wait for its dependencies, issue its copy; claim
+  // the one after and start reading its dependency
   bool f = false;
   if (w.rho == 0) {
-    nx.take_claim(atomicAdd(a.counters, 1));
-    nx.dep_val = 1;
-    nx.dep_target = 0;
-    if (nx.c_valid && !nx.wait_deps(nx.c_pass, nx.c_item, nx.c_chunk)) f = true;
-    nx.pos2 = atomicAdd(a.counters, 1);
-    nx.publish();
+    const QItem first = nx.decode(atomicAdd(a.counters, 1));
+    if (first.valid) {
+      if (!nx.wait_deps(first)) f = true;
+      else nx.issue_copy(first, w);
+    }
+    box->item = first.item;
+    box->pass = first.valid ? first.pass : -1;
+    box->chunk = first.chunk;
+    box->issued = first.valid && !f;
+    nx.n1 = nx.decode(atomicAdd(a.counters, 1));
+    nx.read_dep(nx.n1);
   }
   if (named_bar_or(w.bar_id, 128, f)) w.fail = true;
-  if (!w.fail) nx.prefetch();
 
-  while (!w.fail && nx.npass >= 0) {
-    const int pass = nx.npass, chunk = nx.nchunk;
-    const long long item = nx.nitem;
-    if (pass == 0)
-      process_item<G1, PREC, true>(a.p[0], tw1, item, x, w, nx);
-    else
-      process_item<G2, PREC, false>(a.p[1], tw2, item, x, w, nx);
-    if (w.fail) break;
-    // completion is published during the next item (after its first
-    // barrier), or below
-    if (w.rho == 0)
-      nx.pend_flag = (pass == 0) ? a.counters + 1 + ((item << G1::LOG2GG) >> G1::LOG2UPER)
-                                 : a.counters + 1 + a.batch + chunk;
-    if (nx.npass >= 0 && !nx.loaded) {
-      bool ff = false;
-      // publish our own completion first: the item we wait for may need it
-      if (named_bar_or(w.bar_id, 128, false)) ff = true;
+  bool stg_pending = false;
+  while (!w.fail) {
+    const long long item = box->item;
+    const int pass = box->pass, chunk = box->chunk;
+    const bool issued = box->issued != 0;
+    if (pass < 0) break;
+    if (!issued) {
+      // its dependency was not ready at issue time: publish our own last
+      // completion (it may be what it waits for; the barrier orders every
+      // thread's stores of it first), wait, then copy
+      bool ff = named_bar_or(w.bar_id, 128, false);
       if (w.rho == 0) {
         nx.publish_pending();
-        if (!nx.wait_deps(nx.npass, nx.nitem, nx.nchunk)) ff = true;
+        const QItem q{item, pass, chunk, true};
+        if (!nx.wait_deps(q)) ff = true;
+        else nx.issue_copy(q, w);
       }
       if (named_bar_or(w.bar_id, 128, ff)) {
         w.fail = true;
         break;
       }
-      nx.load(nx.npass, nx.nitem);
     }
+    if (pass == 0)
+      process_item<G1, PREC, true>(a.p[0], &a.tm_tw, tw1, item, w, nx);
+    else
+      process_item<G2, PREC, false>(a.p[1], &a.tm_tw, tw2, item, w, nx);
+    stg_pending = nx.n1_issued;
+    if (w.fail) break;
+    // the mailbox now names the next item; its completion is published
+    // during the next item (after its first barrier), or below
+    if (w.rho == 0)
+      nx.pend_flag = (pass == 0) ? a.counters + 1 + ((item << G1::LOG2GG) >> G1::LOG2UPER)
+                                 : a.counters + 1 + a.batch + chunk;
   }
   // all stores of this warpgroup are issued: publish the last completion
   named_bar_or(w.bar_id, 128, false);
@@ -719,7 +816,7 @@ __global__ void __launch_bounds__(Geo<R, S1, S2, kFirst>::THREADS, 1)
     nx.publish_pending();
     if (w.fail) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);
   }
-  kernel_teardown(tbase);
+  kernel_teardown(tbase, w, w.fail && stg_pending, w.fail && w.tws_inflight);
 }
 
 }  // namespace tcu

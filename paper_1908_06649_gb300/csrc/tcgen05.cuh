@@ -177,4 +177,40 @@ __device__ __forceinline__ bool named_bar_or(int id, int count, bool v) {
   return out != 0;
 }
 
+// ------------------------------------------------------------------ TMA
+// Arm `mbar` for `bytes` of asynchronous copies (one arrival).
+__device__ __forceinline__ void mbar_expect_tx(uint32_t mbar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(mbar),
+               "r"(bytes)
+               : "memory");
+}
+
+// Bulk copy global -> shared (both 16-byte aligned, bytes % 16 == 0),
+// completion counted on `mbar`.
+__device__ __forceinline__ void tma_load_1d(uint32_t smem_dst, const void *gsrc,
+                                            uint32_t bytes, uint32_t mbar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, "
+      "[%3];" ::"r"(smem_dst),
+      "l"(gsrc), "r"(bytes), "r"(mbar)
+      : "memory");
+}
+
+// Tiled tensor copy global -> shared of one box at coordinates (c0, c1, c2);
+// `tmap` points to a CUtensorMap in parameter or global memory.
+__device__ __forceinline__ void tma_load_3d(uint32_t smem_dst, const void *tmap, int c0,
+                                            int c1, int c2, uint32_t mbar) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes "
+      "[%0], [%1, {%2, %3, %4}], [%5];" ::"r"(smem_dst),
+      "l"(tmap), "r"(c0), "r"(c1), "r"(c2), "r"(mbar)
+      : "memory");
+}
+
+// Order this thread's earlier generic-proxy accesses (e.g. an acquire of a
+// flag) before its later async-proxy (TMA) accesses of global memory.
+__device__ __forceinline__ void fence_proxy_async_global() {
+  asm volatile("fence.proxy.async.global;" ::: "memory");
+}
+
 }  // namespace tcu

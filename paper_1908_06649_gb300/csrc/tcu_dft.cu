@@ -25,6 +25,8 @@
 // warpgroup passes of >= 2 stages each run fused in one launch with an
 // L2-resident intermediate.
 
+#include <cuda.h>
+#include <cudaTypedefs.h>
 #include <cuda_runtime.h>
 #include <stdint.h>
 #include <stdio.h>
@@ -82,6 +84,7 @@ struct tcu_dft_plan_s {
   float *bimg[2];          // [dir index] hi | lo images
   float2 *twA[2], *twB[2]; // tile kernel pass 1: two-level w_n^e
   float2 *tw_out[2];       // group kernel pass 1: w_n^{b k} as [k][b]
+  CUtensorMap tw_map[2];   // TMA map of tw_out[d]
   float2 *scratch;         // intermediate (full size, or the fused ring)
   // fused two-pass schedule
   bool fused;
@@ -96,6 +99,39 @@ struct tcu_dft_plan_s {
 namespace {
 
 int dir_index(int dir) { return dir == TCU_DFT_INVERSE ? 1 : 0; }
+
+// cuTensorMapEncodeTiled from the driver, through the runtime (no -lcuda).
+PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  if (!fn) {
+    void *p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000,
+                                         cudaEnableDefault, &q) == cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = (PFN_cuTensorMapEncodeTiled_v12000)p;
+    else
+      cudaGetLastError();
+  }
+  return fn;
+}
+
+// TMA map of a [depth][rows][cols] array of complex64 (cols contiguous, row
+// pitch cols, plane pitch plane_elems), seen as fp32 pairs; boxes of
+// box_cols complex x box_rows rows x 1 plane.
+bool encode_map(CUtensorMap *m, const void *base, long long cols, long long rows,
+                long long depth, long long plane_elems, int box_cols, int box_rows) {
+  PFN_cuTensorMapEncodeTiled_v12000 enc = tensor_map_encoder();
+  if (!enc) return false;
+  const cuuint64_t dims[3] = {(cuuint64_t)(2 * cols), (cuuint64_t)rows, (cuuint64_t)depth};
+  const cuuint64_t strides[2] = {(cuuint64_t)(cols * 8), (cuuint64_t)(plane_elems * 8)};
+  const cuuint32_t box[3] = {(cuuint32_t)(2 * box_cols), (cuuint32_t)box_rows, 1};
+  const cuuint32_t estr[3] = {1, 1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 3, const_cast<void *>(base), dims,
+             strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
 
 // Round an fp32 value to TF32 (10 explicit mantissa bits), nearest, ties away
 // from zero -- the same rule as PTX cvt.rna.tf32.f32.
@@ -348,6 +384,18 @@ int other_stages(const tcu_dft_plan_s *p, int pi) {
   return p->npasses == 1 ? 0 : p->pass[1 - pi].s;
 }
 
+// TMA maps of a first (strided) warpgroup pass: its input x[b][a][v] and
+// its inter-pass twiddles.
+bool first_pass_maps(const tcu_dft_plan_s *p, int di, const void *in, GArgs *g) {
+  const PassPlan &p1 = p->pass[0];
+  const long long n1 = 1ll << p1.log2L, n2 = p->n / n1;
+  const long long gg1 = (128ll * p->r) >> p1.log2L;
+  const int box_rows = n1 < 256 ? (int)n1 : 256;
+  if (!encode_map(&g->tm_in, in, n2, n1, p->batch, p->n, (int)gg1, box_rows)) return false;
+  g->tm_tw = p->tw_map[di];
+  return true;
+}
+
 }  // namespace
 
 extern "C" {
@@ -512,6 +560,11 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
         for (long long k1 = 0; k1 < n1; ++k1)
           for (long long b = 0; b < n2; ++b) t[(size_t)(k1 * n2 + b)] = root(b * k1, n, sign);
         rc = upload(&p->tw_out[d], t);
+        const long long gg1 = (128ll * r) >> p->pass[0].log2L;
+        const int box_rows = n1 < 256 ? (int)n1 : 256;
+        if (rc == TCU_DFT_OK &&
+            !encode_map(&p->tw_map[d], p->tw_out[d], n2, n1, 1, n, (int)gg1, box_rows))
+          rc = TCU_DFT_ERR_CUDA;
       }
     }
   }
@@ -583,6 +636,7 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
     const long long ring_mask = ((long long)p->ring_chunks << p->log2C) - 1;
     g.p[0] = group_pass(p, 0, di, (const float2 *)in, p->scratch, -1, ring_mask, inverse);
     g.p[1] = group_pass(p, 1, di, p->scratch, (float2 *)out, ring_mask, -1, inverse);
+    if (!first_pass_maps(p, di, in, &g)) return TCU_DFT_ERR_CUDA;
     g.bimg = p->bimg[di];
     g.err = p->err;
     g.counters = p->counters;
@@ -618,6 +672,8 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
       GArgs g;
       memset(&g, 0, sizeof(g));
       g.p[0] = group_pass(p, pi, di, src, dst, -1, -1, inverse);
+      if (pass_role(p, pi) == kFirst && !first_pass_maps(p, di, src, &g))
+        return TCU_DFT_ERR_CUDA;
       g.bimg = p->bimg[di];
       g.err = p->err;
       if (pass_dispatch(p->r, p->precision, pp.s, other_stages(p, pi), pass_role(p, pi), g,
