@@ -217,8 +217,9 @@ def main():
     ap.add_argument("--ref-sample", type=int, default=16)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--e2e-steps", type=int, default=20)
-    ap.add_argument("--no-fuse", action="store_true",
-                    help="two separate pass launches instead of the fused one")
+    ap.add_argument("--fuse", action="store_true",
+                    help="one fused launch with an L2-resident intermediate "
+                         "instead of two pass launches")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (profiling cases)")
     args = ap.parse_args()
@@ -254,7 +255,7 @@ def main():
     x = torch.from_numpy(x_host).to(dev)
     y = torch.empty_like(x)
     plan = pkg.Plan(n, batch, r, args.precision,
-                    pkg.PLAN_NO_FUSE if args.no_fuse else pkg.PLAN_DEFAULT)
+                    pkg.PLAN_FUSE if args.fuse else pkg.PLAN_DEFAULT)
     npass = len(plan.passes())
     stream = torch.cuda.current_stream()
 

@@ -71,17 +71,21 @@ enum {
 tcu_dft_plan_t tcu_dft_plan(int64_t n, int64_t batch, int32_t sqrt_m,
                             int32_t precision);
 
-/* Plan flags for tcu_dft_plan_ex. */
+/* Plan flags for tcu_dft_plan_ex.  By default a two-pass transform runs as
+ * two kernel launches with a full batch*n intermediate in HBM. */
 enum {
   TCU_DFT_PLAN_DEFAULT = 0,
-  /* Run a two-pass transform as two separate kernel launches with a full
-   * batch*n intermediate in HBM, instead of the single fused launch whose
-   * intermediate is a small ring kept in L2. */
-  TCU_DFT_PLAN_NO_FUSE = 1
+  /* Explicitly the default two-launch schedule. */
+  TCU_DFT_PLAN_NO_FUSE = 1,
+  /* Run both passes in ONE fused launch whose intermediate is a small ring
+   * of transforms kept in L2 (HBM then moves each point once in and once
+   * out).  Only for two passes of >= 2 stages each; otherwise ignored. */
+  TCU_DFT_PLAN_FUSE = 2
 };
 
-/* tcu_dft_plan with scheduling flags (TCU_DFT_PLAN_*); unknown bits are
- * rejected with ERR_INVALID.  Same results either way. */
+/* tcu_dft_plan with scheduling flags (TCU_DFT_PLAN_*); unknown bits, or
+ * FUSE together with NO_FUSE, are rejected with ERR_INVALID.  Same results
+ * either way. */
 tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
                                int32_t precision, uint32_t flags);
 

@@ -31,6 +31,7 @@ ERR_TIMEOUT = 5
 
 PLAN_DEFAULT = 0
 PLAN_NO_FUSE = 1
+PLAN_FUSE = 2
 
 SYMBOLS = (
     "tcu_dft_plan", "tcu_dft_plan_ex", "tcu_dft_is_fused", "tcu_dft_exec",

@@ -423,7 +423,8 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
                                int32_t precision, uint32_t flags) {
   g_last_error = TCU_DFT_OK;
   if (n < 1 || batch < 1 || (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32) ||
-      (flags & ~(uint32_t)TCU_DFT_PLAN_NO_FUSE)) {
+      (flags & ~(uint32_t)(TCU_DFT_PLAN_NO_FUSE | TCU_DFT_PLAN_FUSE)) ||
+      ((flags & TCU_DFT_PLAN_NO_FUSE) && (flags & TCU_DFT_PLAN_FUSE))) {
     g_last_error = TCU_DFT_ERR_INVALID;
     return nullptr;
   }
@@ -578,7 +579,7 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
   if (rc == TCU_DFT_OK && npasses == 2) {
     const PassPlan &p1 = p->pass[0], &p2 = p->pass[1];
     p->fused = p1.kind == kGroupPass && p2.kind == kGroupPass && p1.s >= 2 && p2.s >= 2 &&
-               !(flags & TCU_DFT_PLAN_NO_FUSE);
+               (flags & TCU_DFT_PLAN_FUSE);
     long long scratch_tf = batch;
     if (p->fused) {
       // chunks of C transforms (a power of two dividing the batch, <= 8);

@@ -59,7 +59,9 @@ def test_strerror_and_null_handling(lib):
     assert lib.tcu_dft_check(None, None) == pkg.ERR_INVALID
     assert lib.tcu_dft_num_passes(None) == -1
     assert lib.tcu_dft_is_fused(None) == -1
-    assert not lib.tcu_dft_plan_ex(256, 4, 16, 3, 2)   # unknown flag bit
+    assert not lib.tcu_dft_plan_ex(256, 4, 16, 3, 4)   # unknown flag bit
+    assert lib.tcu_dft_last_error() == pkg.ERR_INVALID
+    assert not lib.tcu_dft_plan_ex(256, 4, 16, 3, 3)   # FUSE with NO_FUSE
     assert lib.tcu_dft_last_error() == pkg.ERR_INVALID
     assert lib.tcu_dft_pass_stages(None, 0) == -1
 

@@ -26,10 +26,10 @@ def pkg():
     return p
 
 
-def run(pkg, x, r, prec, inverse=False, inplace=False):
+def run(pkg, x, r, prec, inverse=False, inplace=False, flags=0):
     import torch
     batch, n = x.shape
-    plan = pkg.Plan(n, batch, r, prec)
+    plan = pkg.Plan(n, batch, r, prec, flags)
     xd = torch.from_numpy(np.ascontiguousarray(x)).cuda()
     if inplace:
         y = plan.exec(xd, xd, pkg.INVERSE if inverse else pkg.FORWARD)
@@ -80,12 +80,32 @@ def test_single_pass(pkg, r, k, prec):
                                        (16, 6, 1), (8, 7, 1),
                                        (16, 4, 40), (8, 5, 48), (8, 6, 12)])
 @pytest.mark.parametrize("prec", [3, 1])
-def test_two_pass(pkg, r, k, batch, prec):
+@pytest.mark.parametrize("fuse", [False, True])
+def test_two_pass(pkg, r, k, batch, prec, fuse):
     n = r ** k
     x = inputs.make("uniform", n, batch, seed=20 + k)
-    y, passes = run(pkg, x, r, prec)
+    y, passes = run(pkg, x, r, prec, flags=pkg.PLAN_FUSE if fuse else 0)
     assert len(passes) == 2 and sum(passes) == k
     check(y, x, prec)
+
+
+@pytest.mark.parametrize("r,k", [(16, 4), (8, 5), (8, 6), (32, 4)])
+def test_fused_schedule_is_used(pkg, r, k):
+    n = r ** k
+    plan = pkg.Plan(n, 2, r, 3, pkg.PLAN_FUSE)
+    assert plan.fused
+    plan.destroy()
+    plan = pkg.Plan(n, 2, r, 3)
+    assert not plan.fused
+    plan.destroy()
+
+
+@pytest.mark.parametrize("r,k", [(16, 2), (16, 4), (8, 5)])
+def test_inverse_fused(pkg, r, k):
+    n = r ** k
+    x = inputs.make("normal", n, 16, seed=9)
+    y, _ = run(pkg, x, r, 3, inverse=True, flags=pkg.PLAN_FUSE)
+    check(y, x, 3, inverse=True)
 
 
 @pytest.mark.parametrize("r,k", [(16, 2), (16, 4), (8, 5), (32, 3)])
