@@ -54,7 +54,8 @@ enum {
   TCU_DFT_ERR_UNSUPPORTED = 2, /* valid but not supported (radix, n not r^k, n too large) */
   TCU_DFT_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed, or no sm_103 device */
   TCU_DFT_ERR_OOM = 4,         /* device allocation failed */
-  TCU_DFT_ERR_TIMEOUT = 5      /* a device-side wait hit its iteration limit */
+  TCU_DFT_ERR_TIMEOUT = 5,     /* a device-side wait hit its iteration limit */
+  TCU_DFT_ERR_TOO_LARGE = 6    /* beyond the fixed memory of tcu_dft_exec_noalloc */
 };
 
 /* Build a plan for `batch` forward/inverse DFTs of length n with radix
@@ -135,6 +136,37 @@ int tcu_dft_destroy(tcu_dft_plan_t p);
  * -1 for a NULL plan or an index out of range. */
 int tcu_dft_num_passes(tcu_dft_plan_t p);
 int tcu_dft_pass_stages(tcu_dft_plan_t p, int i);
+
+/* Transform without allocating: for callers that may not allocate device
+ * memory at all -- code running where memory belongs to someone else (a
+ * framework's pool, a caching allocator, an embedding application) or where
+ * a cudaMalloc would stall the device and break a latency budget.  The paper
+ * has no counterpart; it is a service of this library.
+ *
+ * Same transform and arguments as tcu_dft_plan + tcu_dft_exec_dir, without
+ * a plan: in, out are caller-owned device buffers of batch*n complex64
+ * (16-byte aligned, in == out allowed), dir is TCU_DFT_FORWARD or
+ * TCU_DFT_INVERSE, stream a cudaStream_t.  Every buffer it uses besides in
+ * and out is a fixed array inside the library (the two-pass intermediate:
+ * 4 Mi complex64 = 32 MiB; twiddle and F_r tables for n <= 2^18), present on
+ * every GPU that loads the library until the process exits.  It never calls
+ * cudaMalloc or cudaFree.
+ *
+ * Limits: n a power of sqrt_m whose stages fit two warpgroup passes (sqrt_m
+ * 16: n <= 16^4; 8: n <= 8^6; 32: n <= 32^3) and n <= 2^18; when n needs two
+ * passes, batch*n <= 2^22.  Larger requests return TCU_DFT_ERR_TOO_LARGE
+ * with nothing launched; other argument errors ERR_INVALID / ERR_UNSUPPORTED
+ * as tcu_dft_plan would.
+ *
+ * The first call on a device resolves the device addresses of those arrays
+ * (with that device current) and fills the tables; make that first call
+ * before any stream capture.  A later call with another n or sqrt_m refills
+ * the tables, stream-ordered on `stream`.  All calls share the arrays, which
+ * keep the last call's contents: calls whose work overlaps on the GPU (other
+ * streams, other host threads) race with each other.  Asynchronous like
+ * tcu_dft_exec_dir; a device-side wait timeout is not reported here. */
+int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t precision,
+                         const void *in, void *out, int dir, void *stream);
 
 /* Status of the last tcu_dft_plan call on this thread. */
 int tcu_dft_last_error(void);

@@ -28,6 +28,7 @@ ERR_UNSUPPORTED = 2
 ERR_CUDA = 3
 ERR_OOM = 4
 ERR_TIMEOUT = 5
+ERR_TOO_LARGE = 6
 
 PLAN_DEFAULT = 0
 PLAN_NO_FUSE = 1
@@ -36,7 +37,7 @@ PLAN_FUSE = 2
 SYMBOLS = (
     "tcu_dft_plan", "tcu_dft_plan_ex", "tcu_dft_is_fused", "tcu_dft_exec",
     "tcu_dft_exec_dir", "tcu_dft_exec_timed",
-    "tcu_dft_exec_host",
+    "tcu_dft_exec_host", "tcu_dft_exec_noalloc",
     "tcu_dft_check", "tcu_dft_destroy", "tcu_dft_num_passes",
     "tcu_dft_pass_stages", "tcu_dft_last_error", "tcu_dft_strerror",
 )
@@ -81,6 +82,9 @@ def lib():
     L.tcu_dft_exec_timed.restype = ctypes.c_int
     L.tcu_dft_exec_host.argtypes = [vp, vp, vp, vp, ctypes.c_int, vp]
     L.tcu_dft_exec_host.restype = ctypes.c_int
+    L.tcu_dft_exec_noalloc.argtypes = [i64, i64, i32, i32, vp, vp, ctypes.c_int,
+                                       vp]
+    L.tcu_dft_exec_noalloc.restype = ctypes.c_int
     L.tcu_dft_check.argtypes = [vp, vp]
     L.tcu_dft_check.restype = ctypes.c_int
     L.tcu_dft_destroy.argtypes = [vp]
@@ -109,6 +113,30 @@ def _stream_handle(stream):
     if stream is None:
         stream = torch.cuda.current_stream()
     return ctypes.c_void_p(stream.cuda_stream)
+
+
+def exec_noalloc(x, out, n: int, batch: int, sqrt_m: int = 16,
+                 precision: int = X3TF32, direction: int = FORWARD, stream=None):
+    """tcu_dft_exec_noalloc: the transform without a plan and without any
+    device allocation, for callers that must not allocate (its working
+    memory is a fixed array inside the library; see include/tcu_dft.h for
+    the size limits).  x, out: contiguous complex64 CUDA tensors of batch*n
+    elements.  Returns out."""
+    import torch
+    for t, nm in ((x, "x"), (out, "out")):
+        if (not isinstance(t, torch.Tensor) or t.dtype != torch.complex64
+                or not t.is_cuda or not t.is_contiguous()
+                or t.numel() != n * batch):
+            raise ValueError("%s must be a contiguous complex64 CUDA tensor "
+                             "of batch*n elements" % nm)
+    rc = lib().tcu_dft_exec_noalloc(int(n), int(batch), int(sqrt_m),
+                                    int(precision),
+                                    ctypes.c_void_p(x.data_ptr()),
+                                    ctypes.c_void_p(out.data_ptr()),
+                                    int(direction), _stream_handle(stream))
+    if rc != OK:
+        raise TcuDftError(rc, "tcu_dft_exec_noalloc")
+    return out
 
 
 class Plan:

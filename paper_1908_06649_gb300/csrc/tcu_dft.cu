@@ -34,6 +34,7 @@
 #include <string.h>
 
 #include <cmath>
+#include <mutex>
 #include <vector>
 
 #include "../../include/tcu_dft.h"
@@ -396,6 +397,36 @@ bool first_pass_maps(const tcu_dft_plan_s *p, int di, const void *in, GArgs *g) 
   return true;
 }
 
+// ------------------------------------------- fixed memory of exec_noalloc
+// tcu_dft_exec_noalloc keeps everything besides the caller's buffers in
+// these file-scope arrays.  In host code their names are only stand-ins:
+// kernels get the device addresses resolved by cudaGetSymbolAddress.
+constexpr long long kNaMaxPoints = 1ll << 22;      // two-pass intermediate
+constexpr long long kNaMaxN = 1ll << 18;           // longest transform
+constexpr int kNaImgFloats = 4 * 16 * 32 * 32 / 4;  // 4 F_r images, r <= 32
+constexpr int kNaStageTw = 1024;                    // stage twiddles of a pass
+static __device__ __align__(256) float2 g_na_scratch[kNaMaxPoints];
+static __device__ __align__(256) float g_na_img[2][kNaImgFloats];
+static __device__ __align__(256) float2 g_na_tw_stage[2][2][kNaStageTw];
+static __device__ __align__(256) float2 g_na_tw_out[2][kNaMaxN];
+static __device__ __align__(256) int g_na_err;
+
+struct NaDevice {
+  bool ready;  // device addresses resolved
+  int num_sms;
+  float2 *scratch;
+  float *img;
+  float2 *tw_stage;
+  float2 *tw_out;
+  int *err;
+  long long n;  // tables currently held (0: none)
+  int r;
+  CUtensorMap tw_map[2];
+};
+
+std::mutex g_na_mutex;
+NaDevice g_na_dev[64];
+
 }  // namespace
 
 extern "C" {
@@ -408,6 +439,8 @@ const char *tcu_dft_strerror(int status) {
     case TCU_DFT_ERR_CUDA: return "CUDA error";
     case TCU_DFT_ERR_OOM: return "device allocation failed";
     case TCU_DFT_ERR_TIMEOUT: return "device wait timed out";
+    case TCU_DFT_ERR_TOO_LARGE:
+      return "size exceeds the fixed memory of tcu_dft_exec_noalloc";
     default: return "unknown status";
   }
 }
@@ -770,6 +803,155 @@ int tcu_dft_is_fused(tcu_dft_plan_t p) { return p ? (p->fused ? 1 : 0) : -1; }
 int tcu_dft_pass_stages(tcu_dft_plan_t p, int i) {
   if (!p || i < 0 || i >= p->npasses) return -1;
   return p->pass[i].s;
+}
+
+int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t precision,
+                         const void *in, void *out, int dir, void *stream) {
+  // ---- arguments (no CUDA call before they are known to be good)
+  if (n < 1 || batch < 1 || (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32) ||
+      !in || !out || (dir != TCU_DFT_FORWARD && dir != TCU_DFT_INVERSE))
+    return TCU_DFT_ERR_INVALID;
+  if (sqrt_m != 8 && sqrt_m != 16 && sqrt_m != 32) return TCU_DFT_ERR_UNSUPPORTED;
+  const int r = sqrt_m, log2r = ilog2(r);
+  int k = 0;
+  long long m = 1;
+  while (m < n) {
+    m *= r;
+    ++k;
+  }
+  if (m != n) return TCU_DFT_ERR_UNSUPPORTED;
+  const int sg = max_group_stages(r);
+  if (k > 2 * sg || n > kNaMaxN) return TCU_DFT_ERR_TOO_LARGE;
+  const int npasses = k <= sg ? 1 : 2;
+  if (npasses == 2 && batch * n > kNaMaxPoints) return TCU_DFT_ERR_TOO_LARGE;
+  int stages[2] = {k, 0};
+  if (npasses == 2) {
+    stages[0] = (k + 1) / 2;
+    stages[1] = k - stages[0];
+  }
+  const int log2n = ilog2(n);
+  cudaStream_t st = (cudaStream_t)stream;
+
+  std::lock_guard<std::mutex> lock(g_na_mutex);
+  int dev = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+    cudaGetLastError();
+    return TCU_DFT_ERR_CUDA;
+  }
+  NaDevice &D = g_na_dev[dev];
+  if (!D.ready) {
+    // once per device, with it current: where the fixed arrays live
+    cudaDeviceProp prop;
+    if (cudaGetDeviceProperties(&prop, dev) != cudaSuccess || prop.major != 10 ||
+        prop.minor != 3 ||
+        cudaGetSymbolAddress((void **)&D.scratch, g_na_scratch) != cudaSuccess ||
+        cudaGetSymbolAddress((void **)&D.img, g_na_img) != cudaSuccess ||
+        cudaGetSymbolAddress((void **)&D.tw_stage, g_na_tw_stage) != cudaSuccess ||
+        cudaGetSymbolAddress((void **)&D.tw_out, g_na_tw_out) != cudaSuccess ||
+        cudaGetSymbolAddress((void **)&D.err, g_na_err) != cudaSuccess) {
+      cudaGetLastError();
+      return TCU_DFT_ERR_CUDA;
+    }
+    D.num_sms = prop.multiProcessorCount;
+    D.n = 0;
+    D.ready = true;
+  }
+
+  // ---- the plan, on the stack, pointing into the fixed arrays
+  tcu_dft_plan_s p;
+  memset(&p, 0, sizeof(p));
+  p.n = n;
+  p.batch = batch;
+  p.r = r;
+  p.log2r = log2r;
+  p.k = k;
+  p.precision = precision;
+  p.npasses = npasses;
+  p.num_sms = D.num_sms;
+  p.device = dev;
+  p.fused = false;
+  p.scratch = D.scratch;
+  p.err = D.err;
+  for (int d = 0; d < 2; ++d) {
+    p.bimg[d] = D.img + (size_t)d * kNaImgFloats;
+    p.tw_out[d] = D.tw_out + (size_t)d * kNaMaxN;
+  }
+  for (int pi = 0; pi < npasses; ++pi) {
+    PassPlan &pp = p.pass[pi];
+    pp.kind = kGroupPass;
+    pp.s = stages[pi];
+    pp.log2L = log2r * pp.s;
+    pp.last = (pi == npasses - 1);
+    const long long L = 1ll << pp.log2L;
+    if (npasses == 1) {
+      pp.U = batch;
+      pp.Uper = 1;
+      pp.in_vstride = n;
+      pp.in_stride = 1;
+      pp.out_vstride = n;
+      pp.out_stride = 1;
+    } else if (pi == 0) {
+      pp.U = batch * (n / L);
+      pp.Uper = n / L;
+      pp.in_vstride = 1;
+      pp.in_stride = n / L;
+      pp.out_vstride = 1;
+      pp.out_stride = n / L;
+    } else {
+      pp.U = batch * (n / L);
+      pp.Uper = n / L;
+      pp.in_vstride = L;
+      pp.in_stride = 1;
+      pp.out_vstride = 1;
+      pp.out_stride = n / L;
+    }
+    pp.log2Uper = ilog2(pp.Uper);
+    pp.modes[0] = pp.in_stride == 1 ? kQF : kUF;
+    pp.modes[1] = kUF;
+    pp.modes[2] = pp.out_stride == 1 ? kRQF : kUF;
+    pp.swz_tab = choose_swizzle(r, pp.s, pp.modes);
+    for (int d = 0; d < 2; ++d)
+      pp.tw_stage[d] = D.tw_stage + ((size_t)d * 2 + pi) * kNaStageTw;
+  }
+
+  // ---- tables for this (n, r), refilled only when they change
+  if (D.n != n || D.r != r) {
+    D.n = 0;
+    for (int d = 0; d < 2; ++d) {
+      const int sign = d == 0 ? -1 : 1;
+      std::vector<float> img;
+      build_images(r, sign, log2n, img);
+      if (cudaMemcpyAsync(p.bimg[d], img.data(), img.size() * sizeof(float),
+                          cudaMemcpyHostToDevice, st) != cudaSuccess)
+        return TCU_DFT_ERR_CUDA;
+      for (int pi = 0; pi < npasses; ++pi) {
+        const std::vector<float2> t = stage_twiddles(r, p.pass[pi].s, sign);
+        if (cudaMemcpyAsync(p.pass[pi].tw_stage[d], t.data(), t.size() * sizeof(float2),
+                            cudaMemcpyHostToDevice, st) != cudaSuccess)
+          return TCU_DFT_ERR_CUDA;
+      }
+      if (npasses == 2) {
+        const long long n1 = 1ll << p.pass[0].log2L, n2 = n / n1;
+        std::vector<float2> t((size_t)n);
+        for (long long k1 = 0; k1 < n1; ++k1)
+          for (long long b = 0; b < n2; ++b) t[(size_t)(k1 * n2 + b)] = root(b * k1, n, sign);
+        if (cudaMemcpyAsync(p.tw_out[d], t.data(), t.size() * sizeof(float2),
+                            cudaMemcpyHostToDevice, st) != cudaSuccess)
+          return TCU_DFT_ERR_CUDA;
+        const long long gg1 = (128ll * r) >> p.pass[0].log2L;
+        if (!encode_map(&D.tw_map[d], p.tw_out[d], n2, n1, 1, n, (int)gg1,
+                        n1 < 256 ? (int)n1 : 256))
+          return TCU_DFT_ERR_CUDA;
+      }
+    }
+    D.n = n;
+    D.r = r;
+  }
+  for (int d = 0; d < 2; ++d) p.tw_map[d] = D.tw_map[d];
+
+  // the timeout word must start at zero; then the ordinary two-launch path
+  if (cudaMemsetAsync(D.err, 0, sizeof(int), st) != cudaSuccess) return TCU_DFT_ERR_CUDA;
+  return exec_impl(&p, in, out, dir, stream, nullptr);
 }
 
 }  // extern "C"

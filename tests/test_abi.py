@@ -96,3 +96,26 @@ def test_python_plan_raises(lib):
     with pytest.raises(pkg.TcuDftError) as e:
         pkg.Plan(48, 1, 16)
     assert e.value.status == pkg.ERR_UNSUPPORTED
+
+
+@pytest.mark.parametrize("args,status", [
+    ((0, 1, 16, 3, -1), 1),            # n < 1
+    ((256, 0, 16, 3, -1), 1),          # batch < 1
+    ((256, 1, 16, 2, -1), 1),          # precision
+    ((256, 1, 16, 3, 0), 1),           # direction
+    ((256, 1, 12, 3, -1), 2),          # radix
+    ((48, 1, 16, 3, -1), 2),           # not a power of the radix
+    ((16 ** 5, 1, 16, 3, -1), 6),      # more stages than two warpgroup passes
+    ((32 ** 4, 1, 32, 3, -1), 6),      # n beyond the fixed twiddle table
+    ((65536, 65, 16, 3, -1), 6),       # batch*n beyond the fixed intermediate
+])
+def test_noalloc_rejects_before_cuda(lib, args, status):
+    import ctypes
+    n, batch, r, prec, d = args
+    fake = ctypes.c_void_p(1 << 20)  # never dereferenced: rejected first
+    assert lib.tcu_dft_exec_noalloc(n, batch, r, prec, fake, fake, d, None) == status
+
+
+def test_noalloc_null_buffers(lib):
+    assert lib.tcu_dft_exec_noalloc(256, 1, 16, 3, None, None, -1, None) == 1
+    assert b"fixed memory" in lib.tcu_dft_strerror(6)
