@@ -125,6 +125,65 @@ class ClockSampler:
                 "reasons": sorted(reasons), "samples": len(sm)}
 
 
+def kernel_sources_sha256():
+    """sha256 over the kernel sources (csrc/*.cu, *.cuh, *.h, name order)."""
+    import glob
+    import hashlib
+    csrc = os.path.join(ROOT, "paper_1908_06649_gb300", "csrc")
+    files = sorted(glob.glob(os.path.join(csrc, "*.cu"))
+                   + glob.glob(os.path.join(csrc, "*.cuh"))
+                   + glob.glob(os.path.join(csrc, "*.h")))
+    h = hashlib.sha256()
+    for f in files:
+        h.update(os.path.basename(f).encode())
+        with open(f, "rb") as fh:
+            h.update(fh.read())
+    return h.hexdigest()
+
+
+def profiled_traffic(batch, fused):
+    """DRAM bytes per launch of the dominant kernel from the committed ncu
+    summary, scaled to `batch`; None if the kernel changed since."""
+    if fused:
+        return None
+    p = os.path.join(ROOT, "profiles", "traffic_dft_pass_kernel_n65536.txt")
+    try:
+        kv = {}
+        with open(p) as f:
+            for line in f:
+                if ":" in line and not line.startswith("#"):
+                    k, v = line.split(":", 1)
+                    kv[k.strip()] = v.strip()
+        if kv.get("sources_sha256") != kernel_sources_sha256():
+            return None
+        return (float(kv["dram_bytes_per_launch_b512"]) * batch
+                / float(kv["profiled_batch"]))
+    except Exception:
+        return None
+
+
+def rank_seed(wl, rank):
+    """Each rank transforms its own batch (weak scaling): the workload's
+    recipe with the seed offset by 1000 * rank."""
+    return wl["seed"] + 1000 * rank
+
+
+def max_over_ranks(value, dist, device):
+    """Max of a float over all ranks (the slowest rank sets the job time);
+    identity without a process group."""
+    if dist is None:
+        return float(value)
+    import torch
+    t = torch.tensor([float(value)], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_rate(units_per_rank, world, steps, elapsed_ms):
+    """Whole-job GFLOP/s: the work of every rank over the max time."""
+    return units_per_rank * world * steps / (elapsed_ms * 1e-3) / 1e9
+
+
 def dist_setup():
     world = int(os.environ.get("WORLD_SIZE", "1"))
     rank = int(os.environ.get("RANK", "0"))
@@ -251,7 +310,7 @@ def main():
     n, batch, r = wl["n"], wl["batch"], wl["sqrt_m"]
     log("rank %d: generating %s inputs n=%d batch=%d" % (rank, wl["kind"], n,
                                                        batch))
-    x_host = inputs.make(wl["kind"], n, batch, wl["seed"] + 1000 * rank)
+    x_host = inputs.make(wl["kind"], n, batch, rank_seed(wl, rank))
     x = torch.from_numpy(x_host).to(dev)
     y = torch.empty_like(x)
     plan = pkg.Plan(n, batch, r, args.precision,
@@ -292,13 +351,10 @@ def main():
     elapsed_ms = t_start.elapsed_time(t_end)
     pass_ms = [[ev[i][p].elapsed_time(ev[i][p + 1]) for i in range(K)]
                for p in range(npass)]
-    if dist is not None:
-        t = torch.tensor([elapsed_ms], device=dev, dtype=torch.float64)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        elapsed_ms = float(t.item())
+    elapsed_ms = max_over_ranks(elapsed_ms, dist, dev)
 
     ms_per_step = elapsed_ms / K
-    value = dft_flops(n, batch) * world * K / (elapsed_ms * 1e-3) / 1e9
+    value = job_rate(dft_flops(n, batch), world, K, elapsed_ms)
 
     peaks, peak_kind = load_peaks()
     hbm = float(peaks["hbm_gbs"])
@@ -344,16 +400,14 @@ def main():
         e1.record(stream)
         torch.cuda.synchronize()
         e2e_ms = e0.elapsed_time(e1)
-        if dist is not None:
-            t = torch.tensor([e2e_ms], device=dev, dtype=torch.float64)
-            dist.all_reduce(t, op=dist.ReduceOp.MAX)
-            e2e_ms = float(t.item())
-        e2e = {"value": dft_flops(n, batch) * world * args.e2e_steps
-                        / (e2e_ms * 1e-3) / 1e9,
+        e2e_ms = max_over_ranks(e2e_ms, dist, dev)
+        e2e = {"value": job_rate(dft_flops(n, batch), world, args.e2e_steps,
+                                 e2e_ms),
                "unit": UNIT, "h2d_bytes_per_step": n * batch * 8,
                "d2h_bytes_per_step": n * batch * 8,
                "steps": args.e2e_steps}
 
+    plan_fused = plan.fused
     plan.destroy()
     cpu = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
@@ -368,7 +422,8 @@ def main():
             "data": "synthetic", "config": workload_config(wl, args),
             "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm,
                          "unit": "GB/s", "frac": achieved / hbm,
-                         "traffic": None,
+                         "traffic": profiled_traffic(batch, plan_fused)
+                         if (n == 65536 and r == 16) else None,
                          "kernel": kname,
                          "peak_source": peak_kind,
                          "launch_ms": avg},
