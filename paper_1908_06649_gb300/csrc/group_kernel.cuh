@@ -75,7 +75,8 @@ struct Geo {
   static constexpr bool TW_SMEM = TW_OUT && R != 32;  // twiddles staged by TMA
   static constexpr int TMA_ROWS = L < 256 ? L : 256;  // tensor box height
   static constexpr int Q = (2 * R > 32) ? 2 * R : 32;
-  static constexpr int GCOLS = 3 * Q;
+  // TMEM slot: A_hi (Q) | A_lo (Q) | D (2Q: [A Bhi | A Blo] in 3xTF32)
+  static constexpr int GCOLS = 4 * Q;
   static constexpr int IMG_BYTES = 16 * R * R;
   // entries of the stage twiddle tables: sum over t < S of R * R^(S-t)
   static constexpr int TW_ENTRIES = S == 1 ? 0 : (S == 2 ? R * R : R * R * R + R * R);
@@ -211,32 +212,64 @@ __device__ __forceinline__ void split_store8(const float2 *x, uint32_t col_hi,
 }
 
 // One stage: D = A * Bf for the 128 rows of this warpgroup's slot.
+// 3xTF32: the hi and lo images of Bf lie back to back with the same 8-row
+// group stride, so one N = 4r descriptor covers [Bhi | Blo]; D accumulates
+// lo * [Bhi | Blo] then hi * [Bhi | Blo] (8 products of K = 8, small terms
+// first) and the epilogue adds its two halves: hi Bhi + lo Bhi + hi Blo
+// (+ lo Blo, below fp32 resolution).  One accumulator chain of 2r/8 * 2
+// products instead of three chains' worth (2r/8 * 3) at N = 2r.
 template <int R, int PREC>
 __device__ __forceinline__ void issue_stage_mma(uint32_t slot, uint32_t img_addr) {
   constexpr int Q = (2 * R > 32) ? 2 * R : 32;
-  constexpr int IMG = 16 * R * R, LBO = 128, SBO = 64 * R, KSTEPS = 2 * R / 8;
-  constexpr uint32_t idesc = idesc_tf32(128, 2 * R);
+  constexpr int LBO = 128, SBO = 64 * R, KSTEPS = 2 * R / 8;
+  constexpr uint32_t idesc = idesc_tf32(128, PREC == 3 ? 4 * R : 2 * R);
   const uint32_t ahi = slot, alo = slot + Q, d = slot + 2 * Q;
-  const uint32_t ihi = img_addr, ilo = img_addr + IMG;
   uint32_t acc = 0;
   if (PREC == 3) {
-    // small terms first: lo*Bhi, hi*Blo, then hi*Bhi
 #pragma unroll
     for (int kk = 0; kk < KSTEPS; ++kk) {
-      mma_tf32_ts(d, alo + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO),
+      mma_tf32_ts(d, alo + 8 * kk, smem_desc_noswz(img_addr + kk * 2 * LBO, LBO, SBO),
                   idesc, acc);
       acc = 1;
     }
-#pragma unroll
-    for (int kk = 0; kk < KSTEPS; ++kk)
-      mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(ilo + kk * 2 * LBO, LBO, SBO),
-                  idesc, 1);
   }
 #pragma unroll
   for (int kk = 0; kk < KSTEPS; ++kk) {
-    mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO),
+    mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(img_addr + kk * 2 * LBO, LBO, SBO),
                 idesc, acc);
     acc = 1;
+  }
+}
+
+// This thread's whole D row (2r values) with the TMEM loads batched under
+// one wait per 64 columns; in 3xTF32 the sum of the [A Bhi] and [A Blo]
+// halves.
+template <class G, int PREC>
+__device__ __forceinline__ void load_d_row(const WG &w, float *d) {
+  constexpr int R = 1 << G::LOG2R;
+  const uint32_t base = w.slot + 2 * G::Q + w.lane_off;
+  if (PREC == 3) {
+    if (R == 8) {
+      float v[32];
+      tmem_ld16x2(base, base + 16, v);
+#pragma unroll
+      for (int i = 0; i < 16; ++i) d[i] = v[i] + v[16 + i];
+    } else {
+#pragma unroll
+      for (int c = 0; c < 2 * R; c += 32) {
+        float v[64];
+        tmem_ld32x2(base + c, base + 2 * R + c, v);
+#pragma unroll
+        for (int i = 0; i < 32; ++i) d[c + i] = v[i] + v[32 + i];
+      }
+    }
+  } else {
+    if (R == 8) {
+      tmem_ld16(base, d);
+    } else {
+#pragma unroll
+      for (int c = 0; c < 2 * R; c += 32) tmem_ld32(base + c, d + c);
+    }
   }
 }
 
@@ -301,7 +334,7 @@ __device__ __forceinline__ void staged_row(const WG &w, float2 *x) {
 }
 
 // Epilogue of stage T < S: D -> registers, stage twiddle, transposed write.
-template <class G, int T>
+template <class G, int PREC, int T>
 __device__ __forceinline__ void stage_epilogue(const PRun &P, const float2 *tws,
                                                const WG &w) {
   constexpr int R = 1 << G::LOG2R;
@@ -314,16 +347,12 @@ __device__ __forceinline__ void stage_epilogue(const PRun &P, const float2 *tws,
   const int base = (ul << G::LOG2L) + (hi << (SH + G::LOG2R)) + lo;
   const uint32_t tabv = (uint32_t)(P.swz_tab >> (4 * (ul & 15))) & 15u;
   const float2 *twrow = tws + TWOFF + lo;  // [j][lo], row length R^(S-T)
+  float d[2 * R];
+  load_d_row<G, PREC>(w, d);
 #pragma unroll
-  for (int c = 0; c < R; c += 8) {
-    float d[16];
-    tmem_ld16(w.slot + 2 * G::Q + w.lane_off + 2 * c, d);
-#pragma unroll
-    for (int jj = 0; jj < 8; ++jj) {
-      const int j = c + jj;
-      const float2 y = cmul(make_float2(d[2 * jj], d[2 * jj + 1]), twrow[j << SH]);
-      w.buf[gswz(base + (j << SH), tabv)] = y;
-    }
+  for (int j = 0; j < R; ++j) {
+    const float2 y = cmul(make_float2(d[2 * j], d[2 * j + 1]), twrow[j << SH]);
+    w.buf[gswz(base + (j << SH), tabv)] = y;
   }
 }
 
@@ -348,7 +377,7 @@ __device__ __forceinline__ void stage_rows(const PRun &P, const WG &w) {
 }
 
 // Last stage: D -> registers -> natural-order output.
-template <class G, bool OUT_L2>
+template <class G, int PREC, bool OUT_L2>
 __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, WG &w) {
   constexpr int R = 1 << G::LOG2R;
   constexpr int S = G::LOG2L / G::LOG2R;
@@ -356,8 +385,7 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, 
   row_of<G>(G::MODE_LAST, w.rho, ul, q);
   const long long u = (item << G::LOG2GG) + ul;
   float d[2 * R];
-#pragma unroll
-  for (int c = 0; c < 2 * R; c += 16) tmem_ld16(w.slot + 2 * G::Q + w.lane_off + c, d + c);
+  load_d_row<G, PREC>(w, d);
   if constexpr (G::TW_SMEM) {
     if (mbar_wait_bounded(w.bar_tws, w.ph_tws))
       w.tws_inflight = false;
@@ -435,8 +463,8 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
   constexpr int S2 = S >= 2 ? 2 : S, S3 = S >= 3 ? 3 : S2;
 #pragma unroll
   for (int t = 1; t < S; ++t) {
-    if (t == 1) stage_epilogue<G, 1>(P, tws, w);
-    if (t == 2) stage_epilogue<G, S2>(P, tws, w);
+    if (t == 1) stage_epilogue<G, PREC, 1>(P, tws, w);
+    if (t == 2) stage_epilogue<G, PREC, S2>(P, tws, w);
     if (t == 1 && w.rho == 0) mid.publish();
     fence_before_sync();
     named_bar_or(w.bar_id, 128, false);
@@ -458,7 +486,7 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
     fence_after_sync();
   }
   if (S == 1 && w.rho == 0) mid.publish();
-  last_stage_store<G, OUT_L2>(P, item, w);
+  last_stage_store<G, PREC, OUT_L2>(P, item, w);
 }
 
 // Common set-up: F images and stage twiddles into SMEM, mbarriers, TMEM.
