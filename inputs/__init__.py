@@ -76,13 +76,29 @@ def _fill(out_flat: np.ndarray, seed: int, kind: str, first_point: int):
 
 def tone_frequencies(seed: int, n: int, batch: int, count: int = 3,
                      first: int = 0) -> np.ndarray:
-    """The ``count`` distinct tone frequencies of transforms first..first+batch-1."""
+    """The ``count`` distinct tone frequencies of transforms first..first+batch-1:
+    8 draws per transform, the first ``count`` distinct values kept (in draw
+    order); if 8 draws hold fewer, the last kept value is stepped by +1 mod n
+    until enough are found (practically never happens)."""
     draws = 8
     d = splitmix64(seed ^ TONE_SALT, draws * first, draws * batch)
     cand = ((d >> np.uint64(32)) % np.uint64(n)).astype(np.int64)
     cand = cand.reshape(batch, draws)
     out = np.empty((batch, count), dtype=np.int64)
-    for b in range(batch):
+    # vectorised "first distinct" selection
+    taken = np.zeros((batch, draws), dtype=bool)
+    chosen = np.full((batch, count), -1, dtype=np.int64)
+    rows = np.arange(batch)
+    for c in range(count):
+        fresh = np.ones((batch, draws), dtype=bool)
+        for prev in range(c):
+            fresh &= cand != chosen[:, prev:prev + 1]
+        idx = np.argmax(fresh, axis=1)
+        ok = fresh[rows, idx]
+        chosen[:, c] = np.where(ok, cand[rows, idx], -1)
+    out[:] = chosen
+    bad = np.nonzero((chosen < 0).any(axis=1))[0]
+    for b in bad:  # deterministic fill, as the scalar definition
         seen = []
         for c in cand[b]:
             if c not in seen:
@@ -90,7 +106,7 @@ def tone_frequencies(seed: int, n: int, batch: int, count: int = 3,
                 if len(seen) == count:
                     break
         f = seen[-1]
-        while len(seen) < count:  # deterministic fill; practically never hit
+        while len(seen) < count:
             f = (f + 1) % n
             if f not in seen:
                 seen.append(f)
@@ -113,15 +129,21 @@ def make(kind: str, n: int, batch: int, seed: int, first: int = 0,
         return out
     if kind == "tones":
         freqs = tone_frequencies(seed, n, count, first=first)
-        noise = np.empty(n, dtype=np.complex64)
         j = np.arange(n, dtype=np.int64)
-        for b in range(count):
-            _fill(noise, seed, "normal", base + b * n)
-            sig = np.zeros(n, dtype=np.complex128)
-            for f in freqs[b]:
-                sig += np.exp(2j * np.pi * ((f * j) % n) / n)
-            sig += sigma * noise.astype(np.complex128)
-            out[b] = sig.astype(np.complex64)
+        # exp(2 pi i m / n) for every residue m, gathered below (the same
+        # values as evaluating it per element)
+        roots = np.exp(2j * np.pi * np.arange(n, dtype=np.int64) / n)
+        step = max(1, CHUNK // n)
+        noise = np.empty(step * n, dtype=np.complex64)
+        for b0 in range(0, count, step):
+            b1 = min(count, b0 + step)
+            nz = noise[:(b1 - b0) * n]
+            _fill(nz, seed, "normal", base + b0 * n)
+            sig = np.zeros((b1 - b0, n), dtype=np.complex128)
+            for t in range(freqs.shape[1]):
+                sig += roots[(freqs[b0:b1, t:t + 1] * j[None, :]) % n]
+            sig += sigma * nz.reshape(b1 - b0, n).astype(np.complex128)
+            out[b0:b1] = sig.astype(np.complex64)
         return out
     raise ValueError(kind)
 
