@@ -44,17 +44,20 @@ enum RowMode { kQF = 0, kUF = 1, kRQF = 2 };
 enum Role { kSingle = 0, kFirst = 1, kSecond = 2 };
 
 constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 16 ? 4 : 5); }
-constexpr int nwg_of(int R) { return R == 32 ? 2 : 4; }
+// Warpgroups per CTA: TMEM holds 512 columns, a warpgroup's slot 3 Q of
+// them; a first (strided) pass also stages its inter-pass twiddles in SMEM,
+// which leaves room for four.
+constexpr int pass_nwg(int R, int ROLE) { return R == 32 ? 2 : (ROLE == 1 ? 4 : 5); }
 
 // Compile-time geometry of one pass: S stages of radix R; the other pass (if
 // any) has SO stages.  Sub-transform u = b * Uper + v of transform b.
 //   kSingle: x[b n + a]                      -> y[b n + k]
 //   kFirst : x[b n + a n2 + v] (n2 = R^SO)   -> T[b n + k n2 + v] * w_n^{v k}
 //   kSecond: T[b n + v L + a]                -> y[b n + v + k n1] (n1 = R^SO)
-template <int R, int S, int SO, int ROLE>
+template <int R, int S, int SO, int ROLE, int NWG_ = pass_nwg(R, ROLE)>
 struct Geo {
   static constexpr int LOG2R = log2_radix(R);
-  static constexpr int NWG = nwg_of(R);
+  static constexpr int NWG = NWG_;
   static constexpr int THREADS = 128 * NWG;
   static constexpr int LOG2GPTS = 7 + LOG2R;   // 128 rows of R points
   static constexpr int GPTS = 1 << LOG2GPTS;
@@ -75,8 +78,8 @@ struct Geo {
   static constexpr bool TW_SMEM = TW_OUT && R != 32;  // twiddles staged by TMA
   static constexpr int TMA_ROWS = L < 256 ? L : 256;  // tensor box height
   static constexpr int Q = (2 * R > 32) ? 2 * R : 32;
-  // TMEM slot: A_hi (Q) | A_lo (Q) | D (2Q: [A Bhi | A Blo] in 3xTF32)
-  static constexpr int GCOLS = 4 * Q;
+  // TMEM slot: A_hi (Q) | A_lo (Q) | D (Q)
+  static constexpr int GCOLS = 3 * Q;
   static constexpr int IMG_BYTES = 16 * R * R;
   // entries of the stage twiddle tables: sum over t < S of R * R^(S-t)
   static constexpr int TW_ENTRIES = S == 1 ? 0 : (S == 2 ? R * R : R * R * R + R * R);
@@ -106,8 +109,8 @@ struct GArgs {
   int *counters;        // [0] queue head, [1, 1+batch) done1, then done2
   long long batch;
   int nchunks, lag, ring_chunks;
-  int items1_per_tf;    // pass-1 items per transform
-  int items1_per_chunk, items2_per_chunk;
+  int items1_per_tf;          // pass-1 items per transform
+  int log2_items_per_chunk;   // items of one chunk, the same in both passes
 };
 
 // Offset of stage t's block [j][lo] in the stage twiddle table.
@@ -126,9 +129,8 @@ __host__ __device__ constexpr int tw_stage_offset(int t) {
 // transpose buffer, input staging and twiddle staging | mbarriers (3 per
 // warpgroup: products, input staging, twiddle staging) | TMEM slot |
 // scheduler mailboxes.
-template <int R, int TW1, int TW2>
+template <int R, int NWG, int TW1, int TW2, bool TWS>
 struct SmemLayout {
-  static constexpr int NWG = nwg_of(R);
   static constexpr size_t IMG = 4 * 16 * R * R;
   static constexpr size_t OFF_TW1 = IMG;
   static constexpr size_t OFF_TW2 = OFF_TW1 + (size_t)TW1 * 8;
@@ -136,7 +138,7 @@ struct SmemLayout {
   static constexpr size_t OFF_BUF = (OFF_TW2 + (size_t)TW2 * 8 + 127) / 128 * 128;
   static constexpr size_t OFF_STG = OFF_BUF + (size_t)NWG * PTS * 8;
   static constexpr size_t OFF_TWS = OFF_STG + (size_t)NWG * PTS * 8;
-  static constexpr size_t TWS_BYTES = (R == 32) ? 0 : (size_t)NWG * PTS * 8;
+  static constexpr size_t TWS_BYTES = TWS ? (size_t)NWG * PTS * 8 : 0;
   static constexpr size_t OFF_BAR = OFF_TWS + TWS_BYTES;
   static constexpr size_t OFF_SCHED = OFF_BAR + 8 * 3 * NWG + 8;
   static constexpr size_t BYTES = OFF_SCHED + 32 * NWG;
@@ -158,7 +160,7 @@ struct WG {
   float2 *tws;        // SMEM twiddle staging (one item)
   uint32_t ph_mma, ph_stg, ph_tws;
   bool fail;
-  bool tws_inflight;  // thread rho == 0: a twiddle copy has not been waited on
+  bool tws_inflight;  // warp 0: a twiddle copy has not been waited on
 };
 
 template <class G>
@@ -212,68 +214,53 @@ __device__ __forceinline__ void split_store8(const float2 *x, uint32_t col_hi,
 }
 
 // One stage: D = A * Bf for the 128 rows of this warpgroup's slot.
-// 3xTF32: the hi and lo images of Bf lie back to back with the same 8-row
-// group stride, so one N = 4r descriptor covers [Bhi | Blo]; D accumulates
-// lo * [Bhi | Blo] then hi * [Bhi | Blo] (8 products of K = 8, small terms
-// first) and the epilogue adds its two halves: hi Bhi + lo Bhi + hi Blo
-// (+ lo Blo, below fp32 resolution).  One accumulator chain of 2r/8 * 2
-// products instead of three chains' worth (2r/8 * 3) at N = 2r.
+// 3xTF32: one accumulator chain over K = 6r, i.e. [A_lo | A_hi | A_hi] times
+// [Bhi; Blo; Bhi] stacked -- lo*Bhi + hi*Blo + hi*Bhi, small terms first
+// (lo*Blo is below fp32 resolution and dropped).  The three K-blocks read the
+// same TMEM columns of A_hi twice; D has N = 2r columns and needs no sum in
+// the epilogue.
 template <int R, int PREC>
 __device__ __forceinline__ void issue_stage_mma(uint32_t slot, uint32_t img_addr) {
   constexpr int Q = (2 * R > 32) ? 2 * R : 32;
-  constexpr int LBO = 128, SBO = 64 * R, KSTEPS = 2 * R / 8;
-  constexpr uint32_t idesc = idesc_tf32(128, PREC == 3 ? 4 * R : 2 * R);
+  constexpr int IMG = 16 * R * R, LBO = 128, SBO = 64 * R, KSTEPS = 2 * R / 8;
+  constexpr uint32_t idesc = idesc_tf32(128, 2 * R);
   const uint32_t ahi = slot, alo = slot + Q, d = slot + 2 * Q;
+  const uint32_t ihi = img_addr, ilo = img_addr + IMG;
   uint32_t acc = 0;
   if (PREC == 3) {
 #pragma unroll
     for (int kk = 0; kk < KSTEPS; ++kk) {
-      mma_tf32_ts(d, alo + 8 * kk, smem_desc_noswz(img_addr + kk * 2 * LBO, LBO, SBO),
-                  idesc, acc);
+      mma_tf32_ts(d, alo + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO), idesc,
+                  acc);
       acc = 1;
     }
+#pragma unroll
+    for (int kk = 0; kk < KSTEPS; ++kk)
+      mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(ilo + kk * 2 * LBO, LBO, SBO), idesc, 1);
   }
 #pragma unroll
   for (int kk = 0; kk < KSTEPS; ++kk) {
-    mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(img_addr + kk * 2 * LBO, LBO, SBO),
-                idesc, acc);
+    mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO), idesc, acc);
     acc = 1;
   }
 }
 
-// This thread's whole D row (2r values) with the TMEM loads batched under
-// one wait per 64 columns; in 3xTF32 the sum of the [A Bhi] and [A Blo]
-// halves.
+// This thread's whole D row (2r values), TMEM loads under one wait.
 template <class G, int PREC>
 __device__ __forceinline__ void load_d_row(const WG &w, float *d) {
   constexpr int R = 1 << G::LOG2R;
   const uint32_t base = w.slot + 2 * G::Q + w.lane_off;
-  if (PREC == 3) {
-    if (R == 8) {
-      float v[32];
-      tmem_ld16x2(base, base + 16, v);
-#pragma unroll
-      for (int i = 0; i < 16; ++i) d[i] = v[i] + v[16 + i];
-    } else {
-#pragma unroll
-      for (int c = 0; c < 2 * R; c += 32) {
-        float v[64];
-        tmem_ld32x2(base + c, base + 2 * R + c, v);
-#pragma unroll
-        for (int i = 0; i < 32; ++i) d[c + i] = v[i] + v[32 + i];
-      }
-    }
+  if (R == 8) {
+    tmem_ld16(base, d);
+  } else if (R == 16) {
+    tmem_ld32(base, d);
   } else {
-    if (R == 8) {
-      tmem_ld16(base, d);
-    } else {
-#pragma unroll
-      for (int c = 0; c < 2 * R; c += 32) tmem_ld32(base + c, d + c);
-    }
+    tmem_ld32x2(base, base + 32, d);
   }
 }
 
-// ---- TMA issue (one thread): the input block of `item` into staging
+// ---- TMA issue (warp 0 of the warpgroup, converged; one elected lane
+// issues): the input block of `item` into staging
 template <class G>
 __device__ __forceinline__ void issue_input(const PRun &P, const CUtensorMap *tm,
                                             long long item, const WG &w) {
@@ -283,10 +270,12 @@ __device__ __forceinline__ void issue_input(const PRun &P, const CUtensorMap *tm
     // strided first pass: box of GG sub-transforms x L points
     const long long b = u0 >> G::LOG2UPER;
     const int v0 = (int)(u0 & ((1ll << G::LOG2UPER) - 1));
-    mbar_expect_tx(w.bar_stg, G::GPTS * 8);
+    if (elect_one()) {
+      mbar_expect_tx(w.bar_stg, G::GPTS * 8);
 #pragma unroll
-    for (int a0 = 0; a0 < G::L; a0 += G::TMA_ROWS)
-      tma_load_3d(dst + a0 * G::GG * 8, tm, 2 * v0, a0, (int)b, w.bar_stg);
+      for (int a0 = 0; a0 < G::L; a0 += G::TMA_ROWS)
+        tma_load_3d(dst + a0 * G::GG * 8, tm, 2 * v0, a0, (int)b, w.bar_stg);
+    }
   } else {
     // contiguous block of GG sub-transforms (the last item may be short)
     long long rem = P.U - u0;
@@ -295,12 +284,16 @@ __device__ __forceinline__ void issue_input(const PRun &P, const CUtensorMap *tm
     const long long b = u0 >> G::LOG2UPER;
     const long long v = u0 & ((1ll << G::LOG2UPER) - 1);
     const float2 *src = P.in + ((b & P.in_bmask) << G::LOG2N) + (v << G::LOG2L);
-    mbar_expect_tx(w.bar_stg, bytes);
-    tma_load_1d(dst, src, bytes, w.bar_stg);
+    if (elect_one()) {
+      mbar_expect_tx(w.bar_stg, bytes);
+      tma_load_1d(dst, src, bytes, w.bar_stg);
+    }
   }
+  __syncwarp();
 }
 
-// ---- TMA issue (one thread): the inter-pass twiddles of a first-pass item
+// ---- TMA issue (warp 0, converged): the inter-pass twiddles of a
+// first-pass item
 template <class G>
 __device__ __forceinline__ void issue_twiddles(const CUtensorMap *tm, long long item,
                                                const WG &w) {
@@ -308,11 +301,26 @@ __device__ __forceinline__ void issue_twiddles(const CUtensorMap *tm, long long 
     const long long u0 = item << G::LOG2GG;
     const int v0 = (int)(u0 & ((1ll << G::LOG2UPER) - 1));
     const uint32_t dst = smem_u32(w.tws);
-    mbar_expect_tx(w.bar_tws, G::GPTS * 8);
+    if (elect_one()) {
+      mbar_expect_tx(w.bar_tws, G::GPTS * 8);
 #pragma unroll
-    for (int k0 = 0; k0 < G::L; k0 += G::TMA_ROWS)
-      tma_load_3d(dst + k0 * G::GG * 8, tm, 2 * v0, k0, 0, w.bar_tws);
+      for (int k0 = 0; k0 < G::L; k0 += G::TMA_ROWS)
+        tma_load_3d(dst + k0 * G::GG * 8, tm, 2 * v0, k0, 0, w.bar_tws);
+    }
+    __syncwarp();
   }
+}
+
+// ---- products of one stage (warp 0, converged): issue and commit from one
+// elected lane
+template <int R, int PREC>
+__device__ __forceinline__ void issue_stage(uint32_t slot, uint32_t img_addr,
+                                            uint32_t bar_mma) {
+  if (elect_one()) {
+    issue_stage_mma<R, PREC>(slot, img_addr);
+    mma_commit(bar_mma);
+  }
+  __syncwarp();
 }
 
 // This thread's stage-1 row, from the staged input block.
@@ -422,9 +430,9 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, 
   }
 }
 
-// The whole item.  `mid` supplies the next-item logic (thread rho == 0 runs
-// issue() right after the stage-1 products and publish() just before the
-// first epilogue barrier).  On entry the item's input copy has been issued.
+// The whole item.  `mid` supplies the next-item logic (warp 0 of the
+// warpgroup runs issue() right after the stage-1 products and publish() just
+// before the first epilogue barrier).  On entry the item's input copy has been issued.
 template <class G, int PREC, bool OUT_L2, class Mid>
 __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *tm_tw,
                                              const float2 *tws, long long item, WG &w,
@@ -447,10 +455,9 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
     return;
   }
   // staging is free again: the next item's copy may land there
-  if (w.rho == 0) {
+  if (w.rho < 32) {
     fence_after_sync();
-    issue_stage_mma<R, PREC>(w.slot, w.img_addr + (S == 1 ? P.last_img : 0));
-    mma_commit(w.bar_mma);
+    issue_stage<R, PREC>(w.slot, w.img_addr + (S == 1 ? P.last_img : 0), w.bar_mma);
     if (G::TW_SMEM) {
       issue_twiddles<G>(tm_tw, item, w);
       w.tws_inflight = true;
@@ -465,7 +472,7 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
   for (int t = 1; t < S; ++t) {
     if (t == 1) stage_epilogue<G, PREC, 1>(P, tws, w);
     if (t == 2) stage_epilogue<G, PREC, S2>(P, tws, w);
-    if (t == 1 && w.rho == 0) mid.publish();
+    if (t == 1 && w.rho < 32) mid.publish();
     fence_before_sync();
     named_bar_or(w.bar_id, 128, false);
     if (t == 1) stage_rows<G, PREC, S2>(P, w);
@@ -476,16 +483,15 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
       w.fail = true;
       return;
     }
-    if (w.rho == 0) {
+    if (w.rho < 32) {
       fence_after_sync();
-      issue_stage_mma<R, PREC>(w.slot, w.img_addr + (t + 1 == S ? P.last_img : 0));
-      mma_commit(w.bar_mma);
+      issue_stage<R, PREC>(w.slot, w.img_addr + (t + 1 == S ? P.last_img : 0), w.bar_mma);
     }
     if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
     w.ph_mma ^= 1;
     fence_after_sync();
   }
-  if (S == 1 && w.rho == 0) mid.publish();
+  if (S == 1 && w.rho < 32) mid.publish();
   last_stage_store<G, PREC, OUT_L2>(P, item, w);
 }
 
@@ -572,7 +578,7 @@ template <int R, int PREC, int S, int SO, int ROLE>
 __global__ void __launch_bounds__(Geo<R, S, SO, ROLE>::THREADS, 1)
     dft_pass_kernel(const __grid_constant__ GArgs a) {
   using G = Geo<R, S, SO, ROLE>;
-  using SM = SmemLayout<R, G::TW_ENTRIES, 0>;
+  using SM = SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM>;
   extern __shared__ __align__(1024) unsigned char smem[];
   float2 *tw = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
   uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + SM::OFF_BAR);
@@ -589,7 +595,7 @@ __global__ void __launch_bounds__(Geo<R, S, SO, ROLE>::THREADS, 1)
   const long long istride = (long long)gridDim.x * G::NWG;
   long long item = (long long)blockIdx.x * G::NWG + wg;
   StaticNext<G> nx{P, &a.tm_in, item, nitems, false};
-  if (w.rho == 0 && item < nitems) issue_input<G>(P, &a.tm_in, item, w);
+  if (w.rho < 32 && item < nitems) issue_input<G>(P, &a.tm_in, item, w);
   while (item < nitems && !w.fail) {
     nx.next = item + istride;
     process_item<G, PREC, false>(P, &a.tm_tw, tw, item, w, nx);
@@ -611,39 +617,40 @@ __device__ __forceinline__ void red_release_add(int *p, int v) {
   asm volatile("red.release.gpu.global.add.s32 [%0], %1;" ::"l"(p), "r"(v) : "memory");
 }
 
-// Queue position -> (pass, item).  Order: P1(0) .. P1(lag-1), then for
-// c >= lag: P1(c), P2(c - lag); then the remaining P2 chunks.  Returns false
-// past the end.
+// Queue position -> (pass, item).  Both passes have the same number of
+// items per chunk, A = 2^lgA (every item is 128 r points).  Order:
+// P1(0) .. P1(lag-1), then for c >= lag: P1(c), P2(c - lag); then the
+// remaining P2 chunks.  Returns false past the end.
 __device__ __forceinline__ bool decode_queue(const GArgs &a, long long pos, int &pass,
                                              long long &item, int &chunk) {
-  const long long A = a.items1_per_chunk, B = a.items2_per_chunk;
+  const int lgA = a.log2_items_per_chunk;
+  const long long A = 1ll << lgA;
   const int lag = a.lag, nc = a.nchunks;
-  if (pos < (long long)lag * A) {
+  if (pos < ((long long)lag << lgA)) {
     pass = 0;
-    chunk = (int)(pos / A);
-    item = chunk * A + pos % A;
+    chunk = (int)(pos >> lgA);
+    item = pos;
     return true;
   }
-  const long long p2 = pos - (long long)lag * A;
-  const long long mid = (long long)(nc - lag) * (A + B);
-  if (p2 < mid) {
-    const long long step = p2 / (A + B), off = p2 % (A + B);
+  const long long p2 = pos - ((long long)lag << lgA);
+  if (p2 < ((long long)(nc - lag) << (lgA + 1))) {
+    const long long step = p2 >> (lgA + 1), off = p2 & (2 * A - 1);
     if (off < A) {
       pass = 0;
       chunk = (int)(lag + step);
-      item = chunk * A + off;
+      item = ((long long)chunk << lgA) + off;
     } else {
       pass = 1;
       chunk = (int)step;
-      item = chunk * B + (off - A);
+      item = ((long long)chunk << lgA) + (off - A);
     }
     return true;
   }
-  const long long p3 = p2 - mid;
-  if (p3 < (long long)lag * B) {
+  const long long p3 = p2 - ((long long)(nc - lag) << (lgA + 1));
+  if (p3 < ((long long)lag << lgA)) {
     pass = 1;
-    chunk = (int)(nc - lag + p3 / B);
-    item = chunk * B + p3 % B;
+    chunk = (int)(nc - lag + (p3 >> lgA));
+    item = ((long long)chunk << lgA) + (p3 & (A - 1));
     return true;
   }
   return false;
@@ -663,7 +670,9 @@ struct QItem {
   bool valid;
 };
 
-// Next-item logic of the fused schedule, run by one thread per warpgroup.
+// Next-item logic of the fused schedule, run by warp 0 of each warpgroup;
+// its state is the same in all 32 lanes, except the results of the global
+// atomic and the flag read, which lane 0 holds until they are needed.
 // Items: cur (being processed), n1 (next), n2 (the one after).  During cur:
 //   issue()   -- right after cur's first products: if n1's dependency value
 //                (read one item earlier) says ready, issue n1's input copy;
@@ -679,11 +688,14 @@ template <class G1, class G2>
 struct FusedNext {
   const GArgs &a;
   FusedSched *box;
-  QItem n1, n2;
-  int dep_val, dep_target;
-  int pos2;
+  QItem n1;
+  int dep_raw;     // lane 0: value read from n1's dependency flag
+  int dep_target;
+  int pos2;        // lane 0: claimed queue position
   bool n1_issued;
   int *pend_flag;
+
+  __device__ static bool lane0() { return (threadIdx.x & 31) == 0; }
 
   // A pass-1 item waits until the ring slot it overwrites has been drained
   // by pass 2; a pass-2 item until every pass-1 item of its transform has
@@ -691,7 +703,7 @@ struct FusedNext {
   __device__ const int *dep_flag(const QItem &q, int &target) const {
     if (q.pass == 0) {
       if (q.chunk < a.ring_chunks) return nullptr;
-      target = a.items2_per_chunk;
+      target = 1 << a.log2_items_per_chunk;
       return a.counters + 1 + a.batch + (q.chunk - a.ring_chunks);
     }
     target = a.items1_per_tf;
@@ -700,29 +712,41 @@ struct FusedNext {
   }
 
   __device__ void read_dep(const QItem &q) {
-    dep_val = 1;
+    dep_raw = 1;
     dep_target = 0;
     if (!q.valid) return;
     const int *flag = dep_flag(q, dep_target);
-    if (flag) dep_val = ld_acquire(flag);
+    if (flag && lane0()) dep_raw = ld_acquire(flag);
   }
 
+  // Bounded wait (lane 0 polls) until q's dependency holds; uniform result.
   __device__ bool wait_deps(const QItem &q) const {
     int target = 0;
     const int *flag = dep_flag(q, target);
-    if (!flag || ld_acquire(flag) >= target) return true;
-    const unsigned long long t0 = global_ns();
-    while (ld_acquire(flag) < target) {
-      if (global_ns() - t0 > kWaitNs) return false;
-      __nanosleep(100);
+    int ok = 1;
+    if (flag && lane0() && ld_acquire(flag) < target) {
+      const unsigned long long t0 = global_ns();
+      while (ld_acquire(flag) < target) {
+        if (global_ns() - t0 > kWaitNs) {
+          ok = 0;
+          break;
+        }
+        __nanosleep(100);
+      }
     }
-    return true;
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
   }
 
-  __device__ QItem decode(int pos) const {
+  __device__ QItem decode(long long pos) const {
     QItem q;
     q.valid = decode_queue(a, pos, q.pass, q.item, q.chunk);
     return q;
+  }
+
+  __device__ int claim() const {
+    int p = 0;
+    if (lane0()) p = atomicAdd(a.counters, 1);
+    return p;
   }
 
   __device__ void issue_copy(const QItem &q, const WG &w) {
@@ -735,27 +759,30 @@ struct FusedNext {
 
   __device__ void publish_pending() {
     if (pend_flag) {
-      red_release_add(pend_flag, 1);
+      if (lane0()) red_release_add(pend_flag, 1);
       pend_flag = nullptr;
     }
   }
 
   __device__ void issue(const WG &w) {
+    const int dep_val = __shfl_sync(0xffffffffu, dep_raw, 0);
     n1_issued = false;
     if (n1.valid && dep_val >= dep_target) {
       issue_copy(n1, w);
       n1_issued = true;
     }
-    pos2 = atomicAdd(a.counters, 1);
+    pos2 = claim();
   }
 
   __device__ void publish() {
     publish_pending();
-    box->item = n1.item;
-    box->pass = n1.valid ? n1.pass : -1;
-    box->chunk = n1.chunk;
-    box->issued = n1_issued ? 1 : 0;
-    n1 = decode(pos2);
+    if (lane0()) {
+      box->item = n1.item;
+      box->pass = n1.valid ? n1.pass : -1;
+      box->chunk = n1.chunk;
+      box->issued = n1_issued ? 1 : 0;
+    }
+    n1 = decode(__shfl_sync(0xffffffffu, pos2, 0));
     read_dep(n1);
   }
 };
@@ -765,8 +792,8 @@ __global__ void __launch_bounds__(Geo<R, S1, S2, kFirst>::THREADS, 1)
     dft_fused_kernel(const __grid_constant__ GArgs a) {
   static_assert(S1 >= 2 && S2 >= 2, "the fused schedule needs an SMEM barrier per item");
   using G1 = Geo<R, S1, S2, kFirst>;
-  using G2 = Geo<R, S2, S1, kSecond>;
-  using SM = SmemLayout<R, G1::TW_ENTRIES, G2::TW_ENTRIES>;
+  using G2 = Geo<R, S2, S1, kSecond, G1::NWG>;
+  using SM = SmemLayout<R, G1::NWG, G1::TW_ENTRIES, G2::TW_ENTRIES, G1::TW_SMEM>;
   constexpr int NWG = G1::NWG;
   extern __shared__ __align__(1024) unsigned char smem[];
   float2 *tw1 = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
@@ -787,19 +814,21 @@ __global__ void __launch_bounds__(Geo<R, S1, S2, kFirst>::THREADS, 1)
   nx.n1_issued = false;
 
   // first item: claim it, wait for its dependencies, issue its copy; claim
-  // the one after and start reading its dependency
+  // the one after and start reading its dependency (warp 0)
   bool f = false;
-  if (w.rho == 0) {
-    const QItem first = nx.decode(atomicAdd(a.counters, 1));
+  if (w.rho < 32) {
+    const QItem first = nx.decode(__shfl_sync(0xffffffffu, nx.claim(), 0));
     if (first.valid) {
       if (!nx.wait_deps(first)) f = true;
       else nx.issue_copy(first, w);
     }
-    box->item = first.item;
-    box->pass = first.valid ? first.pass : -1;
-    box->chunk = first.chunk;
-    box->issued = first.valid && !f;
-    nx.n1 = nx.decode(atomicAdd(a.counters, 1));
+    if (w.rho == 0) {
+      box->item = first.item;
+      box->pass = first.valid ? first.pass : -1;
+      box->chunk = first.chunk;
+      box->issued = first.valid && !f;
+    }
+    nx.n1 = nx.decode(__shfl_sync(0xffffffffu, nx.claim(), 0));
     nx.read_dep(nx.n1);
   }
   if (named_bar_or(w.bar_id, 128, f)) w.fail = true;
@@ -815,7 +844,7 @@ __global__ void __launch_bounds__(Geo<R, S1, S2, kFirst>::THREADS, 1)
       // completion (it may be what it waits for; the barrier orders every
       // thread's stores of it first), wait, then copy
       bool ff = named_bar_or(w.bar_id, 128, false);
-      if (w.rho == 0) {
+      if (w.rho < 32) {
         nx.publish_pending();
         const QItem q{item, pass, chunk, true};
         if (!nx.wait_deps(q)) ff = true;
@@ -834,16 +863,14 @@ __global__ void __launch_bounds__(Geo<R, S1, S2, kFirst>::THREADS, 1)
     if (w.fail) break;
     // the mailbox now names the next item; its completion is published
     // during the next item (after its first barrier), or below
-    if (w.rho == 0)
+    if (w.rho < 32)
       nx.pend_flag = (pass == 0) ? a.counters + 1 + ((item << G1::LOG2GG) >> G1::LOG2UPER)
                                  : a.counters + 1 + a.batch + chunk;
   }
   // all stores of this warpgroup are issued: publish the last completion
   named_bar_or(w.bar_id, 128, false);
-  if (w.rho == 0) {
-    nx.publish_pending();
-    if (w.fail) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);
-  }
+  if (w.rho < 32) nx.publish_pending();
+  if (w.rho == 0 && w.fail) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);
   kernel_teardown(tbase, w, w.fail && stg_pending, w.fail && w.tws_inflight);
 }
 

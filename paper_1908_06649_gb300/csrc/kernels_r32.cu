@@ -8,7 +8,9 @@ cudaError_t launch_pass_r32(int prec, int s, int so, int role, const GArgs &a, i
   constexpr int R = 32;
   TCU_PASS_CASE(1, 0, kSingle)
   TCU_PASS_CASE(2, 0, kSingle)
-  TCU_PASS_CASE(2, 1, kFirst)   // n = 32^3
+  TCU_PASS_CASE(1, 2, kFirst)   // n = 32^3
+  TCU_PASS_CASE(2, 1, kSecond)
+  TCU_PASS_CASE(2, 1, kFirst)
   TCU_PASS_CASE(1, 2, kSecond)
   TCU_PASS_CASE(2, 2, kFirst)   // n = 32^4
   TCU_PASS_CASE(2, 2, kSecond)

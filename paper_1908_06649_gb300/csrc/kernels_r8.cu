@@ -11,7 +11,9 @@ cudaError_t launch_pass_r8(int prec, int s, int so, int role, const GArgs &a, in
   TCU_PASS_CASE(3, 0, kSingle)
   TCU_PASS_CASE(2, 2, kFirst)   // n = 8^4
   TCU_PASS_CASE(2, 2, kSecond)
-  TCU_PASS_CASE(3, 2, kFirst)   // n = 8^5
+  TCU_PASS_CASE(2, 3, kFirst)   // n = 8^5
+  TCU_PASS_CASE(3, 2, kSecond)
+  TCU_PASS_CASE(3, 2, kFirst)
   TCU_PASS_CASE(2, 3, kSecond)
   TCU_PASS_CASE(3, 3, kFirst)   // n = 8^6
   TCU_PASS_CASE(3, 3, kSecond)
@@ -23,6 +25,7 @@ cudaError_t launch_fused_r8(int prec, int s1, int s2, const GArgs &a, int num_sm
                             cudaStream_t st) {
   constexpr int R = 8;
   TCU_FUSED_CASE(2, 2)
+  TCU_FUSED_CASE(2, 3)
   TCU_FUSED_CASE(3, 2)
   TCU_FUSED_CASE(3, 3)
   return cudaErrorInvalidValue;

@@ -8,7 +8,7 @@ namespace tcu {
 template <int R, int PREC, int S, int SO, int ROLE>
 cudaError_t launch_pass_t(const GArgs &a, int num_sms, cudaStream_t st) {
   using G = Geo<R, S, SO, ROLE>;
-  const size_t sm = SmemLayout<R, G::TW_ENTRIES, 0>::BYTES;
+  const size_t sm = SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM>::BYTES;
   cudaError_t e = cudaFuncSetAttribute(dft_pass_kernel<R, PREC, S, SO, ROLE>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)sm);
@@ -23,8 +23,8 @@ cudaError_t launch_pass_t(const GArgs &a, int num_sms, cudaStream_t st) {
 template <int R, int PREC, int S1, int S2>
 cudaError_t launch_fused_t(const GArgs &a, int num_sms, cudaStream_t st) {
   using G1 = Geo<R, S1, S2, kFirst>;
-  using G2 = Geo<R, S2, S1, kSecond>;
-  const size_t sm = SmemLayout<R, G1::TW_ENTRIES, G2::TW_ENTRIES>::BYTES;
+  using G2 = Geo<R, S2, S1, kSecond, G1::NWG>;
+  const size_t sm = SmemLayout<R, G1::NWG, G1::TW_ENTRIES, G2::TW_ENTRIES, G1::TW_SMEM>::BYTES;
   cudaError_t e = cudaFuncSetAttribute(dft_fused_kernel<R, PREC, S1, S2>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)sm);

@@ -90,7 +90,7 @@ struct tcu_dft_plan_s {
   // fused two-pass schedule
   bool fused;
   int log2C, nchunks, lag, ring_chunks;
-  int items1_per_tf, items1_per_chunk, items2_per_chunk;
+  int items1_per_tf, log2_items_per_chunk;
   int *counters;
   size_t counter_bytes;
   int *err;
@@ -214,6 +214,14 @@ std::vector<float2> stage_twiddles(int r, int s, int sign) {
 // SMEM tile) and warpgroup kernel (a sub-transform fits 128 rows).
 int max_tile_stages(int r) { return r == 8 ? 4 : (r == 16 ? 3 : 2); }
 int max_group_stages(int r) { return r == 8 ? 3 : 2; }
+
+// Two warpgroup passes of k stages: the strided first pass takes the smaller
+// half -- its sub-transforms are shorter, so an item spans more adjacent
+// columns and its TMA boxes have wider rows.
+void split_two_passes(int k, int stages[2]) {
+  stages[0] = k / 2;
+  stages[1] = k - stages[0];
+}
 
 int stage_mode(const int modes[3], int t, int S) {
   return t == 1 ? modes[0] : (t == S ? modes[2] : modes[1]);
@@ -485,8 +493,7 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
     stages[0] = k;
   } else if (k <= 2 * sg) {
     npasses = 2;
-    stages[0] = (k + 1) / 2;
-    stages[1] = k - stages[0];
+    split_two_passes(k, stages);
   } else if (k <= stl + sg) {
     npasses = 2;
     stages[0] = k - sg;
@@ -627,8 +634,9 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
       const long long n1 = 1ll << p1.log2L, n2 = 1ll << p2.log2L;
       const long long gg1 = (128ll * r) >> p1.log2L, gg2 = (128ll * r) >> p2.log2L;
       p->items1_per_tf = (int)(n2 / gg1);
-      p->items1_per_chunk = (int)((n2 / gg1) << log2C);
-      p->items2_per_chunk = (int)((n1 / gg2) << log2C);
+      // every item is 128 r points, so both passes have n C / (128 r) per chunk
+      if ((n2 / gg1) != (n1 / gg2)) rc = TCU_DFT_ERR_UNSUPPORTED;
+      p->log2_items_per_chunk = ilog2(n2 / gg1) + log2C;
       scratch_tf = (long long)p->ring_chunks << log2C;
       p->counter_bytes = (size_t)(1 + batch + p->nchunks) * sizeof(int);
       if (cudaMalloc((void **)&p->counters, p->counter_bytes) != cudaSuccess) {
@@ -679,8 +687,7 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
     g.lag = p->lag;
     g.ring_chunks = p->ring_chunks;
     g.items1_per_tf = p->items1_per_tf;
-    g.items1_per_chunk = p->items1_per_chunk;
-    g.items2_per_chunk = p->items2_per_chunk;
+    g.log2_items_per_chunk = p->log2_items_per_chunk;
     if (cudaMemsetAsync(p->counters, 0, p->counter_bytes, st) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
     if (events && cudaEventRecord((cudaEvent_t)events[0], st) != cudaSuccess)
@@ -825,10 +832,7 @@ int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t preci
   const int npasses = k <= sg ? 1 : 2;
   if (npasses == 2 && batch * n > kNaMaxPoints) return TCU_DFT_ERR_TOO_LARGE;
   int stages[2] = {k, 0};
-  if (npasses == 2) {
-    stages[0] = (k + 1) / 2;
-    stages[1] = k - stages[0];
-  }
+  if (npasses == 2) split_two_passes(k, stages);
   const int log2n = ilog2(n);
   cudaStream_t st = (cudaStream_t)stream;
 
