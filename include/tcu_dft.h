@@ -62,13 +62,17 @@ enum {
  * sqrt_m (the TCU side length sqrt(m) of Sec. 3; one of 8, 16, 32) and the
  * given precision.  n must equal sqrt_m^k for some k >= 1 (Theorem 7 assumes
  * all of n, n/sqrt(m), ... are integers).
+ * The k stages run in up to three HBM passes of at most two stages each
+ * (three for sqrt_m = 8), so n <= 16^6, 32^6 or 8^9.
  * Allocates the device tables (F_r operand images, twiddles) and, when n
- * needs two passes, a scratch buffer of batch*n complex64 values; uses the
- * current CUDA device.  This is the only call that allocates.
+ * needs several passes, one scratch buffer of batch*n complex64 values per
+ * intermediate (two for three passes); uses the current CUDA device.  This
+ * is the only call that allocates.
  * Returns NULL on error and sets tcu_dft_last_error():
  *   ERR_INVALID (n < 1, batch < 1, precision not 1 or 3),
- *   ERR_UNSUPPORTED (sqrt_m not in {8,16,32}, n not a power of sqrt_m, or
- *   n beyond two on-chip passes), ERR_CUDA (no sm_103 device), ERR_OOM. */
+ *   ERR_UNSUPPORTED (sqrt_m not in {8,16,32}, n not a power of sqrt_m, n
+ *   beyond three passes, or batch*n > 2^40), ERR_CUDA (no sm_103 device),
+ *   ERR_OOM. */
 tcu_dft_plan_t tcu_dft_plan(int64_t n, int64_t batch, int32_t sqrt_m,
                             int32_t precision);
 
@@ -152,8 +156,8 @@ int tcu_dft_pass_stages(tcu_dft_plan_t p, int i);
  * every GPU that loads the library until the process exits.  It never calls
  * cudaMalloc or cudaFree.
  *
- * Limits: n a power of sqrt_m whose stages fit two warpgroup passes (sqrt_m
- * 16: n <= 16^4; 8: n <= 8^6; 32: n <= 32^3) and n <= 2^18; when n needs two
+ * Limits: n a power of sqrt_m that needs at most two passes (sqrt_m 16:
+ * n <= 16^4; 8: n <= 8^4; 32: n <= 32^3) and n <= 2^18; when n needs two
  * passes, batch*n <= 2^22.  Larger requests return TCU_DFT_ERR_TOO_LARGE
  * with nothing launched; other argument errors ERR_INVALID / ERR_UNSUPPORTED
  * as tcu_dft_plan would.

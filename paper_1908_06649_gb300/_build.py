@@ -12,7 +12,7 @@ import subprocess
 HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 UNITS = ["tcu_dft.cu", "kernels_r8.cu", "kernels_r16.cu", "kernels_r32.cu"]
-HEADERS = ["tcgen05.cuh", "tile_kernel.cuh", "group_kernel.cuh", "launch.h",
+HEADERS = ["tcgen05.cuh", "group_kernel.cuh", "launch.h",
            "launch_impl.cuh"]
 HDR = os.path.join(os.path.dirname(HERE), "include", "tcu_dft.h")
 LIB_PATH = os.path.join(HERE, "libtcu_dft.so")

@@ -49,12 +49,18 @@ constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 16 ? 4 : 5); }
 // which leaves room for four.
 constexpr int pass_nwg(int R, int ROLE) { return R == 32 ? 2 : (ROLE == 1 ? 4 : 5); }
 
-// Compile-time geometry of one pass: S stages of radix R; the other pass (if
-// any) has SO stages.  Sub-transform u = b * Uper + v of transform b.
-//   kSingle: x[b n + a]                      -> y[b n + k]
-//   kFirst : x[b n + a n2 + v] (n2 = R^SO)   -> T[b n + k n2 + v] * w_n^{v k}
-//   kSecond: T[b n + v L + a]                -> y[b n + v + k n1] (n1 = R^SO)
-template <int R, int S, int SO, int ROLE, int NWG_ = pass_nwg(R, ROLE)>
+// Compile-time geometry of one pass: S stages of radix R.  A transform of
+// length n = R^K is computed in up to three passes (the four-step split
+// applied recursively); a pass splits sequences of length M = R^(S+SO) into
+// L = R^S rows by n2 = R^SO columns.
+//   kSingle: x[b n + a]                        -> y[b n + k]
+//   kFirst : strided pass; SP stages come before it, SO after.  Sequence
+//            b' = (b, p), p < Npre = R^SP, holds z[b' M + a n2 + v]; the
+//            DFT over a, times w_M^{v k}, goes to T[b n + (k Npre + p) n2 + v]
+//            (for SP = 0: T[b n + k n2 + v])
+//   kSecond: last of several passes (SO stages before it):
+//            T[b n + v L + a] -> y[b n + v + k n1], n1 = R^SO
+template <int R, int S, int SO, int ROLE, int SP = 0, int NWG_ = pass_nwg(R, ROLE)>
 struct Geo {
   static constexpr int LOG2R = log2_radix(R);
   static constexpr int NWG = NWG_;
@@ -63,19 +69,27 @@ struct Geo {
   static constexpr int GPTS = 1 << LOG2GPTS;
   static constexpr int LOG2L = LOG2R * S;
   static constexpr int L = 1 << LOG2L;
-  static constexpr int LOG2N = LOG2R * (S + SO);
+  static constexpr int LOG2N = LOG2R * (S + SO);        // sequence length M
+  static constexpr int LOG2PRE = ROLE == kFirst ? LOG2R * SP : 0;
+  static constexpr int LOG2NT = LOG2N + LOG2PRE;        // transform length n
   static constexpr int LOG2RPS = LOG2L - LOG2R;   // rows per sub-transform
   static constexpr int LOG2GG = LOG2GPTS - LOG2L; // sub-transforms per item
   static constexpr int GG = 1 << LOG2GG;
   static constexpr int LOG2O = LOG2R * SO;
   static constexpr int LOG2UPER = ROLE == kSingle ? 0 : LOG2O;
-  static constexpr long long OUT_STRIDE = ROLE == kSingle ? 1 : (1ll << LOG2O);
+  static constexpr long long OUT_STRIDE =
+      ROLE == kSingle ? 1 : (1ll << (LOG2O + LOG2PRE));
   static constexpr long long OUT_VSTRIDE = ROLE == kSingle ? 0 : 1;
   static constexpr int MODE_FIRST = ROLE == kFirst ? kUF : kQF;
   static constexpr int MODE_MID = kUF;
   static constexpr int MODE_LAST = ROLE == kSingle ? kRQF : kUF;
   static constexpr bool TW_OUT = ROLE == kFirst;
   static constexpr bool TW_SMEM = TW_OUT && R != 32;  // twiddles staged by TMA
+  // w_M^{k v} with v = vh 2^VL + vl: table A [k][vl] and, for more than 256
+  // columns, table B [vh][k] (two-level, so that no table exceeds L * 256)
+  static constexpr int LOG2VL = (TW_OUT && LOG2UPER > 8) ? 8 : LOG2UPER;
+  static constexpr bool TW2L = TW_OUT && LOG2UPER > 8;
+  static constexpr int TWB = (TW2L && TW_SMEM) ? L : 0;  // SMEM row of table B
   static constexpr int TMA_ROWS = L < 256 ? L : 256;  // tensor box height
   static constexpr int Q = (2 * R > 32) ? 2 * R : 32;
   // TMEM slot: A_hi (Q) | A_lo (Q) | D (Q)
@@ -84,6 +98,7 @@ struct Geo {
   // entries of the stage twiddle tables: sum over t < S of R * R^(S-t)
   static constexpr int TW_ENTRIES = S == 1 ? 0 : (S == 2 ? R * R : R * R * R + R * R);
   static_assert(LOG2GG >= 0, "sub-transform longer than one item");
+  static_assert(LOG2GG <= LOG2VL || !TW_OUT, "an item spans one twiddle column block");
   static_assert(NWG * GCOLS <= 512, "TMEM budget");
 };
 
@@ -93,7 +108,8 @@ struct PRun {
   float2 *out;
   long long in_bmask, out_bmask;  // transform index mask (ring) or ~0
   long long U;                    // sub-transforms in the pass
-  const float2 *tw_out;           // kFirst: w_n^{v k} as [k][v]
+  const float2 *tw_out;           // kFirst: w_M^{vl k} as [k][vl]
+  const float2 *tw_b;             // kFirst, two-level: w_M^{vh 2^VL k} as [vh][k]
   const float2 *tw_stage;         // stage twiddles [t][j][lo]
   unsigned long long swz_tab;     // SMEM swizzle nibble per (ul & 15)
   int last_img;                   // byte offset of the last stage's F images
@@ -129,7 +145,7 @@ __host__ __device__ constexpr int tw_stage_offset(int t) {
 // transpose buffer, input staging and twiddle staging | mbarriers (3 per
 // warpgroup: products, input staging, twiddle staging) | TMEM slot |
 // scheduler mailboxes.
-template <int R, int NWG, int TW1, int TW2, bool TWS>
+template <int R, int NWG, int TW1, int TW2, bool TWS, int TWB = 0>
 struct SmemLayout {
   static constexpr size_t IMG = 4 * 16 * R * R;
   static constexpr size_t OFF_TW1 = IMG;
@@ -139,7 +155,10 @@ struct SmemLayout {
   static constexpr size_t OFF_STG = OFF_BUF + (size_t)NWG * PTS * 8;
   static constexpr size_t OFF_TWS = OFF_STG + (size_t)NWG * PTS * 8;
   static constexpr size_t TWS_BYTES = TWS ? (size_t)NWG * PTS * 8 : 0;
-  static constexpr size_t OFF_BAR = OFF_TWS + TWS_BYTES;
+  static constexpr size_t OFF_TWB = OFF_TWS + TWS_BYTES;  // [k] row of table B
+  static constexpr size_t TWB_PER_WG = TWB;
+  static constexpr size_t TWB_BYTES = (size_t)NWG * TWB * 8;
+  static constexpr size_t OFF_BAR = OFF_TWB + TWB_BYTES;
   static constexpr size_t OFF_SCHED = OFF_BAR + 8 * 3 * NWG + 8;
   static constexpr size_t BYTES = OFF_SCHED + 32 * NWG;
   static_assert(BYTES <= 227 * 1024, "shared memory budget");
@@ -158,6 +177,7 @@ struct WG {
   float2 *buf;        // SMEM transpose buffer
   float2 *stg;        // SMEM input staging (one item)
   float2 *tws;        // SMEM twiddle staging (one item)
+  float2 *twb;        // SMEM row of twiddle table B (two-level tables)
   uint32_t ph_mma, ph_stg, ph_tws;
   bool fail;
   bool tws_inflight;  // warp 0: a twiddle copy has not been waited on
@@ -292,20 +312,25 @@ __device__ __forceinline__ void issue_input(const PRun &P, const CUtensorMap *tm
   __syncwarp();
 }
 
-// ---- TMA issue (warp 0, converged): the inter-pass twiddles of a
-// first-pass item
+// ---- TMA issue (warp 0, converged): the inter-pass twiddles of a strided
+// item -- the [k][vl] box of table A and, for two-level tables, the row of
+// table B for the item's vh
 template <class G>
-__device__ __forceinline__ void issue_twiddles(const CUtensorMap *tm, long long item,
-                                               const WG &w) {
+__device__ __forceinline__ void issue_twiddles(const PRun &P, const CUtensorMap *tm,
+                                               long long item, const WG &w) {
   if constexpr (G::TW_SMEM) {
     const long long u0 = item << G::LOG2GG;
-    const int v0 = (int)(u0 & ((1ll << G::LOG2UPER) - 1));
+    const long long v0 = u0 & ((1ll << G::LOG2UPER) - 1);
+    const int vl0 = (int)(v0 & ((1 << G::LOG2VL) - 1));
     const uint32_t dst = smem_u32(w.tws);
     if (elect_one()) {
-      mbar_expect_tx(w.bar_tws, G::GPTS * 8);
+      mbar_expect_tx(w.bar_tws, G::GPTS * 8 + (G::TW2L ? G::L * 8 : 0));
 #pragma unroll
       for (int k0 = 0; k0 < G::L; k0 += G::TMA_ROWS)
-        tma_load_3d(dst + k0 * G::GG * 8, tm, 2 * v0, k0, 0, w.bar_tws);
+        tma_load_3d(dst + k0 * G::GG * 8, tm, 2 * vl0, k0, 0, w.bar_tws);
+      if (G::TW2L)
+        tma_load_1d(smem_u32(w.twb), P.tw_b + ((v0 >> G::LOG2VL) << G::LOG2L), G::L * 8,
+                    w.bar_tws);
     }
     __syncwarp();
   }
@@ -410,19 +435,31 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, 
   }
   const long long b = u >> G::LOG2UPER;
   const long long v = u & ((1ll << G::LOG2UPER) - 1);
-  float2 *dst = P.out + ((b & P.out_bmask) << G::LOG2N) + v * G::OUT_VSTRIDE +
-                klow * G::OUT_STRIDE;
+  // kFirst after SP stages: sequence b = (transform, p) -> transform-major,
+  // k above p
+  const long long bt = b >> G::LOG2PRE, bp = b & ((1ll << G::LOG2PRE) - 1);
+  float2 *dst = P.out + ((bt & P.out_bmask) << G::LOG2NT) + (bp << G::LOG2UPER) +
+                v * G::OUT_VSTRIDE + klow * G::OUT_STRIDE;
   constexpr long long JS = G::OUT_STRIDE << (G::LOG2L - G::LOG2R);
-  // twiddle of output k = klow + j r^(S-1): SMEM staging [k][ul], or global
+  // twiddle of output k = klow + j r^(S-1): table A staged as [k][ul] in SMEM,
+  // or read from global [k][vl]; two-level: times B[vh][k]
   const float2 *tws = w.tws + klow * G::GG + ul;
   constexpr int TJS = G::GG << (G::LOG2L - G::LOG2R);
-  const float2 *twg = P.tw_out + ((long long)klow << G::LOG2UPER) + v;
-  constexpr long long TWG = 1ll << (G::LOG2UPER + G::LOG2L - G::LOG2R);
+  const long long vl = v & ((1ll << G::LOG2VL) - 1), vh = v >> G::LOG2VL;
+  const float2 *twg = P.tw_out + ((long long)klow << G::LOG2VL) + vl;
+  constexpr long long TWG = 1ll << (G::LOG2VL + G::LOG2L - G::LOG2R);
+  const float2 *twbs = w.twb + klow;
+  const float2 *twbg = P.tw_b + (vh << G::LOG2L) + klow;
+  constexpr int TBJ = 1 << (G::LOG2L - G::LOG2R);
 #pragma unroll
   for (int j = 0; j < R; ++j) {
     float2 y = make_float2(d[2 * j], d[2 * j + 1]);
-    if (G::TW_SMEM) y = cmul(y, tws[j * TJS]);
-    else if (G::TW_OUT) y = cmul(y, __ldg(twg + j * TWG));
+    if (G::TW_SMEM) {
+      y = G::TW2L ? cmul(y, cmul(tws[j * TJS], twbs[j * TBJ])) : cmul(y, tws[j * TJS]);
+    } else if (G::TW_OUT) {
+      y = G::TW2L ? cmul(y, cmul(__ldg(twg + j * TWG), __ldg(twbg + j * TBJ)))
+                  : cmul(y, __ldg(twg + j * TWG));
+    }
     if (OUT_L2)
       __stcg(dst + j * JS, y);
     else
@@ -459,7 +496,7 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
     fence_after_sync();
     issue_stage<R, PREC>(w.slot, w.img_addr + (S == 1 ? P.last_img : 0), w.bar_mma);
     if (G::TW_SMEM) {
-      issue_twiddles<G>(tm_tw, item, w);
+      issue_twiddles<G>(P, tm_tw, item, w);
       w.tws_inflight = true;
     }
     mid.issue(w);
@@ -555,6 +592,7 @@ __device__ __forceinline__ void init_wg(WG &w, uint32_t tbase, unsigned char *sm
   w.buf = reinterpret_cast<float2 *>(smem + SM::OFF_BUF) + wg * SM::PTS;
   w.stg = reinterpret_cast<float2 *>(smem + SM::OFF_STG) + wg * SM::PTS;
   w.tws = reinterpret_cast<float2 *>(smem + SM::OFF_TWS) + (SM::TWS_BYTES ? wg * SM::PTS : 0);
+  w.twb = reinterpret_cast<float2 *>(smem + SM::OFF_TWB) + wg * SM::TWB_PER_WG;
   w.ph_mma = w.ph_stg = w.ph_tws = 0;
   w.fail = false;
   w.tws_inflight = false;
@@ -574,11 +612,11 @@ struct StaticNext {
   __device__ void publish() {}
 };
 
-template <int R, int PREC, int S, int SO, int ROLE>
-__global__ void __launch_bounds__(Geo<R, S, SO, ROLE>::THREADS, 1)
+template <int R, int PREC, int S, int SO, int ROLE, int SP>
+__global__ void __launch_bounds__(Geo<R, S, SO, ROLE, SP>::THREADS, 1)
     dft_pass_kernel(const __grid_constant__ GArgs a) {
-  using G = Geo<R, S, SO, ROLE>;
-  using SM = SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM>;
+  using G = Geo<R, S, SO, ROLE, SP>;
+  using SM = SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM, G::TWB>;
   extern __shared__ __align__(1024) unsigned char smem[];
   float2 *tw = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
   uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + SM::OFF_BAR);
@@ -792,8 +830,8 @@ __global__ void __launch_bounds__(Geo<R, S1, S2, kFirst>::THREADS, 1)
     dft_fused_kernel(const __grid_constant__ GArgs a) {
   static_assert(S1 >= 2 && S2 >= 2, "the fused schedule needs an SMEM barrier per item");
   using G1 = Geo<R, S1, S2, kFirst>;
-  using G2 = Geo<R, S2, S1, kSecond, G1::NWG>;
-  using SM = SmemLayout<R, G1::NWG, G1::TW_ENTRIES, G2::TW_ENTRIES, G1::TW_SMEM>;
+  using G2 = Geo<R, S2, S1, kSecond, 0, G1::NWG>;
+  using SM = SmemLayout<R, G1::NWG, G1::TW_ENTRIES, G2::TW_ENTRIES, G1::TW_SMEM, G1::TWB>;
   constexpr int NWG = G1::NWG;
   extern __shared__ __align__(1024) unsigned char smem[];
   float2 *tw1 = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);

@@ -3,17 +3,22 @@
 
 namespace tcu {
 
-cudaError_t launch_pass_r32(int prec, int s, int so, int role, const GArgs &a, int num_sms,
-                            cudaStream_t st) {
+// (stages, stages after (kFirst) or before (kSecond), role, stages before)
+cudaError_t launch_pass_r32(int prec, int s, int so, int role, int sp, const GArgs &a,
+                            int num_sms, cudaStream_t st) {
   constexpr int R = 32;
-  TCU_PASS_CASE(1, 0, kSingle)
-  TCU_PASS_CASE(2, 0, kSingle)
-  TCU_PASS_CASE(1, 2, kFirst)   // n = 32^3
-  TCU_PASS_CASE(2, 1, kSecond)
-  TCU_PASS_CASE(2, 1, kFirst)
-  TCU_PASS_CASE(1, 2, kSecond)
-  TCU_PASS_CASE(2, 2, kFirst)   // n = 32^4
-  TCU_PASS_CASE(2, 2, kSecond)
+  TCU_PASS_CASE(1, 0, kSingle, 0)
+  TCU_PASS_CASE(2, 0, kSingle, 0)
+  TCU_PASS_CASE(1, 2, kFirst, 0)   // n = 32^3: 1 + 2
+  TCU_PASS_CASE(2, 1, kSecond, 0)
+  TCU_PASS_CASE(2, 2, kFirst, 0)   // n = 32^4: 2 + 2
+  TCU_PASS_CASE(2, 2, kSecond, 0)
+  TCU_PASS_CASE(1, 4, kFirst, 0)   // n = 32^5: 1 + 2 + 2
+  TCU_PASS_CASE(2, 2, kFirst, 1)
+  TCU_PASS_CASE(2, 3, kSecond, 0)
+  TCU_PASS_CASE(2, 4, kFirst, 0)   // n = 32^6: 2 + 2 + 2
+  TCU_PASS_CASE(2, 2, kFirst, 2)
+  TCU_PASS_CASE(2, 4, kSecond, 0)
   return cudaErrorInvalidValue;
 }
 
@@ -22,10 +27,6 @@ cudaError_t launch_fused_r32(int prec, int s1, int s2, const GArgs &a, int num_s
   constexpr int R = 32;
   TCU_FUSED_CASE(2, 2)
   return cudaErrorInvalidValue;
-}
-
-cudaError_t launch_tile_r32(int prec, const PassArgs &a, long long grid, cudaStream_t st) {
-  return prec == 3 ? launch_tile_t<32, 3>(a, grid, st) : launch_tile_t<32, 1>(a, grid, st);
 }
 
 }  // namespace tcu

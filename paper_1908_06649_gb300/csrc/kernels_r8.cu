@@ -3,21 +3,30 @@
 
 namespace tcu {
 
-cudaError_t launch_pass_r8(int prec, int s, int so, int role, const GArgs &a, int num_sms,
-                           cudaStream_t st) {
+// (stages, stages after (kFirst) or before (kSecond), role, stages before)
+cudaError_t launch_pass_r8(int prec, int s, int so, int role, int sp, const GArgs &a,
+                           int num_sms, cudaStream_t st) {
   constexpr int R = 8;
-  TCU_PASS_CASE(1, 0, kSingle)
-  TCU_PASS_CASE(2, 0, kSingle)
-  TCU_PASS_CASE(3, 0, kSingle)
-  TCU_PASS_CASE(2, 2, kFirst)   // n = 8^4
-  TCU_PASS_CASE(2, 2, kSecond)
-  TCU_PASS_CASE(2, 3, kFirst)   // n = 8^5
-  TCU_PASS_CASE(3, 2, kSecond)
-  TCU_PASS_CASE(3, 2, kFirst)
-  TCU_PASS_CASE(2, 3, kSecond)
-  TCU_PASS_CASE(3, 3, kFirst)   // n = 8^6
-  TCU_PASS_CASE(3, 3, kSecond)
-  TCU_PASS_CASE(3, 4, kSecond)  // n = 8^7 after a 4-stage tile pass
+  TCU_PASS_CASE(1, 0, kSingle, 0)
+  TCU_PASS_CASE(2, 0, kSingle, 0)
+  TCU_PASS_CASE(3, 0, kSingle, 0)
+  TCU_PASS_CASE(2, 2, kFirst, 0)   // n = 8^4: 2 + 2
+  TCU_PASS_CASE(2, 2, kSecond, 0)
+  TCU_PASS_CASE(1, 4, kFirst, 0)   // n = 8^5: 1 + 2 + 2
+  TCU_PASS_CASE(2, 2, kFirst, 1)
+  TCU_PASS_CASE(2, 3, kSecond, 0)
+  TCU_PASS_CASE(2, 4, kFirst, 0)   // n = 8^6: 2 + 2 + 2
+  TCU_PASS_CASE(2, 2, kFirst, 2)
+  TCU_PASS_CASE(2, 4, kSecond, 0)
+  TCU_PASS_CASE(2, 5, kFirst, 0)   // n = 8^7: 2 + 2 + 3
+  TCU_PASS_CASE(2, 3, kFirst, 2)
+  TCU_PASS_CASE(3, 4, kSecond, 0)
+  TCU_PASS_CASE(2, 6, kFirst, 0)   // n = 8^8: 2 + 3 + 3
+  TCU_PASS_CASE(3, 3, kFirst, 2)
+  TCU_PASS_CASE(3, 5, kSecond, 0)
+  TCU_PASS_CASE(3, 6, kFirst, 0)   // n = 8^9: 3 + 3 + 3
+  TCU_PASS_CASE(3, 3, kFirst, 3)
+  TCU_PASS_CASE(3, 6, kSecond, 0)
   return cudaErrorInvalidValue;
 }
 
@@ -25,14 +34,7 @@ cudaError_t launch_fused_r8(int prec, int s1, int s2, const GArgs &a, int num_sm
                             cudaStream_t st) {
   constexpr int R = 8;
   TCU_FUSED_CASE(2, 2)
-  TCU_FUSED_CASE(2, 3)
-  TCU_FUSED_CASE(3, 2)
-  TCU_FUSED_CASE(3, 3)
   return cudaErrorInvalidValue;
-}
-
-cudaError_t launch_tile_r8(int prec, const PassArgs &a, long long grid, cudaStream_t st) {
-  return prec == 3 ? launch_tile_t<8, 3>(a, grid, st) : launch_tile_t<8, 1>(a, grid, st);
 }
 
 }  // namespace tcu

@@ -5,18 +5,18 @@
 
 namespace tcu {
 
-template <int R, int PREC, int S, int SO, int ROLE>
+template <int R, int PREC, int S, int SO, int ROLE, int SP>
 cudaError_t launch_pass_t(const GArgs &a, int num_sms, cudaStream_t st) {
-  using G = Geo<R, S, SO, ROLE>;
-  const size_t sm = SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM>::BYTES;
-  cudaError_t e = cudaFuncSetAttribute(dft_pass_kernel<R, PREC, S, SO, ROLE>,
+  using G = Geo<R, S, SO, ROLE, SP>;
+  const size_t sm = SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM, G::TWB>::BYTES;
+  cudaError_t e = cudaFuncSetAttribute(dft_pass_kernel<R, PREC, S, SO, ROLE, SP>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)sm);
   if (e != cudaSuccess) return e;
   const long long nitems = (a.p[0].U + G::GG - 1) >> G::LOG2GG;
   long long grid = (nitems + G::NWG - 1) / G::NWG;
   if (grid > num_sms) grid = num_sms;
-  dft_pass_kernel<R, PREC, S, SO, ROLE><<<(unsigned)grid, G::THREADS, sm, st>>>(a);
+  dft_pass_kernel<R, PREC, S, SO, ROLE, SP><<<(unsigned)grid, G::THREADS, sm, st>>>(a);
   return cudaGetLastError();
 }
 
@@ -33,24 +33,12 @@ cudaError_t launch_fused_t(const GArgs &a, int num_sms, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-template <int R, int PREC>
-cudaError_t launch_tile_t(const PassArgs &a, long long grid, cudaStream_t st) {
-  size_t sm = Cfg<R>::SMEM_BYTES;
-  if (sm < 120 * 1024) sm = 120 * 1024;  // one CTA per SM: it takes all of TMEM
-  cudaError_t e = cudaFuncSetAttribute(dft_tile_kernel<R, PREC>,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                       (int)sm);
-  if (e != cudaSuccess) return e;
-  dft_tile_kernel<R, PREC><<<(unsigned)grid, kThreads, sm, st>>>(a);
-  return cudaGetLastError();
-}
-
-// Supported (s, so, role) combinations of the warpgroup pass kernel for
+// Supported (s, so, role, sp) combinations of the warpgroup pass kernel for
 // radix R, listed as a compile-time table; the plan only asks for these.
-#define TCU_PASS_CASE(S, SO, ROLE)                                                  \
-  if (s == S && so == SO && role == ROLE)                                           \
-    return prec == 3 ? launch_pass_t<R, 3, S, SO, ROLE>(a, num_sms, st)             \
-                     : launch_pass_t<R, 1, S, SO, ROLE>(a, num_sms, st);
+#define TCU_PASS_CASE(S, SO, ROLE, SP)                                              \
+  if (s == S && so == SO && role == ROLE && sp == SP)                               \
+    return prec == 3 ? launch_pass_t<R, 3, S, SO, ROLE, SP>(a, num_sms, st)         \
+                     : launch_pass_t<R, 1, S, SO, ROLE, SP>(a, num_sms, st);
 #define TCU_FUSED_CASE(S1, S2)                                                      \
   if (s1 == S1 && s2 == S2)                                                         \
     return prec == 3 ? launch_fused_t<R, 3, S1, S2>(a, num_sms, st)                 \

@@ -16,14 +16,16 @@
 //     Bf[2j+1][2c] = -Im w, Bf[2j+1][2c+1] = Re w,   w = w_r^{jc},
 // gives [Re y0, Im y0, Re y1, ...].
 //
-// Passes.  The k stages are grouped into at most two HBM passes (the
-// four-step split n = n1 * n2): pass 1 transforms the n2 stride-n2
-// subsequences of length n1 and multiplies by w_n^{b k1}; pass 2 transforms
-// the n1 contiguous rows of length n2 and writes y[k1 + n1 k2].  A pass whose
-// sub-transforms fit 128 data rows runs on the warpgroup kernel
-// (group_kernel.cuh); longer ones on the tile kernel (tile_kernel.cuh).  Two
-// warpgroup passes of >= 2 stages each run fused in one launch with an
-// L2-resident intermediate.
+// Passes.  The k stages are grouped into at most three HBM passes of at most
+// two stages (three for r = 8) -- the four-step split n = n1 * n2 applied
+// recursively, so that every pass's sub-transforms fit one warpgroup item of
+// 128 data rows (group_kernel.cuh).  Pass p splits each length-M_p sequence
+// left by the passes before it (M_1 = n) into L_p rows of n2_p = M_p / L_p
+// columns: it transforms the strided columns, multiplies by w_{M_p}^{k v}
+// and stores row k of sequence q as row (k, q) of the next pass's input,
+// transform-major with k above q; the last pass transforms contiguous rows
+// and writes y[q + k * n / L] in natural order.  A two-pass transform may
+// instead run fused in one launch with an L2-resident intermediate.
 
 #include <cuda.h>
 #include <cudaTypedefs.h>
@@ -48,22 +50,23 @@ using namespace tcu;
 
 namespace {
 
-enum PassKind { kTilePass = 0, kGroupPass = 1 };
+constexpr int kMaxPasses = 3;
 
 struct PassPlan {
-  int kind;        // kTilePass or kGroupPass
-  int s;
-  int log2L;
-  int log2G;       // tile kernel: sub-transforms per tile
-  long long U, Uper;
-  int log2Uper;
-  long long in_vstride, in_stride, out_vstride, out_stride;
-  int tw_log2N, tw_h;  // tile kernel: inter-pass twiddle, two-level table
-  int modes[3];        // group kernel: row map of first / middle / last stage
+  int s;            // stages
+  int role;         // kSingle, kFirst (strided) or kSecond (last of several)
+  int so;           // kFirst: stages after this pass; kSecond: stages before
+  int sp;           // kFirst: stages before this pass
+  int log2L;        // sub-transform length L = r^s
+  long long U;      // sub-transforms in the pass
+  int modes[3];     // row map of the first / middle / last stage
   unsigned long long swz_tab;
   bool last;
-  float2 *twL[2];      // tile kernel: w_L^e          [dir index]
-  float2 *tw_stage[2]; // group kernel: [t][j][lo]    [dir index]
+  float2 *tw_stage[2];   // stage twiddles [t][j][lo]          [dir index]
+  // kFirst: w_M^{k v}, M = r^(s + so): A [k][vl], B [vh][k] (v = vh 256 + vl,
+  // B only when n2 = r^so exceeds 256)
+  float2 *tw_a[2], *tw_b[2];
+  CUtensorMap tw_map[2];  // TMA map of tw_a[d]
 };
 
 thread_local int g_last_error = TCU_DFT_OK;
@@ -81,12 +84,9 @@ struct tcu_dft_plan_s {
   int r, log2r, k, precision;
   int npasses;
   int num_sms;
-  PassPlan pass[2];
-  float *bimg[2];          // [dir index] hi | lo images
-  float2 *twA[2], *twB[2]; // tile kernel pass 1: two-level w_n^e
-  float2 *tw_out[2];       // group kernel pass 1: w_n^{b k} as [k][b]
-  CUtensorMap tw_map[2];   // TMA map of tw_out[d]
-  float2 *scratch;         // intermediate (full size, or the fused ring)
+  PassPlan pass[kMaxPasses];
+  float *bimg[2];          // [dir index] hi | lo | scaled hi | scaled lo images
+  float2 *scratch[2];      // intermediates (or the fused ring in scratch[0])
   // fused two-pass schedule
   bool fused;
   int log2C, nchunks, lag, ring_chunks;
@@ -186,13 +186,6 @@ void build_images(int r, int sign, int log2n, std::vector<float> &out) {
   }
 }
 
-std::vector<float2> twiddle_table(long long period, long long count, long long step,
-                                  int sign) {
-  std::vector<float2> t((size_t)count);
-  for (long long e = 0; e < count; ++e) t[(size_t)e] = root(e * step, period, sign);
-  return t;
-}
-
 // Stage twiddles of a warpgroup pass: for t = 1 .. s-1 a block [j][lo],
 // j < r, lo < r^(s-t), holding w_L^{j * lo * r^(t-1)}.
 std::vector<float2> stage_twiddles(int r, int s, int sign) {
@@ -208,19 +201,6 @@ std::vector<float2> stage_twiddles(int r, int s, int sign) {
   }
   if (t.empty()) t.push_back(make_float2(1.f, 0.f));
   return t;
-}
-
-// Largest stage count per pass: tile kernel (a sub-transform fills at most one
-// SMEM tile) and warpgroup kernel (a sub-transform fits 128 rows).
-int max_tile_stages(int r) { return r == 8 ? 4 : (r == 16 ? 3 : 2); }
-int max_group_stages(int r) { return r == 8 ? 3 : 2; }
-
-// Two warpgroup passes of k stages: the strided first pass takes the smaller
-// half -- its sub-transforms are shorter, so an item spans more adjacent
-// columns and its TMA boxes have wider rows.
-void split_two_passes(int k, int stages[2]) {
-  stages[0] = k / 2;
-  stages[1] = k - stages[0];
 }
 
 int stage_mode(const int modes[3], int t, int S) {
@@ -319,39 +299,118 @@ int upload(T **dst, const std::vector<T> &src) {
   return TCU_DFT_OK;
 }
 
+// Stages per pass.  Passes hold at most two stages (three for r = 8, whose
+// 3-stage sub-transforms of 512 points still fit a 128-row item); up to
+// three passes; the earlier passes take the smaller shares, so the strided
+// passes have shorter sub-transforms, more adjacent columns per item and
+// wider TMA rows.  Returns the number of passes, 0 if n is too long.
+int plan_stages(int r, int k, int st[kMaxPasses]) {
+  const int sg = r == 8 ? 3 : 2;
+  if (k <= sg) {
+    st[0] = k;
+    return 1;
+  }
+  int P = (k + 1) / 2;
+  if (P > kMaxPasses) P = kMaxPasses;
+  const int base = k / P, extra = k % P;
+  for (int i = 0; i < P; ++i) {
+    st[i] = base + (i >= P - extra ? 1 : 0);
+    if (st[i] > sg) return 0;
+  }
+  return P;
+}
+
+// Role, neighbouring stage counts, size and row maps of pass `pi`.
+void pass_geometry(PassPlan &pp, int pi, int P, const int st[kMaxPasses], int k, int r,
+                   long long n, long long batch) {
+  int before = 0;
+  for (int i = 0; i < pi; ++i) before += st[i];
+  pp.s = st[pi];
+  pp.log2L = ilog2(r) * pp.s;
+  pp.last = (pi == P - 1);
+  if (P == 1) {
+    pp.role = kSingle;
+    pp.so = pp.sp = 0;
+  } else if (pp.last) {
+    pp.role = kSecond;
+    pp.so = before;
+    pp.sp = 0;
+  } else {
+    pp.role = kFirst;
+    pp.so = k - before - pp.s;
+    pp.sp = before;
+  }
+  pp.U = batch * (n >> pp.log2L);
+  pp.modes[0] = pp.role == kFirst ? kUF : kQF;
+  pp.modes[1] = kUF;
+  pp.modes[2] = pp.role == kSingle ? kRQF : kUF;
+  pp.swz_tab = choose_swizzle(r, pp.s, pp.modes);
+}
+
+// Inter-pass twiddles of a strided pass: w_M^{k v}, k < L = r^s,
+// v < n2 = r^so, M = L n2; A[k][vl] for vl < min(n2, 256) and, if n2 > 256,
+// B[vh][k] = w_M^{k vh 256}.
+void pass_twiddles(int r, int s, int so, int sign, std::vector<float2> &A,
+                   std::vector<float2> &B) {
+  long long L = 1, n2 = 1;
+  for (int i = 0; i < s; ++i) L *= r;
+  for (int i = 0; i < so; ++i) n2 *= r;
+  const long long M = L * n2, VL = n2 > 256 ? 256 : n2;
+  A.resize((size_t)(L * VL));
+  for (long long k = 0; k < L; ++k)
+    for (long long vl = 0; vl < VL; ++vl) A[(size_t)(k * VL + vl)] = root(k * vl, M, sign);
+  B.clear();
+  if (n2 > VL) {
+    B.resize((size_t)((n2 / VL) * L));
+    for (long long vh = 0; vh < n2 / VL; ++vh)
+      for (long long k = 0; k < L; ++k)
+        B[(size_t)(vh * L + k)] = root(k * vh * VL, M, sign);
+  }
+}
+
+// TMA map of table A of a strided pass (boxes of GG columns x L rows).
+bool twiddle_map(CUtensorMap *m, const float2 *A, int r, const PassPlan &pp) {
+  const long long L = 1ll << pp.log2L;
+  long long n2 = 1;
+  for (int i = 0; i < pp.so; ++i) n2 *= r;
+  const long long VL = n2 > 256 ? 256 : n2;
+  const long long gg = (128ll * r) >> pp.log2L;
+  return encode_map(m, A, VL, L, 1, L * VL, (int)gg, L < 256 ? (int)L : 256);
+}
+
+// TMA map of a strided pass's input: sequences of M = L n2 points, batch *
+// r^sp of them, seen as [sequence][row a][column v].
+bool input_map(CUtensorMap *m, const void *in, const tcu_dft_plan_s *p, const PassPlan &pp) {
+  const long long L = 1ll << pp.log2L;
+  long long n2 = 1, pre = 1;
+  for (int i = 0; i < pp.so; ++i) n2 *= p->r;
+  for (int i = 0; i < pp.sp; ++i) pre *= p->r;
+  const long long gg = (128ll * p->r) >> pp.log2L;
+  return encode_map(m, in, n2, L, p->batch * pre, L * n2, (int)gg, L < 256 ? (int)L : 256);
+}
+
 void free_plan(tcu_dft_plan_s *p) {
   if (!p) return;
   for (int d = 0; d < 2; ++d) {
     cudaFree(p->bimg[d]);
-    cudaFree(p->twA[d]);
-    cudaFree(p->twB[d]);
-    cudaFree(p->tw_out[d]);
-    for (int i = 0; i < 2; ++i) {
-      cudaFree(p->pass[i].twL[d]);
+    for (int i = 0; i < kMaxPasses; ++i) {
       cudaFree(p->pass[i].tw_stage[d]);
+      cudaFree(p->pass[i].tw_a[d]);
+      cudaFree(p->pass[i].tw_b[d]);
     }
+    cudaFree(p->scratch[d]);
   }
-  cudaFree(p->scratch);
   cudaFree(p->counters);
   cudaFree(p->err);
   delete p;
 }
 
-int tile_points(int r) { return r == 8 ? 4096 : 8192; }
-
 // ---------------------------------------------------------------- launches
-cudaError_t tile_dispatch(int r, int prec, const PassArgs &a, long long grid,
+cudaError_t pass_dispatch(int r, int prec, const PassPlan &pp, const GArgs &a, int num_sms,
                           cudaStream_t st) {
-  if (r == 8) return launch_tile_r8(prec, a, grid, st);
-  if (r == 16) return launch_tile_r16(prec, a, grid, st);
-  return launch_tile_r32(prec, a, grid, st);
-}
-
-cudaError_t pass_dispatch(int r, int prec, int s, int so, int role, const GArgs &a,
-                          int num_sms, cudaStream_t st) {
-  if (r == 8) return launch_pass_r8(prec, s, so, role, a, num_sms, st);
-  if (r == 16) return launch_pass_r16(prec, s, so, role, a, num_sms, st);
-  return launch_pass_r32(prec, s, so, role, a, num_sms, st);
+  if (r == 8) return launch_pass_r8(prec, pp.s, pp.so, pp.role, pp.sp, a, num_sms, st);
+  if (r == 16) return launch_pass_r16(prec, pp.s, pp.so, pp.role, pp.sp, a, num_sms, st);
+  return launch_pass_r32(prec, pp.s, pp.so, pp.role, pp.sp, a, num_sms, st);
 }
 
 cudaError_t fused_dispatch(int r, int prec, int s1, int s2, const GArgs &a, int num_sms,
@@ -377,7 +436,8 @@ PRun group_pass(const tcu_dft_plan_s *p, int pi, int di, const float2 *in, float
   g.in_bmask = in_bmask;
   g.out_bmask = out_bmask;
   g.U = pp.U;
-  g.tw_out = (pi == 0 && p->npasses == 2) ? p->tw_out[di] : nullptr;
+  g.tw_out = pp.tw_a[di];
+  g.tw_b = pp.tw_b[di];
   g.tw_stage = pp.tw_stage[di];
   g.swz_tab = pp.swz_tab;
   // the inverse's last stage uses the F images scaled by 1/n
@@ -385,24 +445,21 @@ PRun group_pass(const tcu_dft_plan_s *p, int pi, int di, const float2 *in, float
   return g;
 }
 
-int pass_role(const tcu_dft_plan_s *p, int pi) {
-  return p->npasses == 1 ? kSingle : (pi == 0 ? kFirst : kSecond);
-}
+// Tables of a plan for one direction d: F images, stage twiddles and the
+// inter-pass twiddles, as host vectors (uploaded by the caller).
+struct DirTables {
+  std::vector<float> img;
+  std::vector<float2> stage[kMaxPasses], A[kMaxPasses], B[kMaxPasses];
+};
 
-int other_stages(const tcu_dft_plan_s *p, int pi) {
-  return p->npasses == 1 ? 0 : p->pass[1 - pi].s;
-}
-
-// TMA maps of a first (strided) warpgroup pass: its input x[b][a][v] and
-// its inter-pass twiddles.
-bool first_pass_maps(const tcu_dft_plan_s *p, int di, const void *in, GArgs *g) {
-  const PassPlan &p1 = p->pass[0];
-  const long long n1 = 1ll << p1.log2L, n2 = p->n / n1;
-  const long long gg1 = (128ll * p->r) >> p1.log2L;
-  const int box_rows = n1 < 256 ? (int)n1 : 256;
-  if (!encode_map(&g->tm_in, in, n2, n1, p->batch, p->n, (int)gg1, box_rows)) return false;
-  g->tm_tw = p->tw_map[di];
-  return true;
+void dir_tables(const tcu_dft_plan_s *p, int d, DirTables &t) {
+  const int sign = d == 0 ? -1 : 1;
+  build_images(p->r, sign, ilog2(p->n), t.img);
+  for (int pi = 0; pi < p->npasses; ++pi) {
+    const PassPlan &pp = p->pass[pi];
+    t.stage[pi] = stage_twiddles(p->r, pp.s, sign);
+    if (pp.role == kFirst) pass_twiddles(p->r, pp.s, pp.so, sign, t.A[pi], t.B[pi]);
+  }
 }
 
 // ------------------------------------------- fixed memory of exec_noalloc
@@ -416,7 +473,7 @@ constexpr int kNaStageTw = 1024;                    // stage twiddles of a pass
 static __device__ __align__(256) float2 g_na_scratch[kNaMaxPoints];
 static __device__ __align__(256) float g_na_img[2][kNaImgFloats];
 static __device__ __align__(256) float2 g_na_tw_stage[2][2][kNaStageTw];
-static __device__ __align__(256) float2 g_na_tw_out[2][kNaMaxN];
+static __device__ __align__(256) float2 g_na_tw_out[2][kNaMaxN];  // A, then B
 static __device__ __align__(256) int g_na_err;
 
 struct NaDevice {
@@ -480,35 +537,9 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
     m *= r;
     ++k;
   }
-  if (m != n || k < 1) {
-    g_last_error = TCU_DFT_ERR_UNSUPPORTED;
-    return nullptr;
-  }
-  // Pass grouping: prefer the warpgroup kernel (sub-transforms of <= 128
-  // rows), fall back to the tile kernel for longer sub-transforms.
-  const int sg = max_group_stages(r), stl = max_tile_stages(r);
-  int stages[2] = {0, 0}, kinds[2] = {kGroupPass, kGroupPass}, npasses;
-  if (k <= sg) {
-    npasses = 1;
-    stages[0] = k;
-  } else if (k <= 2 * sg) {
-    npasses = 2;
-    split_two_passes(k, stages);
-  } else if (k <= stl + sg) {
-    npasses = 2;
-    stages[0] = k - sg;
-    kinds[0] = kTilePass;
-    stages[1] = sg;
-  } else if (k <= 2 * stl) {
-    npasses = 2;
-    stages[0] = (k + 1) / 2;
-    stages[1] = k - stages[0];
-    kinds[0] = kinds[1] = kTilePass;
-  } else {
-    g_last_error = TCU_DFT_ERR_UNSUPPORTED;
-    return nullptr;
-  }
-  if ((long long)batch * n > (1ll << 40)) {
+  int st[kMaxPasses] = {0, 0, 0};
+  const int npasses = (m == n && k >= 1) ? plan_stages(r, k, st) : 0;
+  if (npasses == 0 || (long long)batch * n > (1ll << 40)) {
     g_last_error = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
   }
@@ -533,78 +564,19 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
   p->npasses = npasses;
   p->device = dev;
   p->num_sms = prop.multiProcessorCount;
-  const int log2n = ilog2(n);
+  for (int pi = 0; pi < npasses; ++pi) pass_geometry(p->pass[pi], pi, npasses, st, k, r, n, batch);
   int rc = TCU_DFT_OK;
-  for (int pi = 0; pi < npasses && rc == TCU_DFT_OK; ++pi) {
-    PassPlan &pp = p->pass[pi];
-    pp.kind = kinds[pi];
-    pp.s = stages[pi];
-    pp.log2L = log2r * pp.s;
-    pp.log2G = ilog2(tile_points(r)) - pp.log2L;
-    pp.last = (pi == npasses - 1);
-    const long long L = 1ll << pp.log2L;
-    if (npasses == 1) {
-      pp.U = batch;
-      pp.Uper = 1;
-      pp.in_vstride = n;
-      pp.in_stride = 1;
-      pp.out_vstride = n;
-      pp.out_stride = 1;
-      pp.tw_log2N = 0;
-    } else if (pi == 0) {
-      const long long n2 = n / L;  // four-step: x[n2 a + b], DFT over a
-      pp.U = batch * n2;
-      pp.Uper = n2;
-      pp.in_vstride = 1;
-      pp.in_stride = n2;
-      pp.out_vstride = 1;
-      pp.out_stride = n2;
-      pp.tw_log2N = log2n;       // w_n^{b k1}
-      pp.tw_h = (log2n + 1) / 2;
-    } else {
-      const long long n1 = n / L;  // rows k1 of the four-step, DFT over b
-      pp.U = batch * n1;
-      pp.Uper = n1;
-      pp.in_vstride = L;
-      pp.in_stride = 1;
-      pp.out_vstride = 1;
-      pp.out_stride = n1;
-      pp.tw_log2N = 0;
-    }
-    pp.log2Uper = ilog2(pp.Uper);
-    pp.modes[0] = pp.in_stride == 1 ? kQF : kUF;
-    pp.modes[1] = kUF;
-    pp.modes[2] = pp.out_stride == 1 ? kRQF : kUF;
-    pp.swz_tab = choose_swizzle(r, pp.s, pp.modes);
-    for (int d = 0; d < 2 && rc == TCU_DFT_OK; ++d) {
-      const int sign = d == 0 ? -1 : 1;
-      if (pp.kind == kTilePass)
-        rc = upload(&pp.twL[d], twiddle_table(L, L, 1, sign));
-      else
-        rc = upload(&pp.tw_stage[d], stage_twiddles(r, pp.s, sign));
-    }
-  }
   for (int d = 0; d < 2 && rc == TCU_DFT_OK; ++d) {
-    const int sign = d == 0 ? -1 : 1;
-    std::vector<float> img;
-    build_images(r, sign, log2n, img);
-    rc = upload(&p->bimg[d], img);
-    if (rc == TCU_DFT_OK && npasses == 2) {
-      if (p->pass[0].kind == kTilePass) {
-        const int h = p->pass[0].tw_h;
-        rc = upload(&p->twA[d], twiddle_table(n, n >> h, 1ll << h, sign));
-        if (rc == TCU_DFT_OK) rc = upload(&p->twB[d], twiddle_table(n, 1ll << h, 1, sign));
-      } else {
-        // [k1][b] = w_n^{b k1}, b < n2, k1 < n1
-        const long long n1 = 1ll << p->pass[0].log2L, n2 = n / n1;
-        std::vector<float2> t((size_t)n);
-        for (long long k1 = 0; k1 < n1; ++k1)
-          for (long long b = 0; b < n2; ++b) t[(size_t)(k1 * n2 + b)] = root(b * k1, n, sign);
-        rc = upload(&p->tw_out[d], t);
-        const long long gg1 = (128ll * r) >> p->pass[0].log2L;
-        const int box_rows = n1 < 256 ? (int)n1 : 256;
-        if (rc == TCU_DFT_OK &&
-            !encode_map(&p->tw_map[d], p->tw_out[d], n2, n1, 1, n, (int)gg1, box_rows))
+    DirTables t;
+    dir_tables(p, d, t);
+    rc = upload(&p->bimg[d], t.img);
+    for (int pi = 0; pi < npasses && rc == TCU_DFT_OK; ++pi) {
+      PassPlan &pp = p->pass[pi];
+      rc = upload(&pp.tw_stage[d], t.stage[pi]);
+      if (rc == TCU_DFT_OK && pp.role == kFirst) {
+        rc = upload(&pp.tw_a[d], t.A[pi]);
+        if (rc == TCU_DFT_OK && !t.B[pi].empty()) rc = upload(&pp.tw_b[d], t.B[pi]);
+        if (rc == TCU_DFT_OK && !twiddle_map(&pp.tw_map[d], pp.tw_a[d], r, pp))
           rc = TCU_DFT_ERR_CUDA;
       }
     }
@@ -616,10 +588,9 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
       rc = TCU_DFT_ERR_OOM;
     }
   }
-  if (rc == TCU_DFT_OK && npasses == 2) {
+  if (rc == TCU_DFT_OK && npasses >= 2) {
     const PassPlan &p1 = p->pass[0], &p2 = p->pass[1];
-    p->fused = p1.kind == kGroupPass && p2.kind == kGroupPass && p1.s >= 2 && p2.s >= 2 &&
-               (flags & TCU_DFT_PLAN_FUSE);
+    p->fused = npasses == 2 && p1.s >= 2 && p2.s >= 2 && (flags & TCU_DFT_PLAN_FUSE);
     long long scratch_tf = batch;
     if (p->fused) {
       // chunks of C transforms (a power of two dividing the batch, <= 8);
@@ -639,17 +610,17 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
       p->log2_items_per_chunk = ilog2(n2 / gg1) + log2C;
       scratch_tf = (long long)p->ring_chunks << log2C;
       p->counter_bytes = (size_t)(1 + batch + p->nchunks) * sizeof(int);
-      if (cudaMalloc((void **)&p->counters, p->counter_bytes) != cudaSuccess) {
+      if (rc == TCU_DFT_OK && cudaMalloc((void **)&p->counters, p->counter_bytes) != cudaSuccess) {
         cudaGetLastError();
         rc = TCU_DFT_ERR_OOM;
       }
     }
-    if (rc == TCU_DFT_OK &&
-        cudaMalloc((void **)&p->scratch, (size_t)scratch_tf * n * sizeof(float2)) !=
-            cudaSuccess) {
-      cudaGetLastError();
-      rc = TCU_DFT_ERR_OOM;
-    }
+    for (int i = 0; i < npasses - 1 && rc == TCU_DFT_OK; ++i)
+      if (cudaMalloc((void **)&p->scratch[i], (size_t)scratch_tf * n * sizeof(float2)) !=
+          cudaSuccess) {
+        cudaGetLastError();
+        rc = TCU_DFT_ERR_OOM;
+      }
   }
   if (rc != TCU_DFT_OK) {
     free_plan(p);
@@ -668,17 +639,15 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
   if (in != out && overlaps(in, out, bytes)) return TCU_DFT_ERR_INVALID;
   cudaStream_t st = (cudaStream_t)stream;
   const int di = dir_index(dir);
-  const float scale_last =
-      dir == TCU_DFT_INVERSE ? (float)(1.0 / (double)p->n) : 1.0f;
-
   const bool inverse = dir == TCU_DFT_INVERSE;
   if (p->fused) {
     GArgs g;
     memset(&g, 0, sizeof(g));
     const long long ring_mask = ((long long)p->ring_chunks << p->log2C) - 1;
-    g.p[0] = group_pass(p, 0, di, (const float2 *)in, p->scratch, -1, ring_mask, inverse);
-    g.p[1] = group_pass(p, 1, di, p->scratch, (float2 *)out, ring_mask, -1, inverse);
-    if (!first_pass_maps(p, di, in, &g)) return TCU_DFT_ERR_CUDA;
+    g.p[0] = group_pass(p, 0, di, (const float2 *)in, p->scratch[0], -1, ring_mask, inverse);
+    g.p[1] = group_pass(p, 1, di, p->scratch[0], (float2 *)out, ring_mask, -1, inverse);
+    if (!input_map(&g.tm_in, in, p, p->pass[0])) return TCU_DFT_ERR_CUDA;
+    g.tm_tw = p->pass[0].tw_map[di];
     g.bimg = p->bimg[di];
     g.err = p->err;
     g.counters = p->counters;
@@ -702,50 +671,23 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
     return TCU_DFT_OK;
   }
 
+  // in -> scratch[0] -> scratch[1] -> out
   for (int pi = 0; pi < p->npasses; ++pi) {
     const PassPlan &pp = p->pass[pi];
-    const float2 *src = (pi == 0) ? (const float2 *)in : p->scratch;
-    float2 *dst = pp.last ? (float2 *)out : p->scratch;
-    const float scale = pp.last ? scale_last : 1.0f;
+    const float2 *src = (pi == 0) ? (const float2 *)in : p->scratch[pi - 1];
+    float2 *dst = pp.last ? (float2 *)out : p->scratch[pi];
     if (events && cudaEventRecord((cudaEvent_t)events[pi], st) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
-    if (pp.kind == kGroupPass) {
-      GArgs g;
-      memset(&g, 0, sizeof(g));
-      g.p[0] = group_pass(p, pi, di, src, dst, -1, -1, inverse);
-      if (pass_role(p, pi) == kFirst && !first_pass_maps(p, di, src, &g))
-        return TCU_DFT_ERR_CUDA;
-      g.bimg = p->bimg[di];
-      g.err = p->err;
-      if (pass_dispatch(p->r, p->precision, pp.s, other_stages(p, pi), pass_role(p, pi), g,
-                        p->num_sms, st) != cudaSuccess)
-        return TCU_DFT_ERR_CUDA;
-      continue;
+    GArgs g;
+    memset(&g, 0, sizeof(g));
+    g.p[0] = group_pass(p, pi, di, src, dst, -1, -1, inverse);
+    if (pp.role == kFirst) {
+      if (!input_map(&g.tm_in, src, p, pp)) return TCU_DFT_ERR_CUDA;
+      g.tm_tw = pp.tw_map[di];
     }
-    PassArgs a;
-    memset(&a, 0, sizeof(a));
-    a.in = src;
-    a.out = dst;
-    a.bimg = p->bimg[di];
-    a.twL = pp.twL[di];
-    a.twA = p->twA[di];
-    a.twB = p->twB[di];
-    a.err = p->err;
-    a.U = pp.U;
-    a.Uper = pp.Uper;
-    a.n = p->n;
-    a.in_vstride = pp.in_vstride;
-    a.in_stride = pp.in_stride;
-    a.out_vstride = pp.out_vstride;
-    a.out_stride = pp.out_stride;
-    a.s = pp.s;
-    a.log2L = pp.log2L;
-    a.log2G = pp.log2G;
-    a.tw_log2N = pp.tw_log2N;
-    a.tw_h = pp.tw_h;
-    a.scale = scale;
-    const long long grid = (pp.U + (1ll << pp.log2G) - 1) >> pp.log2G;
-    if (tile_dispatch(p->r, p->precision, a, grid, st) != cudaSuccess)
+    g.bimg = p->bimg[di];
+    g.err = p->err;
+    if (pass_dispatch(p->r, p->precision, pp, g, p->num_sms, st) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
   }
   if (events && cudaEventRecord((cudaEvent_t)events[p->npasses], st) != cudaSuccess)
@@ -827,14 +769,11 @@ int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t preci
     ++k;
   }
   if (m != n) return TCU_DFT_ERR_UNSUPPORTED;
-  const int sg = max_group_stages(r);
-  if (k > 2 * sg || n > kNaMaxN) return TCU_DFT_ERR_TOO_LARGE;
-  const int npasses = k <= sg ? 1 : 2;
+  int st[kMaxPasses] = {0, 0, 0};
+  const int npasses = plan_stages(r, k, st);
+  if (npasses == 0 || npasses > 2 || n > kNaMaxN) return TCU_DFT_ERR_TOO_LARGE;
   if (npasses == 2 && batch * n > kNaMaxPoints) return TCU_DFT_ERR_TOO_LARGE;
-  int stages[2] = {k, 0};
-  if (npasses == 2) split_two_passes(k, stages);
-  const int log2n = ilog2(n);
-  cudaStream_t st = (cudaStream_t)stream;
+  cudaStream_t stream_ = (cudaStream_t)stream;
 
   std::lock_guard<std::mutex> lock(g_na_mutex);
   int dev = 0;
@@ -874,87 +813,56 @@ int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t preci
   p.num_sms = D.num_sms;
   p.device = dev;
   p.fused = false;
-  p.scratch = D.scratch;
+  p.scratch[0] = D.scratch;
   p.err = D.err;
-  for (int d = 0; d < 2; ++d) {
-    p.bimg[d] = D.img + (size_t)d * kNaImgFloats;
-    p.tw_out[d] = D.tw_out + (size_t)d * kNaMaxN;
-  }
-  for (int pi = 0; pi < npasses; ++pi) {
-    PassPlan &pp = p.pass[pi];
-    pp.kind = kGroupPass;
-    pp.s = stages[pi];
-    pp.log2L = log2r * pp.s;
-    pp.last = (pi == npasses - 1);
-    const long long L = 1ll << pp.log2L;
-    if (npasses == 1) {
-      pp.U = batch;
-      pp.Uper = 1;
-      pp.in_vstride = n;
-      pp.in_stride = 1;
-      pp.out_vstride = n;
-      pp.out_stride = 1;
-    } else if (pi == 0) {
-      pp.U = batch * (n / L);
-      pp.Uper = n / L;
-      pp.in_vstride = 1;
-      pp.in_stride = n / L;
-      pp.out_vstride = 1;
-      pp.out_stride = n / L;
-    } else {
-      pp.U = batch * (n / L);
-      pp.Uper = n / L;
-      pp.in_vstride = L;
-      pp.in_stride = 1;
-      pp.out_vstride = 1;
-      pp.out_stride = n / L;
-    }
-    pp.log2Uper = ilog2(pp.Uper);
-    pp.modes[0] = pp.in_stride == 1 ? kQF : kUF;
-    pp.modes[1] = kUF;
-    pp.modes[2] = pp.out_stride == 1 ? kRQF : kUF;
-    pp.swz_tab = choose_swizzle(r, pp.s, pp.modes);
+  for (int pi = 0; pi < npasses; ++pi) pass_geometry(p.pass[pi], pi, npasses, st, k, r, n, batch);
+  for (int d = 0; d < 2; ++d) p.bimg[d] = D.img + (size_t)d * kNaImgFloats;
+  for (int pi = 0; pi < npasses; ++pi)
     for (int d = 0; d < 2; ++d)
-      pp.tw_stage[d] = D.tw_stage + ((size_t)d * 2 + pi) * kNaStageTw;
-  }
+      p.pass[pi].tw_stage[d] = D.tw_stage + ((size_t)d * 2 + pi) * kNaStageTw;
 
-  // ---- tables for this (n, r), refilled only when they change
+  // ---- tables for this (n, r), refilled only when they change; table A of
+  // the strided pass at the start of the direction's twiddle array, B after it
+  DirTables t[2];
+  for (int d = 0; d < 2; ++d) {
+    dir_tables(&p, d, t[d]);
+    if (npasses == 2) {
+      p.pass[0].tw_a[d] = D.tw_out + (size_t)d * kNaMaxN;
+      if (!t[d].B[0].empty()) p.pass[0].tw_b[d] = p.pass[0].tw_a[d] + t[d].A[0].size();
+    }
+  }
   if (D.n != n || D.r != r) {
     D.n = 0;
     for (int d = 0; d < 2; ++d) {
-      const int sign = d == 0 ? -1 : 1;
-      std::vector<float> img;
-      build_images(r, sign, log2n, img);
-      if (cudaMemcpyAsync(p.bimg[d], img.data(), img.size() * sizeof(float),
-                          cudaMemcpyHostToDevice, st) != cudaSuccess)
+      if (cudaMemcpyAsync(p.bimg[d], t[d].img.data(), t[d].img.size() * sizeof(float),
+                          cudaMemcpyHostToDevice, stream_) != cudaSuccess)
         return TCU_DFT_ERR_CUDA;
-      for (int pi = 0; pi < npasses; ++pi) {
-        const std::vector<float2> t = stage_twiddles(r, p.pass[pi].s, sign);
-        if (cudaMemcpyAsync(p.pass[pi].tw_stage[d], t.data(), t.size() * sizeof(float2),
-                            cudaMemcpyHostToDevice, st) != cudaSuccess)
+      for (int pi = 0; pi < npasses; ++pi)
+        if (cudaMemcpyAsync(p.pass[pi].tw_stage[d], t[d].stage[pi].data(),
+                            t[d].stage[pi].size() * sizeof(float2), cudaMemcpyHostToDevice,
+                            stream_) != cudaSuccess)
           return TCU_DFT_ERR_CUDA;
-      }
       if (npasses == 2) {
-        const long long n1 = 1ll << p.pass[0].log2L, n2 = n / n1;
-        std::vector<float2> t((size_t)n);
-        for (long long k1 = 0; k1 < n1; ++k1)
-          for (long long b = 0; b < n2; ++b) t[(size_t)(k1 * n2 + b)] = root(b * k1, n, sign);
-        if (cudaMemcpyAsync(p.tw_out[d], t.data(), t.size() * sizeof(float2),
-                            cudaMemcpyHostToDevice, st) != cudaSuccess)
+        if (cudaMemcpyAsync(p.pass[0].tw_a[d], t[d].A[0].data(),
+                            t[d].A[0].size() * sizeof(float2), cudaMemcpyHostToDevice,
+                            stream_) != cudaSuccess)
           return TCU_DFT_ERR_CUDA;
-        const long long gg1 = (128ll * r) >> p.pass[0].log2L;
-        if (!encode_map(&D.tw_map[d], p.tw_out[d], n2, n1, 1, n, (int)gg1,
-                        n1 < 256 ? (int)n1 : 256))
+        if (!t[d].B[0].empty() &&
+            cudaMemcpyAsync(p.pass[0].tw_b[d], t[d].B[0].data(),
+                            t[d].B[0].size() * sizeof(float2), cudaMemcpyHostToDevice,
+                            stream_) != cudaSuccess)
+          return TCU_DFT_ERR_CUDA;
+        if (!twiddle_map(&D.tw_map[d], p.pass[0].tw_a[d], r, p.pass[0]))
           return TCU_DFT_ERR_CUDA;
       }
     }
     D.n = n;
     D.r = r;
   }
-  for (int d = 0; d < 2; ++d) p.tw_map[d] = D.tw_map[d];
+  for (int d = 0; d < 2; ++d) p.pass[0].tw_map[d] = D.tw_map[d];
 
-  // the timeout word must start at zero; then the ordinary two-launch path
-  if (cudaMemsetAsync(D.err, 0, sizeof(int), st) != cudaSuccess) return TCU_DFT_ERR_CUDA;
+  // the timeout word must start at zero; then the ordinary launch path
+  if (cudaMemsetAsync(D.err, 0, sizeof(int), stream_) != cudaSuccess) return TCU_DFT_ERR_CUDA;
   return exec_impl(&p, in, out, dir, stream, nullptr);
 }
 

@@ -74,8 +74,9 @@ def test_strerror_and_null_handling(lib):
     (16, 1, 64, 3, 2),
     (48, 1, 16, 3, 2),       # not a power of the radix
     (128, 1, 16, 3, 2),      # power of two but not of 16
-    (16 ** 7, 1, 16, 3, 2),  # beyond two on-chip passes
-    (32 ** 5, 1, 32, 3, 2),
+    (16 ** 7, 1, 16, 3, 2),  # beyond three passes
+    (32 ** 7, 1, 32, 3, 2),
+    (8 ** 10, 1, 8, 3, 2),
 ])
 def test_plan_rejects_before_cuda(lib, n, batch, r, prec, status):
     h = lib.tcu_dft_plan(n, batch, r, prec)
@@ -105,7 +106,8 @@ def test_python_plan_raises(lib):
     ((256, 1, 16, 3, 0), 1),           # direction
     ((256, 1, 12, 3, -1), 2),          # radix
     ((48, 1, 16, 3, -1), 2),           # not a power of the radix
-    ((16 ** 5, 1, 16, 3, -1), 6),      # more stages than two warpgroup passes
+    ((16 ** 5, 1, 16, 3, -1), 6),      # three passes
+    ((8 ** 5, 1, 8, 3, -1), 6),
     ((32 ** 4, 1, 32, 3, -1), 6),      # n beyond the fixed twiddle table
     ((65536, 65, 16, 3, -1), 6),       # batch*n beyond the fixed intermediate
 ])

@@ -58,7 +58,8 @@ def _rel(a, b):
 
 @pytest.mark.parametrize("n,batch,r,direction", [
     (65536, 16, 16, -1),   # two passes: the intermediate uses the fixed array
-    (32768, 24, 8, 1),     # two passes, radix 8, inverse
+    (4096, 200, 8, 1),     # two passes, radix 8, inverse
+    (32768, 24, 32, 1),    # two passes, radix 32: two-level inter-pass twiddles
 ])
 def test_two_calls_in_a_row_match_the_plan_path(pkg, n, batch, r, direction):
     import torch
