@@ -172,7 +172,61 @@ int tcu_dft_pass_stages(tcu_dft_plan_t p, int i);
 int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t precision,
                          const void *in, void *out, int dir, void *stream);
 
-/* Status of the last tcu_dft_plan call on this thread. */
+/* ---------------------------------------------------------------- 2-D
+ * 2-D DFT and circular 2-D convolution (Sec. 4.6: a 2-D DFT is a 1-D DFT of
+ * every row and of every column; Lemma 1 reduces stencils to batched
+ * convolutions computed through it).  Arrays are row-major n1 x n2
+ * complex64, batch-major (x[(b n1 + i) n2 + j]), 16-byte aligned, caller
+ * owned.  n1 and n2 are powers of sqrt_m of at most one warpgroup pass each
+ * (sqrt_m^2 for 16 and 32, 8^3 for 8) with n1 * n2 >= 128 sqrt_m.  Forward
+ * unscaled; inverse with the conjugate exponent and 1/(n1 n2).
+ * tcu_dft2_plan allocates its tables and one batch-size scratch array and
+ * returns NULL with tcu_dft_last_error() set on error (ERR_INVALID,
+ * ERR_UNSUPPORTED, ERR_CUDA, ERR_OOM).  The exec calls are asynchronous on
+ * `stream`, allocate nothing, allow in == out and reject partial overlap
+ * (ERR_INVALID) before launching. */
+typedef struct tcu_dft2_plan_s *tcu_dft2_plan_t;
+tcu_dft2_plan_t tcu_dft2_plan(int64_t n1, int64_t n2, int64_t batch, int32_t sqrt_m,
+                              int32_t precision);
+int tcu_dft2_exec(tcu_dft2_plan_t p, const void *in, void *out, int dir, void *stream);
+/* out = IDFT2(DFT2(in) * spectrum) for every array of the batch: the
+ * circular convolution of each array with the one n1 x n2 array whose 2-D
+ * DFT is `spectrum` (device, n1*n2 complex64, e.g. from tcu_dft2_exec on a
+ * batch-1 plan).  Four passes: columns, rows times the spectrum, inverse
+ * rows, inverse columns. */
+int tcu_conv2_exec(tcu_dft2_plan_t p, const void *in, const void *spectrum, void *out,
+                   void *stream);
+int tcu_dft2_check(tcu_dft2_plan_t p, void *stream);  /* as tcu_dft_check */
+int tcu_dft2_destroy(tcu_dft2_plan_t p);                /* NULL: no-op, OK */
+
+/* ------------------------------------------------------------- stencils
+ * Linear (n, k)-stencil of Sec. 4.6 on a side x side row-major fp32 grid A
+ * (device, caller owned): A_k[i][j] = sum over |a|, |b| <= k of
+ * W[k+a][k+b] A[i+a][j+b], W the weight matrix of k sweeps of the 3 x 3
+ * update w3x3[(a+1)*3 + (b+1)] (a, b in {-1, 0, 1}); cells outside the grid
+ * are 0 at time 0 and the sweeps act on the free plane.
+ * tcu_stencil_weights: W ((2k+1)^2 fp32, device) as the coefficients of
+ *   P(x,y)^k (Lemma 2): P on an Nw x Nw grid, 2-D DFT, pointwise k-th power,
+ *   inverse 2-D DFT, Nw the smallest power of sqrt_m >= 2k + 1.
+ * tcu_stencil_exec: Lemma 1 -- the (side/k)^2 tiles A'_{r,c} (3k x 3k,
+ *   zero-padded to N x N, N the smallest power of sqrt_m >= 3k) convolved
+ *   with the flipped, padded W as ONE batch, centres written to A_k (device,
+ *   side^2 fp32; A_k == A allowed).
+ * Needs side % k == 0 and N, Nw within one warpgroup pass (k <= 85 for
+ * sqrt_m 16, 170 for 8, 341 for 32); else ERR_UNSUPPORTED.  The plan
+ * allocates (side/k)^2 N^2 complex64 of tiles plus tables; the calls are
+ * asynchronous on `stream` and allocate nothing.  w3x3 is a host array. */
+typedef struct tcu_stencil_plan_s *tcu_stencil_plan_t;
+tcu_stencil_plan_t tcu_stencil_plan(int64_t side, int32_t steps, int32_t sqrt_m,
+                                    int32_t precision);
+int tcu_stencil_weights(tcu_stencil_plan_t p, const float *w3x3, float *W, void *stream);
+int tcu_stencil_exec(tcu_stencil_plan_t p, const float *w3x3, const float *A, float *Ak,
+                     void *stream);
+int tcu_stencil_check(tcu_stencil_plan_t p, void *stream);
+int tcu_stencil_destroy(tcu_stencil_plan_t p);
+
+/* Status of the last plan call (tcu_dft_plan*, tcu_dft2_plan,
+ * tcu_stencil_plan) on this thread. */
 int tcu_dft_last_error(void);
 
 /* Static, human-readable name of a status code. */

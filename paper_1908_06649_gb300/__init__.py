@@ -40,6 +40,9 @@ SYMBOLS = (
     "tcu_dft_exec_host", "tcu_dft_exec_noalloc",
     "tcu_dft_check", "tcu_dft_destroy", "tcu_dft_num_passes",
     "tcu_dft_pass_stages", "tcu_dft_last_error", "tcu_dft_strerror",
+    "tcu_dft2_plan", "tcu_dft2_exec", "tcu_conv2_exec", "tcu_dft2_check",
+    "tcu_dft2_destroy", "tcu_stencil_plan", "tcu_stencil_weights",
+    "tcu_stencil_exec", "tcu_stencil_check", "tcu_stencil_destroy",
 )
 
 _lib = None
@@ -97,6 +100,25 @@ def lib():
     L.tcu_dft_last_error.restype = ctypes.c_int
     L.tcu_dft_strerror.argtypes = [ctypes.c_int]
     L.tcu_dft_strerror.restype = ctypes.c_char_p
+    L.tcu_dft2_plan.argtypes = [i64, i64, i64, i32, i32]
+    L.tcu_dft2_plan.restype = vp
+    L.tcu_dft2_exec.argtypes = [vp, vp, vp, ctypes.c_int, vp]
+    L.tcu_dft2_exec.restype = ctypes.c_int
+    L.tcu_conv2_exec.argtypes = [vp, vp, vp, vp, vp]
+    L.tcu_conv2_exec.restype = ctypes.c_int
+    fp = ctypes.POINTER(ctypes.c_float)
+    L.tcu_stencil_plan.argtypes = [i64, i32, i32, i32]
+    L.tcu_stencil_plan.restype = vp
+    L.tcu_stencil_weights.argtypes = [vp, fp, vp, vp]
+    L.tcu_stencil_weights.restype = ctypes.c_int
+    L.tcu_stencil_exec.argtypes = [vp, fp, vp, vp, vp]
+    L.tcu_stencil_exec.restype = ctypes.c_int
+    for nm in ("tcu_dft2_check", "tcu_stencil_check"):
+        getattr(L, nm).argtypes = [vp, vp]
+        getattr(L, nm).restype = ctypes.c_int
+    for nm in ("tcu_dft2_destroy", "tcu_stencil_destroy"):
+        getattr(L, nm).argtypes = [vp]
+        getattr(L, nm).restype = ctypes.c_int
     _lib = L
     return L
 
@@ -241,6 +263,148 @@ class Plan:
     def destroy(self):
         if getattr(self, "_h", None):
             lib().tcu_dft_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+def _check_cuda(t, dtype, numel, what):
+    import torch
+    if (not isinstance(t, torch.Tensor) or t.dtype != dtype or not t.is_cuda
+            or not t.is_contiguous() or t.numel() != numel):
+        raise ValueError("%s must be a contiguous %s CUDA tensor of %d elements"
+                         % (what, dtype, numel))
+
+
+class Plan2:
+    """2-D DFT / circular 2-D convolution plan (tcu_dft2_*): batch row-major
+    n1 x n2 complex64 arrays (Sec. 4.6)."""
+
+    def __init__(self, n1: int, n2: int, batch: int, sqrt_m: int = 16,
+                 precision: int = X3TF32):
+        L = lib()
+        self._h = L.tcu_dft2_plan(int(n1), int(n2), int(batch), int(sqrt_m),
+                                  int(precision))
+        if not self._h:
+            raise TcuDftError(L.tcu_dft_last_error(), "tcu_dft2_plan")
+        self.n1, self.n2, self.batch = int(n1), int(n2), int(batch)
+
+    def _n(self):
+        return self.n1 * self.n2 * self.batch
+
+    def exec(self, x, out=None, direction: int = FORWARD, stream=None):
+        import torch
+        _check_cuda(x, torch.complex64, self._n(), "x")
+        if out is None:
+            out = torch.empty_like(x)
+        _check_cuda(out, torch.complex64, self._n(), "out")
+        rc = lib().tcu_dft2_exec(self._h, ctypes.c_void_p(x.data_ptr()),
+                                 ctypes.c_void_p(out.data_ptr()), int(direction),
+                                 _stream_handle(stream))
+        if rc != OK:
+            raise TcuDftError(rc, "tcu_dft2_exec")
+        return out
+
+    def forward(self, x, out=None, stream=None):
+        return self.exec(x, out, FORWARD, stream)
+
+    def inverse(self, x, out=None, stream=None):
+        return self.exec(x, out, INVERSE, stream)
+
+    def conv(self, x, spectrum, out=None, stream=None):
+        """IDFT2(DFT2(x) * spectrum) for every array of x."""
+        import torch
+        _check_cuda(x, torch.complex64, self._n(), "x")
+        _check_cuda(spectrum, torch.complex64, self.n1 * self.n2, "spectrum")
+        if out is None:
+            out = torch.empty_like(x)
+        _check_cuda(out, torch.complex64, self._n(), "out")
+        rc = lib().tcu_conv2_exec(self._h, ctypes.c_void_p(x.data_ptr()),
+                                  ctypes.c_void_p(spectrum.data_ptr()),
+                                  ctypes.c_void_p(out.data_ptr()),
+                                  _stream_handle(stream))
+        if rc != OK:
+            raise TcuDftError(rc, "tcu_conv2_exec")
+        return out
+
+    def check(self, stream=None):
+        rc = lib().tcu_dft2_check(self._h, _stream_handle(stream))
+        if rc != OK:
+            raise TcuDftError(rc, "tcu_dft2_check")
+
+    def destroy(self):
+        if getattr(self, "_h", None):
+            lib().tcu_dft2_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.destroy()
+        except Exception:
+            pass
+
+
+class StencilPlan:
+    """Linear (n, k)-stencil on a side x side fp32 grid (tcu_stencil_*):
+    the weight matrix by polynomial powering (Lemma 2) and the stencil by
+    batched tile convolutions (Lemma 1)."""
+
+    def __init__(self, side: int, steps: int, sqrt_m: int = 16,
+                 precision: int = X3TF32):
+        L = lib()
+        self._h = L.tcu_stencil_plan(int(side), int(steps), int(sqrt_m),
+                                     int(precision))
+        if not self._h:
+            raise TcuDftError(L.tcu_dft_last_error(), "tcu_stencil_plan")
+        self.side, self.steps = int(side), int(steps)
+
+    @staticmethod
+    def _w3(w3x3):
+        vals = [float(v) for row in w3x3 for v in row]
+        if len(vals) != 9:
+            raise ValueError("w3x3 must be 3 x 3")
+        return (ctypes.c_float * 9)(*vals)
+
+    def weights(self, w3x3, out=None, stream=None):
+        import torch
+        side = 2 * self.steps + 1
+        if out is None:
+            out = torch.empty(side * side, dtype=torch.float32, device="cuda")
+        _check_cuda(out, torch.float32, side * side, "out")
+        rc = lib().tcu_stencil_weights(self._h, self._w3(w3x3),
+                                       ctypes.c_void_p(out.data_ptr()),
+                                       _stream_handle(stream))
+        if rc != OK:
+            raise TcuDftError(rc, "tcu_stencil_weights")
+        return out.reshape(side, side)
+
+    def apply(self, A, out=None, w3x3=None, stream=None):
+        import torch
+        n = self.side * self.side
+        _check_cuda(A, torch.float32, n, "A")
+        if out is None:
+            out = torch.empty_like(A)
+        _check_cuda(out, torch.float32, n, "out")
+        rc = lib().tcu_stencil_exec(self._h, self._w3(w3x3),
+                                    ctypes.c_void_p(A.data_ptr()),
+                                    ctypes.c_void_p(out.data_ptr()),
+                                    _stream_handle(stream))
+        if rc != OK:
+            raise TcuDftError(rc, "tcu_stencil_exec")
+        return out
+
+    def check(self, stream=None):
+        rc = lib().tcu_stencil_check(self._h, _stream_handle(stream))
+        if rc != OK:
+            raise TcuDftError(rc, "tcu_stencil_check")
+
+    def destroy(self):
+        if getattr(self, "_h", None):
+            lib().tcu_stencil_destroy(self._h)
             self._h = None
 
     def __del__(self):

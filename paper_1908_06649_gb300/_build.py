@@ -11,7 +11,8 @@ import subprocess
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
-UNITS = ["tcu_dft.cu", "kernels_r8.cu", "kernels_r16.cu", "kernels_r32.cu"]
+UNITS = ["tcu_dft.cu", "kernels_r8.cu", "kernels_r16.cu", "kernels_r32.cu",
+         "grid_kernels.cu"]
 HEADERS = ["tcgen05.cuh", "group_kernel.cuh", "launch.h",
            "launch_impl.cuh"]
 HDR = os.path.join(os.path.dirname(HERE), "include", "tcu_dft.h")

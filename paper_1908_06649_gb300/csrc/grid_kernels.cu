@@ -1,0 +1,156 @@
+// grid_kernels.cu -- the element-wise steps of the stencil path of
+// arXiv 1908.06649, Sec. 4.6 (Lemmas 1 and 2) around the 2-D DFTs: placing
+// the 3 x 3 stencil polynomial on a grid, the pointwise power of its
+// spectrum, the flipped weight kernel W', and the gather / extract of the
+// 3k x 3k tiles A'_{r,c}.  All are HBM-bound index maps (no contraction),
+// so they are plain coalesced CUDA kernels: one thread per output element,
+// grids in multiples of the SM count.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "launch.h"
+
+namespace tcu {
+namespace {
+
+constexpr int kBlock = 256;
+
+// Signed offset of grid index i on a periodic axis of length N: i for
+// i <= N/2, i - N above.
+__device__ __forceinline__ long long centred(long long i, long long N) {
+  return i <= N / 2 ? i : i - N;
+}
+
+// P(x, y) = sum w3[a+1][b+1] x^a y^b on an Nw x Nw periodic grid:
+// g[a mod Nw][b mod Nw] = w3[a+1][b+1] for a, b in {-1, 0, 1}, 0 elsewhere.
+__global__ void place_poly_kernel(float2 *g, long long Nw, Stencil3 w) {
+  const long long count = Nw * Nw;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < count;
+       e += (long long)gridDim.x * blockDim.x) {
+    const long long a = centred(e / Nw, Nw), b = centred(e % Nw, Nw);
+    float v = 0.f;
+    if (a >= -1 && a <= 1 && b >= -1 && b <= 1) v = w.w[(a + 1) * 3 + (b + 1)];
+    g[e] = make_float2(v, 0.f);
+  }
+}
+
+// g <- g^k elementwise (complex, by repeated squaring).
+__global__ void cpow_kernel(float2 *g, long long count, int k) {
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < count;
+       e += (long long)gridDim.x * blockDim.x) {
+    float2 base = g[e], acc = make_float2(1.f, 0.f);
+    for (int m = k; m > 0; m >>= 1) {
+      if (m & 1) acc = cmul(acc, base);
+      base = cmul(base, base);
+    }
+    g[e] = acc;
+  }
+}
+
+// W[(k + a)(2k + 1) + (k + b)] = Re g[a mod Nw][b mod Nw], |a|, |b| <= k.
+__global__ void extract_weights_kernel(float *W, const float2 *g, long long Nw, int k) {
+  const long long side = 2 * k + 1, count = side * side;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < count;
+       e += (long long)gridDim.x * blockDim.x) {
+    const long long a = e / side - k, b = e % side - k;
+    const long long ia = (a + Nw) % Nw, ib = (b + Nw) % Nw;
+    W[e] = g[ia * Nw + ib].x;
+  }
+}
+
+// The convolution kernel of Lemma 1 on an N x N periodic grid: w[-a mod N]
+// [-b mod N] = W[k + a][k + b] for |a|, |b| <= k (W flipped and padded with
+// zeros), so that (x (*) w)[i][j] = sum W[k+a][k+b] x[i+a][j+b].  W is read
+// from the Nw x Nw grid of the weight computation.
+__global__ void place_kernel_kernel(float2 *w, long long N, const float2 *g, long long Nw,
+                                    int k) {
+  const long long count = N * N;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < count;
+       e += (long long)gridDim.x * blockDim.x) {
+    const long long a = -centred(e / N, N), b = -centred(e % N, N);
+    float v = 0.f;
+    if (a >= -k && a <= k && b >= -k && b <= k) v = g[((a + Nw) % Nw) * Nw + (b + Nw) % Nw].x;
+    w[e] = make_float2(v, 0.f);
+  }
+}
+
+// Tile (r, c) of the side x side grid A as the N x N complex array whose
+// top-left 3k x 3k block is A'_{r,c} = A[(r-1)k .. (r+2)k)[(c-1)k .. (c+2)k)
+// (zero outside A) and whose other entries are 0.
+__global__ void gather_tiles_kernel(float2 *tiles, const float *A, long long side, int k,
+                                    long long N, long long tpr) {
+  const long long count = tpr * tpr * N * N;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < count;
+       e += (long long)gridDim.x * blockDim.x) {
+    const long long t = e / (N * N), ij = e % (N * N);
+    const long long i = ij / N, j = ij % N;
+    const long long gi = (t / tpr - 1) * k + i, gj = (t % tpr - 1) * k + j;
+    float v = 0.f;
+    if (i < 3 * k && j < 3 * k && gi >= 0 && gi < side && gj >= 0 && gj < side)
+      v = __ldg(A + gi * side + gj);
+    tiles[e] = make_float2(v, 0.f);
+  }
+}
+
+// A_k[rk + i][ck + j] = Re tile_{r,c}[k + i][k + j] for i, j < k.
+__global__ void extract_tiles_kernel(float *Ak, const float2 *tiles, long long side, int k,
+                                     long long N, long long tpr) {
+  const long long count = side * side;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < count;
+       e += (long long)gridDim.x * blockDim.x) {
+    const long long gi = e / side, gj = e % side;
+    const long long t = (gi / k) * tpr + gj / k;
+    Ak[e] = tiles[t * N * N + (k + gi % k) * N + (k + gj % k)].x;
+  }
+}
+
+unsigned grid_for(long long count, int num_sms) {
+  long long blocks = (count + kBlock - 1) / kBlock;
+  const long long cap = (long long)num_sms * 8;  // 8 resident 256-thread blocks per SM
+  if (blocks > cap) blocks = cap;
+  return (unsigned)(blocks < 1 ? 1 : blocks);
+}
+
+}  // namespace
+
+cudaError_t launch_place_poly(float2 *g, long long Nw, const Stencil3 &w, int num_sms,
+                              cudaStream_t st) {
+  place_poly_kernel<<<grid_for(Nw * Nw, num_sms), kBlock, 0, st>>>(g, Nw, w);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_cpow(float2 *g, long long count, int k, int num_sms, cudaStream_t st) {
+  cpow_kernel<<<grid_for(count, num_sms), kBlock, 0, st>>>(g, count, k);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_extract_weights(float *W, const float2 *g, long long Nw, int k,
+                                   int num_sms, cudaStream_t st) {
+  const long long side = 2 * k + 1;
+  extract_weights_kernel<<<grid_for(side * side, num_sms), kBlock, 0, st>>>(W, g, Nw, k);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_place_kernel(float2 *w, long long N, const float2 *g, long long Nw, int k,
+                                int num_sms, cudaStream_t st) {
+  place_kernel_kernel<<<grid_for(N * N, num_sms), kBlock, 0, st>>>(w, N, g, Nw, k);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_gather_tiles(float2 *tiles, const float *A, long long side, int k,
+                                long long N, int num_sms, cudaStream_t st) {
+  const long long tpr = side / k;
+  gather_tiles_kernel<<<grid_for(tpr * tpr * N * N, num_sms), kBlock, 0, st>>>(tiles, A, side,
+                                                                              k, N, tpr);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_extract_tiles(float *Ak, const float2 *tiles, long long side, int k,
+                                 long long N, int num_sms, cudaStream_t st) {
+  const long long tpr = side / k;
+  extract_tiles_kernel<<<grid_for(side * side, num_sms), kBlock, 0, st>>>(Ak, tiles, side, k,
+                                                                         N, tpr);
+  return cudaGetLastError();
+}
+
+}  // namespace tcu

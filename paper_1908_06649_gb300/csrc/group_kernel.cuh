@@ -41,7 +41,7 @@
 namespace tcu {
 
 enum RowMode { kQF = 0, kUF = 1, kRQF = 2 };
-enum Role { kSingle = 0, kFirst = 1, kSecond = 2 };
+enum Role { kSingle = 0, kFirst = 1, kSecond = 2, kCols = 3 };
 
 constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 16 ? 4 : 5); }
 // Warpgroups per CTA: TMEM holds 512 columns, a warpgroup's slot 3 Q of
@@ -58,6 +58,9 @@ constexpr int pass_nwg(int R, int ROLE) { return R == 32 ? 2 : (ROLE == 1 ? 4 : 
 //            b' = (b, p), p < Npre = R^SP, holds z[b' M + a n2 + v]; the
 //            DFT over a, times w_M^{v k}, goes to T[b n + (k Npre + p) n2 + v]
 //            (for SP = 0: T[b n + k n2 + v])
+//   kCols  : the column pass of a 2-D DFT of n1 x n2 arrays (n1 = R^S,
+//            n2 = R^SO): kFirst's geometry with SP = 0 and no twiddle,
+//            x[b n + a n2 + v] -> X[b n + k n2 + v]
 //   kSecond: last of several passes (SO stages before it):
 //            T[b n + v L + a] -> y[b n + v + k n1], n1 = R^SO
 template <int R, int S, int SO, int ROLE, int SP = 0, int NWG_ = pass_nwg(R, ROLE)>
@@ -80,7 +83,8 @@ struct Geo {
   static constexpr long long OUT_STRIDE =
       ROLE == kSingle ? 1 : (1ll << (LOG2O + LOG2PRE));
   static constexpr long long OUT_VSTRIDE = ROLE == kSingle ? 0 : 1;
-  static constexpr int MODE_FIRST = ROLE == kFirst ? kUF : kQF;
+  static constexpr bool STRIDED = ROLE == kFirst || ROLE == kCols;
+  static constexpr int MODE_FIRST = STRIDED ? kUF : kQF;
   static constexpr int MODE_MID = kUF;
   static constexpr int MODE_LAST = ROLE == kSingle ? kRQF : kUF;
   static constexpr bool TW_OUT = ROLE == kFirst;
@@ -99,6 +103,7 @@ struct Geo {
   static constexpr int TW_ENTRIES = S == 1 ? 0 : (S == 2 ? R * R : R * R * R + R * R);
   static_assert(LOG2GG >= 0, "sub-transform longer than one item");
   static_assert(LOG2GG <= LOG2VL || !TW_OUT, "an item spans one twiddle column block");
+  static_assert(LOG2GG <= LOG2UPER || !STRIDED, "an item spans columns of one sequence");
   static_assert(NWG * GCOLS <= 512, "TMEM budget");
 };
 
@@ -113,6 +118,11 @@ struct PRun {
   const float2 *tw_stage;         // stage twiddles [t][j][lo]
   unsigned long long swz_tab;     // SMEM swizzle nibble per (ul & 15)
   int last_img;                   // byte offset of the last stage's F images
+  // kSingle: if set, output k of sub-transform u is multiplied by
+  // spec[(u & spec_mask) L + k] (a 2-D spectrum whose rows are the
+  // sub-transforms: the pointwise product of a circular convolution)
+  const float2 *spec;
+  long long spec_mask;
 };
 
 struct GArgs {
@@ -451,9 +461,12 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, 
   const float2 *twbs = w.twb + klow;
   const float2 *twbg = P.tw_b + (vh << G::LOG2L) + klow;
   constexpr int TBJ = 1 << (G::LOG2L - G::LOG2R);
+  const float2 *sp = P.spec + ((u & P.spec_mask) << G::LOG2L) + klow;
+  const bool mul = G::MODE_LAST == kRQF && P.spec != nullptr;
 #pragma unroll
   for (int j = 0; j < R; ++j) {
     float2 y = make_float2(d[2 * j], d[2 * j + 1]);
+    if (G::MODE_LAST == kRQF && mul) y = cmul(y, __ldg(sp + j * JS));
     if (G::TW_SMEM) {
       y = G::TW2L ? cmul(y, cmul(tws[j * TJS], twbs[j * TBJ])) : cmul(y, tws[j * TJS]);
     } else if (G::TW_OUT) {

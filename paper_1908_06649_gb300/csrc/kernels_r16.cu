@@ -19,6 +19,9 @@ cudaError_t launch_pass_r16(int prec, int s, int so, int role, int sp, const GAr
   TCU_PASS_CASE(2, 4, kFirst, 0)   // n = 16^6: 2 + 2 + 2
   TCU_PASS_CASE(2, 2, kFirst, 2)
   TCU_PASS_CASE(2, 4, kSecond, 0)
+  TCU_PASS_CASE(1, 2, kCols, 0)   // 2-D DFT column passes: n1 = R^s, n2 = R^so
+  TCU_PASS_CASE(2, 1, kCols, 0)
+  TCU_PASS_CASE(2, 2, kCols, 0)
   return cudaErrorInvalidValue;
 }
 

@@ -27,6 +27,12 @@ cudaError_t launch_pass_r8(int prec, int s, int so, int role, int sp, const GArg
   TCU_PASS_CASE(3, 6, kFirst, 0)   // n = 8^9: 3 + 3 + 3
   TCU_PASS_CASE(3, 3, kFirst, 3)
   TCU_PASS_CASE(3, 6, kSecond, 0)
+  TCU_PASS_CASE(1, 3, kCols, 0)   // 2-D DFT column passes: n1 = R^s, n2 = R^so
+  TCU_PASS_CASE(2, 2, kCols, 0)
+  TCU_PASS_CASE(2, 3, kCols, 0)
+  TCU_PASS_CASE(3, 1, kCols, 0)
+  TCU_PASS_CASE(3, 2, kCols, 0)
+  TCU_PASS_CASE(3, 3, kCols, 0)
   return cudaErrorInvalidValue;
 }
 

@@ -25,4 +25,20 @@ cudaError_t launch_fused_r16(int prec, int s1, int s2, const GArgs &a, int num_s
 cudaError_t launch_fused_r32(int prec, int s1, int s2, const GArgs &a, int num_sms,
                              cudaStream_t st);
 
+// Element-wise steps of the stencil path (grid_kernels.cu).
+struct Stencil3 {
+  float w[9];  // w[(a + 1) * 3 + (b + 1)], a, b in {-1, 0, 1}
+};
+cudaError_t launch_place_poly(float2 *g, long long Nw, const Stencil3 &w, int num_sms,
+                              cudaStream_t st);
+cudaError_t launch_cpow(float2 *g, long long count, int k, int num_sms, cudaStream_t st);
+cudaError_t launch_extract_weights(float *W, const float2 *g, long long Nw, int k,
+                                   int num_sms, cudaStream_t st);
+cudaError_t launch_place_kernel(float2 *w, long long N, const float2 *g, long long Nw, int k,
+                                int num_sms, cudaStream_t st);
+cudaError_t launch_gather_tiles(float2 *tiles, const float *A, long long side, int k,
+                                long long N, int num_sms, cudaStream_t st);
+cudaError_t launch_extract_tiles(float *Ak, const float2 *tiles, long long side, int k,
+                                 long long N, int num_sms, cudaStream_t st);
+
 }  // namespace tcu

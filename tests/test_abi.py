@@ -16,7 +16,7 @@ HEADER = os.path.join(ROOT, "include", "tcu_dft.h")
 def declared_functions():
     src = open(HEADER).read()
     src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
-    return sorted(set(re.findall(r"\b(tcu_dft_[a-z_]+)\s*\(", src)))
+    return sorted(set(re.findall(r"\b(tcu_[a-z0-9_]+)\s*\(", src)))
 
 
 @pytest.fixture(scope="module")
@@ -121,3 +121,39 @@ def test_noalloc_rejects_before_cuda(lib, args, status):
 def test_noalloc_null_buffers(lib):
     assert lib.tcu_dft_exec_noalloc(256, 1, 16, 3, None, None, -1, None) == 1
     assert b"fixed memory" in lib.tcu_dft_strerror(6)
+
+
+@pytest.mark.parametrize("args,status", [
+    ((0, 256, 1, 16, 3), 1),        # n1 < 1
+    ((16, 256, 0, 16, 3), 1),       # batch < 1
+    ((16, 256, 1, 16, 2), 1),       # precision
+    ((16, 16, 1, 16, 3), 2),        # n1 n2 below one column item (128 r)
+    ((4096, 16, 1, 16, 3), 2),      # an axis beyond one warpgroup pass
+    ((48, 256, 1, 16, 3), 2),       # not a power of the radix
+    ((16, 256, 1, 12, 3), 2),       # radix
+])
+def test_dft2_plan_rejects_before_cuda(lib, args, status):
+    assert not lib.tcu_dft2_plan(*args)
+    assert lib.tcu_dft_last_error() == status
+
+
+@pytest.mark.parametrize("args,status", [
+    ((0, 4, 8, 3), 1),              # side
+    ((64, 0, 8, 3), 1),             # steps
+    ((66, 4, 8, 3), 2),             # side not a multiple of the steps
+    ((1024, 200, 8, 3), 2),         # 3k beyond one pass (8^3)
+    ((64, 4, 12, 3), 2),            # radix
+])
+def test_stencil_plan_rejects_before_cuda(lib, args, status):
+    assert not lib.tcu_stencil_plan(*args)
+    assert lib.tcu_dft_last_error() == status
+
+
+def test_grid_null_handling(lib):
+    import paper_1908_06649_gb300 as pkg
+    assert lib.tcu_dft2_destroy(None) == pkg.OK
+    assert lib.tcu_stencil_destroy(None) == pkg.OK
+    assert lib.tcu_dft2_exec(None, None, None, -1, None) == pkg.ERR_INVALID
+    assert lib.tcu_conv2_exec(None, None, None, None, None) == pkg.ERR_INVALID
+    assert lib.tcu_stencil_exec(None, None, None, None, None) == pkg.ERR_INVALID
+    assert lib.tcu_dft2_check(None, None) == pkg.ERR_INVALID
