@@ -249,6 +249,183 @@ def run_reference(args, wl):
     return 0
 
 
+GRID = {
+    # 2-D DFT / circular convolution of tiles the size the stencil path
+    # uses, and the stencil itself (Sec. 4.6, Lemmas 1-2)
+    "dft2": {"n1": 256, "n2": 256, "batch": 4096, "sqrt_m": 16, "seed": 5},
+    "conv2": {"n1": 256, "n2": 256, "batch": 4096, "sqrt_m": 16, "seed": 6},
+    "stencil": {"side": 4096, "steps": 16, "sqrt_m": 8, "seed": 7},
+}
+HEAT3 = [[0.0, 0.1, 0.0], [0.15, 0.5, 0.15], [0.0, 0.1, 0.0]]
+
+
+def grid_cpu_baseline(args, g):
+    """The fp64 oracle on a bounded sample of the 2-D workload (one core)."""
+    from oracle import grid as ogrid
+    t0 = time.perf_counter()
+    if args.grid in ("dft2", "conv2"):
+        n1, n2 = g["n1"], g["n2"]
+        N = n1 * n2
+        x = inputs.make("normal", N, 8, g["seed"]).reshape(8, n1, n2)
+        done = 0
+        while time.perf_counter() - t0 < args.cpu_seconds:
+            y = ogrid.dft2(x)
+            if args.grid == "conv2":
+                ogrid.dft2(y, inverse=True)
+            done += 8
+        el = time.perf_counter() - t0
+        per = 5.0 * N * math.log2(N) * (2 if args.grid == "conv2" else 1)
+        return {"value": per * done / el / 1e9, "unit": "GFLOP/s", "cores": 1,
+                "kind": "oracle",
+                "sample": "%d arrays of %dx%d through the fp64 oracle 2-D DFT "
+                          "(rows then columns)%s, %.1f s" % (
+                              done, n1, n2, " and its inverse" if args.grid == "conv2"
+                              else "", el)}
+    k = g["steps"]
+    side = 256
+    rng = np.random.default_rng(g["seed"])
+    A = rng.standard_normal((side, side))
+    done = 0
+    while time.perf_counter() - t0 < args.cpu_seconds:
+        ogrid.stencil_direct(A, np.array(HEAT3), k)
+        done += 1
+    el = time.perf_counter() - t0
+    return {"value": side * side * k * done / el / 1e9, "unit": "Gupdates/s", "cores": 1,
+            "kind": "oracle",
+            "sample": "%d runs of the fp64 oracle stencil (direct sweeps, free "
+                      "plane) on a %dx%d grid for %d steps, %.1f s" % (done, side, side, k, el)}
+
+
+def run_grid(args):
+    """One JSON line for a 2-D workload: 2-D DFT or batched circular 2-D
+    convolution of 256 x 256 arrays (GFLOP/s, 5 N log2 N per array and
+    transform, N = n1 n2), or the stencil of a 4096^2 grid over 16 steps
+    (grid-point updates per second).  Every pass kernel moves 16 B per
+    point; the roofline line is the average pass launch of the step."""
+    import torch
+    from paper_1908_06649_gb300 import _build
+    _build.build()
+    import paper_1908_06649_gb300 as pkg
+    g = GRID[args.grid]
+    peaks, peak_kind = load_peaks()
+    hbm = float(peaks["hbm_gbs"])
+    stream = torch.cuda.current_stream()
+    if args.grid in ("dft2", "conv2"):
+        n1, n2, batch, r = g["n1"], g["n2"], g["batch"], g["sqrt_m"]
+        N = n1 * n2
+        x_host = inputs.make("normal", N, batch, g["seed"])
+        x = torch.from_numpy(x_host).cuda()
+        y = torch.empty_like(x)
+        plan = pkg.Plan2(n1, n2, batch, r, args.precision)
+        if args.grid == "conv2":
+            one = pkg.Plan2(n1, n2, 1, r, args.precision)
+            w = torch.from_numpy(inputs.make("normal", N, 1, g["seed"] + 1)).cuda()
+            spec = one.forward(w)
+            one.check()
+            step = lambda: plan.conv(x, spec, y)
+            passes, flops = 4, 2 * 5.0 * N * math.log2(N) * batch
+        else:
+            step = lambda: plan.forward(x, y)
+            passes, flops = 2, 5.0 * N * math.log2(N) * batch
+        launches = passes
+        points = N * batch
+        unit, metric = "GFLOP/s", ("%s GFLOP/s (5N·log2N per array%s), %dx%d x%d "
+                                   "complex64, 1xGB300" % (
+                                       "2-D DFT" if args.grid == "dft2" else
+                                       "circular 2-D convolution",
+                                       "" if args.grid == "dft2" else " x2 transforms",
+                                       n1, n2, batch))
+        config = {"workload": "batched complex64 %s of %dx%d arrays x batch %d, "
+                              "normal inputs seed %d, %s" % (
+                                  "2-D DFT" if args.grid == "dft2" else
+                                  "circular 2-D convolution with one array",
+                                  n1, n2, batch, g["seed"],
+                                  "3xTF32" if args.precision == 3 else "TF32"),
+                  "n1": n1, "n2": n2, "batch": batch, "sqrt_m": r,
+                  "l2": "inputs larger than L2, no flush"}
+        value_of = lambda ms: flops / (ms * 1e-3) / 1e9
+        bytes_min = 16.0 * points
+    else:
+        side, k, r = g["side"], g["steps"], g["sqrt_m"]
+        rng = np.random.default_rng(g["seed"])
+        A = torch.from_numpy(rng.standard_normal((side, side)).astype(np.float32)).cuda().reshape(-1)
+        out = torch.empty_like(A)
+        plan = pkg.StencilPlan(side, k, r, args.precision)
+        step = lambda: plan.apply(A, out, w3x3=HEAT3)
+        Nt = 1
+        while Nt < 3 * k or Nt * Nt < 128 * r:
+            Nt *= r
+        tiles = (side // k) ** 2
+        points = tiles * Nt * Nt
+        passes = 4
+        # weights: place, 2-D DFT (2), power, inverse (2); kernel W': place,
+        # 2-D DFT (2); tiles: gather, convolution (4), extract
+        launches = 15
+        unit = "Gupdates/s"
+        metric = ("linear stencil grid-point updates/s (side^2 x steps), "
+                  "%d^2 grid x %d steps, 1xGB300" % (side, k))
+        config = {"workload": "linear 3x3 stencil (heat update) on a %dx%d fp32 "
+                              "grid for %d steps via Lemma 1 tiles (%d tiles of "
+                              "%dx%d) and Lemma 2 weights, %s" % (
+                                  side, side, k, tiles, Nt, Nt,
+                                  "3xTF32" if args.precision == 3 else "TF32"),
+                  "side": side, "steps": k, "sqrt_m": r, "tile": Nt,
+                  "l2": "inputs larger than L2, no flush"}
+        value_of = lambda ms: side * side * k / (ms * 1e-3) / 1e9
+        bytes_min = 8.0 * side * side
+    for _ in range(max(3, args.warmup)):
+        step()
+    plan.check()
+    K = args.steps
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    clocks = ClockSampler(torch.cuda.current_device())
+    clocks.start()
+    time.sleep(0.2)
+    torch.cuda.synchronize()
+    t0.record(stream)
+    for _ in range(K):
+        step()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    plan.check()
+    ms = t0.elapsed_time(t1) / K
+    cpu = None if args.no_cpu_baseline else grid_cpu_baseline(args, g)
+    if args.grid == "stencil":
+        # whole step: the four convolution passes (16 B per tile point each),
+        # the gather (tile points written, the grid read once) and the
+        # extract (one tile point read and one grid point written per cell);
+        # the weight and kernel-spectrum transforms are tiny
+        S = float(side * side)
+        step_bytes = 64.0 * points + 8.0 * points + 4.0 * S + 8.0 * S + 4.0 * S
+        achieved = step_bytes / (ms * 1e-3) / 1e9
+        kname = ("whole step (%d launches: weights, kernel spectrum, gather, 4 "
+                 "convolution passes, extract), %.2f GB algorithmic" % (launches, step_bytes / 1e9))
+    else:
+        achieved = 16.0 * points / (ms / passes * 1e-3) / 1e9
+        kname = "average pass launch (%d pass launches per step)" % passes
+    line = {
+        "metric": metric, "value": value_of(ms), "unit": unit, "n_gpus": 1,
+        "steps": K, "warmup": max(3, args.warmup), "ms_per_step": ms,
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+        "dtype": "tf32x3" if args.precision == 3 else "tf32", "data": "synthetic",
+        "config": config,
+        "roofline": {"bound": "hbm", "achieved": achieved, "peak": hbm, "unit": "GB/s",
+                     "frac": achieved / hbm, "traffic": None,
+                     "kernel": kname, "peak_source": peak_kind},
+        "roofline_step": {"hbm_bytes_min": bytes_min,
+                          "t_roof_ms": bytes_min / (hbm * 1e9) * 1e3,
+                          "frac": bytes_min / (hbm * 1e9) / (ms * 1e-3)},
+        "cpu_baseline": cpu, "e2e": None,
+        "gpu_launches": K * launches, "clocks": clk,
+    }
+    print(json.dumps(line), flush=True)
+    plan.destroy()
+    return 0
+
+
 def workload_config(wl, args):
     return {"workload": "batched complex64 forward DFT n=%d (=%d^%d) x batch "
                         "%d, %s inputs seed %d, %s" % (
@@ -281,6 +458,9 @@ def main():
                          "instead of two pass launches")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (profiling cases)")
+    ap.add_argument("--grid", default=None, choices=sorted(GRID),
+                    help="measure a 2-D workload (2-D DFT, circular 2-D "
+                         "convolution or the stencil) instead of the 1-D one")
     args = ap.parse_args()
     if args.warmup < 3:
         args.warmup = 3
@@ -289,6 +469,8 @@ def main():
         wl["batch"] = args.batch
     if args.impl == "reference":
         return run_reference(args, wl)
+    if args.grid:
+        return run_grid(args)
 
     import torch
     world, rank, local = dist_setup()
