@@ -154,3 +154,62 @@ cudaError_t launch_extract_tiles(float *Ak, const float2 *tiles, long long side,
 }
 
 }  // namespace tcu
+
+// ---------------------------------------------------------- mixed radix
+// The q-point pass of a mixed-radix transform n = q R^k (q < R, a power of
+// two): the four-step split n = q x n2 with the q-point DFTs over the
+// stride-n2 columns done on the CUDA cores -- for q <= 16 a tensor-core
+// product would be mostly padding -- straight from the definition
+// y_k = sum_a x_a w_q^{a k}, then the inter-pass twiddle w_n^{k v} from the
+// two-level tables A[k][vl], B[vh][k] (v = vh 256 + vl).  One thread per
+// column (b, v), v fastest: every load and store is coalesced.
+namespace tcu {
+namespace {
+
+template <int Q>
+__global__ void radix_q_kernel(const float2 *x, float2 *out, long long batch, int log2n2,
+                               const float2 *twA, const float2 *twB, RootsQ roots) {
+  const long long n2 = 1ll << log2n2, n = Q * n2, count = batch * n2;
+  const int log2vl = log2n2 > 8 ? 8 : log2n2;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < count;
+       e += (long long)gridDim.x * blockDim.x) {
+    const long long b = e >> log2n2, v = e & (n2 - 1);
+    const float2 *src = x + b * n + v;
+    float2 a[Q];
+#pragma unroll
+    for (int i = 0; i < Q; ++i) a[i] = __ldcs(src + i * n2);
+    const long long vl = v & ((1ll << log2vl) - 1), vh = v >> log2vl;
+    float2 *dst = out + b * n + v;
+#pragma unroll
+    for (int k = 0; k < Q; ++k) {
+      float2 y = a[0];
+#pragma unroll
+      for (int i = 1; i < Q; ++i) {
+        const float2 w = roots.w[(i * k) % Q];
+        y.x = fmaf(a[i].x, w.x, fmaf(-a[i].y, w.y, y.x));
+        y.y = fmaf(a[i].x, w.y, fmaf(a[i].y, w.x, y.y));
+      }
+      float2 tw = __ldg(twA + ((long long)k << log2vl) + vl);
+      if (log2n2 > 8) tw = cmul(tw, __ldg(twB + vh * Q + k));
+      __stcs(dst + k * n2, cmul(y, tw));
+    }
+  }
+}
+
+}  // namespace
+
+cudaError_t launch_radix_q(int q, const float2 *x, float2 *out, long long batch, int log2n2,
+                           const float2 *twA, const float2 *twB, const RootsQ &roots,
+                           int num_sms, cudaStream_t st) {
+  const unsigned grid = grid_for(batch << log2n2, num_sms);
+  switch (q) {
+    case 2: radix_q_kernel<2><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 4: radix_q_kernel<4><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 8: radix_q_kernel<8><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 16: radix_q_kernel<16><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    default: return cudaErrorInvalidValue;
+  }
+  return cudaGetLastError();
+}
+
+}  // namespace tcu

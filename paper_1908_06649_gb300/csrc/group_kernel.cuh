@@ -43,27 +43,28 @@ namespace tcu {
 enum RowMode { kQF = 0, kUF = 1, kRQF = 2 };
 enum Role { kSingle = 0, kFirst = 1, kSecond = 2, kCols = 3 };
 
-constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 16 ? 4 : 5); }
+__host__ __device__ constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 16 ? 4 : 5); }
 // Warpgroups per CTA: TMEM holds 512 columns, a warpgroup's slot 3 Q of
 // them; a first (strided) pass also stages its inter-pass twiddles in SMEM,
 // which leaves room for four.
 constexpr int pass_nwg(int R, int ROLE) { return R == 32 ? 2 : (ROLE == 1 ? 4 : 5); }
 
 // Compile-time geometry of one pass: S stages of radix R.  A transform of
-// length n = R^K is computed in up to three passes (the four-step split
-// applied recursively); a pass splits sequences of length M = R^(S+SO) into
-// L = R^S rows by n2 = R^SO columns.
+// length n is computed in up to three passes (the four-step split applied
+// recursively); a pass splits sequences of length M = R^S * 2^LO into
+// L = R^S rows by n2 = 2^LO columns.  (With n = R^k every size is a power
+// of R; a mixed-radix transform n = q R^k has one more factor q = 2^LP.)
 //   kSingle: x[b n + a]                        -> y[b n + k]
-//   kFirst : strided pass; SP stages come before it, SO after.  Sequence
-//            b' = (b, p), p < Npre = R^SP, holds z[b' M + a n2 + v]; the
-//            DFT over a, times w_M^{v k}, goes to T[b n + (k Npre + p) n2 + v]
-//            (for SP = 0: T[b n + k n2 + v])
+//   kFirst : strided pass after a prefix of P = 2^LP sequences per
+//            transform.  Sequence b' = (b, p), p < P, holds z[b' M + a n2 + v];
+//            the DFT over a, times w_M^{v k}, goes to T[b n + (k P + p) n2 + v]
+//            (for LP = 0: T[b n + k n2 + v])
 //   kCols  : the column pass of a 2-D DFT of n1 x n2 arrays (n1 = R^S,
-//            n2 = R^SO): kFirst's geometry with SP = 0 and no twiddle,
+//            n2 = 2^LO): kFirst's geometry with LP = 0 and no twiddle,
 //            x[b n + a n2 + v] -> X[b n + k n2 + v]
-//   kSecond: last of several passes (SO stages before it):
-//            T[b n + v L + a] -> y[b n + v + k n1], n1 = R^SO
-template <int R, int S, int SO, int ROLE, int SP = 0, int NWG_ = pass_nwg(R, ROLE)>
+//   kSecond: last of several passes, n1 = 2^LO points before it per row:
+//            T[b n + v L + a] -> y[b n + v + k n1]
+template <int R, int S, int LO, int ROLE, int LP = 0, int NWG_ = pass_nwg(R, ROLE)>
 struct Geo {
   static constexpr int LOG2R = log2_radix(R);
   static constexpr int NWG = NWG_;
@@ -72,13 +73,13 @@ struct Geo {
   static constexpr int GPTS = 1 << LOG2GPTS;
   static constexpr int LOG2L = LOG2R * S;
   static constexpr int L = 1 << LOG2L;
-  static constexpr int LOG2N = LOG2R * (S + SO);        // sequence length M
-  static constexpr int LOG2PRE = ROLE == kFirst ? LOG2R * SP : 0;
+  static constexpr int LOG2N = LOG2R * S + LO;          // sequence length M
+  static constexpr int LOG2PRE = ROLE == kFirst ? LP : 0;
   static constexpr int LOG2NT = LOG2N + LOG2PRE;        // transform length n
   static constexpr int LOG2RPS = LOG2L - LOG2R;   // rows per sub-transform
   static constexpr int LOG2GG = LOG2GPTS - LOG2L; // sub-transforms per item
   static constexpr int GG = 1 << LOG2GG;
-  static constexpr int LOG2O = LOG2R * SO;
+  static constexpr int LOG2O = LO;
   static constexpr int LOG2UPER = ROLE == kSingle ? 0 : LOG2O;
   static constexpr long long OUT_STRIDE =
       ROLE == kSingle ? 1 : (1ll << (LOG2O + LOG2PRE));
@@ -445,7 +446,7 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, 
   }
   const long long b = u >> G::LOG2UPER;
   const long long v = u & ((1ll << G::LOG2UPER) - 1);
-  // kFirst after SP stages: sequence b = (transform, p) -> transform-major,
+  // kFirst after a prefix: sequence b = (transform, p) -> transform-major,
   // k above p
   const long long bt = b >> G::LOG2PRE, bp = b & ((1ll << G::LOG2PRE) - 1);
   float2 *dst = P.out + ((bt & P.out_bmask) << G::LOG2NT) + (bp << G::LOG2UPER) +
@@ -625,10 +626,10 @@ struct StaticNext {
   __device__ void publish() {}
 };
 
-template <int R, int PREC, int S, int SO, int ROLE, int SP>
-__global__ void __launch_bounds__(Geo<R, S, SO, ROLE, SP>::THREADS, 1)
+template <int R, int PREC, int S, int LO, int ROLE, int LP>
+__global__ void __launch_bounds__(Geo<R, S, LO, ROLE, LP>::THREADS, 1)
     dft_pass_kernel(const __grid_constant__ GArgs a) {
-  using G = Geo<R, S, SO, ROLE, SP>;
+  using G = Geo<R, S, LO, ROLE, LP>;
   using SM = SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM, G::TWB>;
   extern __shared__ __align__(1024) unsigned char smem[];
   float2 *tw = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
@@ -839,11 +840,11 @@ struct FusedNext {
 };
 
 template <int R, int PREC, int S1, int S2>
-__global__ void __launch_bounds__(Geo<R, S1, S2, kFirst>::THREADS, 1)
+__global__ void __launch_bounds__(Geo<R, S1, log2_radix(R) * S2, kFirst>::THREADS, 1)
     dft_fused_kernel(const __grid_constant__ GArgs a) {
   static_assert(S1 >= 2 && S2 >= 2, "the fused schedule needs an SMEM barrier per item");
-  using G1 = Geo<R, S1, S2, kFirst>;
-  using G2 = Geo<R, S2, S1, kSecond, 0, G1::NWG>;
+  using G1 = Geo<R, S1, log2_radix(R) * S2, kFirst>;
+  using G2 = Geo<R, S2, log2_radix(R) * S1, kSecond, 0, G1::NWG>;
   using SM = SmemLayout<R, G1::NWG, G1::TW_ENTRIES, G2::TW_ENTRIES, G1::TW_SMEM, G1::TWB>;
   constexpr int NWG = G1::NWG;
   extern __shared__ __align__(1024) unsigned char smem[];

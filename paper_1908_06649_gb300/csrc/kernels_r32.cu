@@ -4,7 +4,7 @@
 namespace tcu {
 
 // (stages, stages after (kFirst) or before (kSecond), role, stages before)
-cudaError_t launch_pass_r32(int prec, int s, int so, int role, int sp, const GArgs &a,
+cudaError_t launch_pass_r32(int prec, int s, int lo, int role, int lp, const GArgs &a,
                             int num_sms, cudaStream_t st) {
   constexpr int R = 32;
   TCU_PASS_CASE(1, 0, kSingle, 0)

@@ -8,14 +8,14 @@
 namespace tcu {
 
 // One warpgroup pass of radix 8, 16 or 32: s stages, role kSingle / kFirst /
-// kSecond; so = stages after a kFirst pass or before a kSecond pass; sp =
-// stages before a kFirst pass.  cudaErrorInvalidValue for a combination that
-// is not instantiated.
-cudaError_t launch_pass_r8(int prec, int s, int so, int role, int sp, const GArgs &a,
+// kSecond / kCols; lo = log2 of the columns of a strided pass or of the
+// points before a last pass; lp = log2 of the prefix count of a strided pass.
+// cudaErrorInvalidValue for a combination that is not instantiated.
+cudaError_t launch_pass_r8(int prec, int s, int lo, int role, int lp, const GArgs &a,
                            int num_sms, cudaStream_t st);
-cudaError_t launch_pass_r16(int prec, int s, int so, int role, int sp, const GArgs &a,
+cudaError_t launch_pass_r16(int prec, int s, int lo, int role, int lp, const GArgs &a,
                             int num_sms, cudaStream_t st);
-cudaError_t launch_pass_r32(int prec, int s, int so, int role, int sp, const GArgs &a,
+cudaError_t launch_pass_r32(int prec, int s, int lo, int role, int lp, const GArgs &a,
                             int num_sms, cudaStream_t st);
 // Both passes of a two-pass transform fused in one launch (s1, s2 >= 2).
 cudaError_t launch_fused_r8(int prec, int s1, int s2, const GArgs &a, int num_sms,
@@ -40,5 +40,21 @@ cudaError_t launch_gather_tiles(float2 *tiles, const float *A, long long side, i
                                 long long N, int num_sms, cudaStream_t st);
 cudaError_t launch_extract_tiles(float *Ak, const float2 *tiles, long long side, int k,
                                  long long N, int num_sms, cudaStream_t st);
+
+// The q-point first pass of a mixed-radix transform (grid_kernels.cu).
+struct RootsQ {
+  float2 w[16];  // w_q^m, m < q, of the direction
+};
+cudaError_t launch_radix_q(int q, const float2 *x, float2 *out, long long batch, int log2n2,
+                           const float2 *twA, const float2 *twB, const RootsQ &roots,
+                           int num_sms, cudaStream_t st);
+// Mixed-radix warpgroup passes (kernels_mixed_r*.cu): same arguments as
+// launch_pass_r*.
+cudaError_t launch_pass_mixed_r8(int prec, int s, int lo, int role, int lp, const GArgs &a,
+                                 int num_sms, cudaStream_t st);
+cudaError_t launch_pass_mixed_r16(int prec, int s, int lo, int role, int lp, const GArgs &a,
+                                  int num_sms, cudaStream_t st);
+cudaError_t launch_pass_mixed_r32(int prec, int s, int lo, int role, int lp, const GArgs &a,
+                                  int num_sms, cudaStream_t st);
 
 }  // namespace tcu

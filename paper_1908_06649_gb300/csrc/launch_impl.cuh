@@ -5,26 +5,27 @@
 
 namespace tcu {
 
-template <int R, int PREC, int S, int SO, int ROLE, int SP>
+template <int R, int PREC, int S, int LO, int ROLE, int LP>
 cudaError_t launch_pass_t(const GArgs &a, int num_sms, cudaStream_t st) {
-  using G = Geo<R, S, SO, ROLE, SP>;
+  using G = Geo<R, S, LO, ROLE, LP>;
   const size_t sm = SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM, G::TWB>::BYTES;
-  cudaError_t e = cudaFuncSetAttribute(dft_pass_kernel<R, PREC, S, SO, ROLE, SP>,
+  cudaError_t e = cudaFuncSetAttribute(dft_pass_kernel<R, PREC, S, LO, ROLE, LP>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)sm);
   if (e != cudaSuccess) return e;
   const long long nitems = (a.p[0].U + G::GG - 1) >> G::LOG2GG;
   long long grid = (nitems + G::NWG - 1) / G::NWG;
   if (grid > num_sms) grid = num_sms;
-  dft_pass_kernel<R, PREC, S, SO, ROLE, SP><<<(unsigned)grid, G::THREADS, sm, st>>>(a);
+  dft_pass_kernel<R, PREC, S, LO, ROLE, LP><<<(unsigned)grid, G::THREADS, sm, st>>>(a);
   return cudaGetLastError();
 }
 
 template <int R, int PREC, int S1, int S2>
 cudaError_t launch_fused_t(const GArgs &a, int num_sms, cudaStream_t st) {
-  using G1 = Geo<R, S1, S2, kFirst>;
-  using G2 = Geo<R, S2, S1, kSecond, G1::NWG>;
-  const size_t sm = SmemLayout<R, G1::NWG, G1::TW_ENTRIES, G2::TW_ENTRIES, G1::TW_SMEM>::BYTES;
+  using G1 = Geo<R, S1, log2_radix(R) * S2, kFirst>;
+  using G2 = Geo<R, S2, log2_radix(R) * S1, kSecond, 0, G1::NWG>;
+  const size_t sm =
+      SmemLayout<R, G1::NWG, G1::TW_ENTRIES, G2::TW_ENTRIES, G1::TW_SMEM, G1::TWB>::BYTES;
   cudaError_t e = cudaFuncSetAttribute(dft_fused_kernel<R, PREC, S1, S2>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)sm);
@@ -33,12 +34,18 @@ cudaError_t launch_fused_t(const GArgs &a, int num_sms, cudaStream_t st) {
   return cudaGetLastError();
 }
 
-// Supported (s, so, role, sp) combinations of the warpgroup pass kernel for
-// radix R, listed as a compile-time table; the plan only asks for these.
-#define TCU_PASS_CASE(S, SO, ROLE, SP)                                              \
-  if (s == S && so == SO && role == ROLE && sp == SP)                               \
-    return prec == 3 ? launch_pass_t<R, 3, S, SO, ROLE, SP>(a, num_sms, st)         \
-                     : launch_pass_t<R, 1, S, SO, ROLE, SP>(a, num_sms, st);
+// Supported combinations of the warpgroup pass kernel for radix R, listed as
+// a compile-time table; the plan only asks for these.  The dispatcher gets
+// (s, lo, role, lp): stages, log2 of the other size (columns of a strided
+// pass, points before the last pass) and log2 of the prefix count.
+// TCU_PASS_CASE names sizes in stages of R, TCU_PASS_CASE_L in log2 units
+// (mixed radix, where a factor q < R enters).
+#define TCU_PASS_CASE_L(S, LO, ROLE, LP)                                            \
+  if (s == S && lo == LO && role == ROLE && lp == LP)                               \
+    return prec == 3 ? launch_pass_t<R, 3, S, LO, ROLE, LP>(a, num_sms, st)         \
+                     : launch_pass_t<R, 1, S, LO, ROLE, LP>(a, num_sms, st);
+#define TCU_PASS_CASE(S, SO, ROLE, SP) \
+  TCU_PASS_CASE_L(S, log2_radix(R) * (SO), ROLE, log2_radix(R) * (SP))
 #define TCU_FUSED_CASE(S1, S2)                                                      \
   if (s1 == S1 && s2 == S2)                                                         \
     return prec == 3 ? launch_fused_t<R, 3, S1, S2>(a, num_sms, st)                 \

@@ -57,6 +57,8 @@ struct PassPlan {
   int role;         // kSingle, kFirst (strided) or kSecond (last of several)
   int so;           // kFirst: stages after this pass; kSecond: stages before
   int sp;           // kFirst: stages before this pass
+  int lo;           // log2: columns of a strided pass / points before the last
+  int lp;           // log2: prefix sequences per transform of a strided pass
   int log2L;        // sub-transform length L = r^s
   long long U;      // sub-transforms in the pass
   int modes[3];     // row map of the first / middle / last stage
@@ -67,6 +69,11 @@ struct PassPlan {
   // B only when n2 = r^so exceeds 256)
   float2 *tw_a[2], *tw_b[2];
   CUtensorMap tw_map[2];  // TMA map of tw_a[d]
+  // mixed radix: q > 0 marks the CUDA-core q-point first pass (roots of the
+  // direction); `mixed` a tensor-core pass of a mixed-radix transform
+  int q;
+  RootsQ roots[2];
+  bool mixed;
 };
 
 thread_local int g_last_error = TCU_DFT_OK;
@@ -320,6 +327,59 @@ int plan_stages(int r, int k, int st[kMaxPasses]) {
   return P;
 }
 
+// Mixed radix n = q r^k (q < r a power of two; the base case of the
+// recursion is a DFT of size q < sqrt(m)): a CUDA-core q-point first pass,
+// then the r^k-point transforms of its q rows in one or two tensor-core
+// passes (stage split as plan_stages).  Instantiated: k = 2..4 for r = 8
+// and 16, k = 2..3 for r = 32.  Returns the number of passes (0: not such
+// an n) and fills the passes.
+int plan_mixed(int r, long long n, long long batch, PassPlan pass[kMaxPasses]) {
+  const int log2r = ilog2(r);
+  if (n < 1 || (n & (n - 1))) return 0;
+  const int log2n = ilog2(n), k = log2n / log2r, lq = log2n - k * log2r;
+  const int kmax = r == 32 ? 3 : 4;
+  if (lq == 0 || k < 2 || k > kmax) return 0;
+  int st[kMaxPasses] = {0, 0, 0};
+  const int tc = k <= (r == 8 ? 3 : 2) ? 1 : 2;
+  if (tc == 1) st[0] = k;
+  else {
+    st[0] = k / 2;
+    st[1] = k - st[0];
+  }
+  PassPlan &p0 = pass[0];
+  p0.q = 1 << lq;
+  p0.s = 1;
+  p0.role = kFirst;
+  p0.log2L = lq;
+  p0.lo = k * log2r;
+  p0.lp = 0;
+  p0.U = batch * (n >> lq);
+  for (int d = 0; d < 2; ++d)
+    for (int m = 0; m < 16; ++m) p0.roots[d].w[m] = root(m, p0.q, d == 0 ? -1 : 1);
+  for (int i = 0; i < tc; ++i) {
+    PassPlan &pp = pass[1 + i];
+    pp.mixed = true;
+    pp.s = st[i];
+    pp.log2L = log2r * pp.s;
+    pp.last = (i == tc - 1);
+    if (pp.last) {
+      pp.role = kSecond;
+      pp.lo = lq + (i ? log2r * st[0] : 0);
+      pp.lp = 0;
+    } else {
+      pp.role = kFirst;
+      pp.lo = log2r * st[1];
+      pp.lp = lq;
+    }
+    pp.U = batch * (n >> pp.log2L);
+    pp.modes[0] = pp.role == kFirst ? kUF : kQF;
+    pp.modes[1] = kUF;
+    pp.modes[2] = kUF;
+    pp.swz_tab = choose_swizzle(r, pp.s, pp.modes);
+  }
+  return 1 + tc;
+}
+
 // Role, neighbouring stage counts, size and row maps of pass `pi`.
 void pass_geometry(PassPlan &pp, int pi, int P, const int st[kMaxPasses], int k, int r,
                    long long n, long long batch) {
@@ -340,6 +400,8 @@ void pass_geometry(PassPlan &pp, int pi, int P, const int st[kMaxPasses], int k,
     pp.so = k - before - pp.s;
     pp.sp = before;
   }
+  pp.lo = ilog2(r) * pp.so;
+  pp.lp = ilog2(r) * pp.sp;
   pp.U = batch * (n >> pp.log2L);
   pp.modes[0] = pp.role == kFirst ? kUF : kQF;
   pp.modes[1] = kUF;
@@ -347,14 +409,10 @@ void pass_geometry(PassPlan &pp, int pi, int P, const int st[kMaxPasses], int k,
   pp.swz_tab = choose_swizzle(r, pp.s, pp.modes);
 }
 
-// Inter-pass twiddles of a strided pass: w_M^{k v}, k < L = r^s,
-// v < n2 = r^so, M = L n2; A[k][vl] for vl < min(n2, 256) and, if n2 > 256,
-// B[vh][k] = w_M^{k vh 256}.
-void pass_twiddles(int r, int s, int so, int sign, std::vector<float2> &A,
+// Inter-pass twiddles of a strided pass: w_M^{k v}, k < L, v < n2, M = L n2;
+// A[k][vl] for vl < min(n2, 256) and, if n2 > 256, B[vh][k] = w_M^{k vh 256}.
+void pass_twiddles(long long L, long long n2, int sign, std::vector<float2> &A,
                    std::vector<float2> &B) {
-  long long L = 1, n2 = 1;
-  for (int i = 0; i < s; ++i) L *= r;
-  for (int i = 0; i < so; ++i) n2 *= r;
   const long long M = L * n2, VL = n2 > 256 ? 256 : n2;
   A.resize((size_t)(L * VL));
   for (long long k = 0; k < L; ++k)
@@ -370,9 +428,7 @@ void pass_twiddles(int r, int s, int so, int sign, std::vector<float2> &A,
 
 // TMA map of table A of a strided pass (boxes of GG columns x L rows).
 bool twiddle_map(CUtensorMap *m, const float2 *A, int r, const PassPlan &pp) {
-  const long long L = 1ll << pp.log2L;
-  long long n2 = 1;
-  for (int i = 0; i < pp.so; ++i) n2 *= r;
+  const long long L = 1ll << pp.log2L, n2 = 1ll << pp.lo;
   const long long VL = n2 > 256 ? 256 : n2;
   const long long gg = (128ll * r) >> pp.log2L;
   return encode_map(m, A, VL, L, 1, L * VL, (int)gg, L < 256 ? (int)L : 256);
@@ -381,10 +437,7 @@ bool twiddle_map(CUtensorMap *m, const float2 *A, int r, const PassPlan &pp) {
 // TMA map of a strided pass's input: sequences of M = L n2 points, batch *
 // r^sp of them, seen as [sequence][row a][column v].
 bool input_map(CUtensorMap *m, const void *in, const tcu_dft_plan_s *p, const PassPlan &pp) {
-  const long long L = 1ll << pp.log2L;
-  long long n2 = 1, pre = 1;
-  for (int i = 0; i < pp.so; ++i) n2 *= p->r;
-  for (int i = 0; i < pp.sp; ++i) pre *= p->r;
+  const long long L = 1ll << pp.log2L, n2 = 1ll << pp.lo, pre = 1ll << pp.lp;
   const long long gg = (128ll * p->r) >> pp.log2L;
   return encode_map(m, in, n2, L, p->batch * pre, L * n2, (int)gg, L < 256 ? (int)L : 256);
 }
@@ -408,9 +461,14 @@ void free_plan(tcu_dft_plan_s *p) {
 // ---------------------------------------------------------------- launches
 cudaError_t pass_dispatch(int r, int prec, const PassPlan &pp, const GArgs &a, int num_sms,
                           cudaStream_t st) {
-  if (r == 8) return launch_pass_r8(prec, pp.s, pp.so, pp.role, pp.sp, a, num_sms, st);
-  if (r == 16) return launch_pass_r16(prec, pp.s, pp.so, pp.role, pp.sp, a, num_sms, st);
-  return launch_pass_r32(prec, pp.s, pp.so, pp.role, pp.sp, a, num_sms, st);
+  if (pp.mixed) {
+    if (r == 8) return launch_pass_mixed_r8(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
+    if (r == 16) return launch_pass_mixed_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
+    return launch_pass_mixed_r32(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
+  }
+  if (r == 8) return launch_pass_r8(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
+  if (r == 16) return launch_pass_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
+  return launch_pass_r32(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
 }
 
 cudaError_t fused_dispatch(int r, int prec, int s1, int s2, const GArgs &a, int num_sms,
@@ -457,8 +515,8 @@ void dir_tables(const tcu_dft_plan_s *p, int d, DirTables &t) {
   build_images(p->r, sign, ilog2(p->n), t.img);
   for (int pi = 0; pi < p->npasses; ++pi) {
     const PassPlan &pp = p->pass[pi];
-    t.stage[pi] = stage_twiddles(p->r, pp.s, sign);
-    if (pp.role == kFirst) pass_twiddles(p->r, pp.s, pp.so, sign, t.A[pi], t.B[pi]);
+    t.stage[pi] = stage_twiddles(p->r, pp.q ? 1 : pp.s, sign);
+    if (pp.role == kFirst) pass_twiddles(1ll << pp.log2L, 1ll << pp.lo, sign, t.A[pi], t.B[pi]);
   }
 }
 
@@ -538,7 +596,11 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
     ++k;
   }
   int st[kMaxPasses] = {0, 0, 0};
-  const int npasses = (m == n && k >= 1) ? plan_stages(r, k, st) : 0;
+  PassPlan mixed[kMaxPasses];
+  memset(mixed, 0, sizeof(mixed));
+  const bool is_mixed = m != n;
+  const int npasses = is_mixed ? plan_mixed(r, n, batch, mixed)
+                               : (k >= 1 ? plan_stages(r, k, st) : 0);
   if (npasses == 0 || (long long)batch * n > (1ll << 40)) {
     g_last_error = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
@@ -564,7 +626,10 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
   p->npasses = npasses;
   p->device = dev;
   p->num_sms = prop.multiProcessorCount;
-  for (int pi = 0; pi < npasses; ++pi) pass_geometry(p->pass[pi], pi, npasses, st, k, r, n, batch);
+  if (is_mixed)
+    for (int pi = 0; pi < npasses; ++pi) p->pass[pi] = mixed[pi];
+  else
+    for (int pi = 0; pi < npasses; ++pi) pass_geometry(p->pass[pi], pi, npasses, st, k, r, n, batch);
   int rc = TCU_DFT_OK;
   for (int d = 0; d < 2 && rc == TCU_DFT_OK; ++d) {
     DirTables t;
@@ -576,7 +641,7 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
       if (rc == TCU_DFT_OK && pp.role == kFirst) {
         rc = upload(&pp.tw_a[d], t.A[pi]);
         if (rc == TCU_DFT_OK && !t.B[pi].empty()) rc = upload(&pp.tw_b[d], t.B[pi]);
-        if (rc == TCU_DFT_OK && !twiddle_map(&pp.tw_map[d], pp.tw_a[d], r, pp))
+        if (rc == TCU_DFT_OK && !pp.q && !twiddle_map(&pp.tw_map[d], pp.tw_a[d], r, pp))
           rc = TCU_DFT_ERR_CUDA;
       }
     }
@@ -590,7 +655,8 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
   }
   if (rc == TCU_DFT_OK && npasses >= 2) {
     const PassPlan &p1 = p->pass[0], &p2 = p->pass[1];
-    p->fused = npasses == 2 && p1.s >= 2 && p2.s >= 2 && (flags & TCU_DFT_PLAN_FUSE);
+    p->fused = !is_mixed && npasses == 2 && p1.s >= 2 && p2.s >= 2 &&
+               (flags & TCU_DFT_PLAN_FUSE);
     long long scratch_tf = batch;
     if (p->fused) {
       // chunks of C transforms (a power of two dividing the batch, <= 8);
@@ -678,6 +744,12 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
     float2 *dst = pp.last ? (float2 *)out : p->scratch[pi];
     if (events && cudaEventRecord((cudaEvent_t)events[pi], st) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
+    if (pp.q) {
+      if (launch_radix_q(pp.q, src, dst, p->batch, pp.lo, pp.tw_a[di], pp.tw_b[di],
+                         pp.roots[di], p->num_sms, st) != cudaSuccess)
+        return TCU_DFT_ERR_CUDA;
+      continue;
+    }
     GArgs g;
     memset(&g, 0, sizeof(g));
     g.p[0] = group_pass(p, pi, di, src, dst, -1, -1, inverse);
@@ -1005,13 +1077,15 @@ tcu_dft2_plan_s *make_dft2(int64_t n1, int64_t n2, int64_t batch, int32_t r,
   c.role = kCols;
   c.so = k2;
   c.sp = 0;
+  c.lo = log2r * k2;
+  c.lp = 0;
   c.log2L = log2r * k1;
   c.U = batch * n2;
   c.modes[0] = c.modes[1] = c.modes[2] = kUF;
   c.swz_tab = choose_swizzle(r, c.s, c.modes);
   w.s = k2;
   w.role = kSingle;
-  w.so = w.sp = 0;
+  w.so = w.sp = w.lo = w.lp = 0;
   w.log2L = log2r * k2;
   w.U = batch * n1;
   w.modes[0] = kQF;

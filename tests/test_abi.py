@@ -74,6 +74,9 @@ def test_strerror_and_null_handling(lib):
     (16, 1, 64, 3, 2),
     (48, 1, 16, 3, 2),       # not a power of the radix
     (128, 1, 16, 3, 2),      # power of two but not of 16
+    (2 * 16, 1, 16, 3, 2),   # mixed radix with one radix-16 stage (k < 2)
+    (2 * 16 ** 5, 1, 16, 3, 2),  # mixed radix beyond k = 4
+    (3 * 256, 1, 16, 3, 2),  # a factor that is not a power of two
     (16 ** 7, 1, 16, 3, 2),  # beyond three passes
     (32 ** 7, 1, 32, 3, 2),
     (8 ** 10, 1, 8, 3, 2),

@@ -292,3 +292,28 @@ def test_argument_errors_launch_nothing(pkg):
     assert torch.count_nonzero(buf).item() == 0
     plan.check()
     plan.destroy()
+
+
+# ---- mixed final radix (the base case of size q < sqrt(m)): n = q r^k, a
+# CUDA-core q-point first pass, then tensor-core passes of radix r
+@pytest.mark.parametrize("r,q,k", [(16, 2, 2), (16, 4, 2), (16, 8, 2), (16, 2, 3), (16, 8, 3),
+                                   (16, 2, 4), (16, 4, 4), (16, 8, 4),
+                                   (8, 2, 2), (8, 4, 3), (8, 2, 4), (8, 4, 4),
+                                   (32, 2, 2), (32, 16, 2), (32, 4, 3), (32, 16, 3)])
+@pytest.mark.parametrize("prec", [3, 1])
+def test_mixed_radix(pkg, r, q, k, prec):
+    n = q * r ** k
+    batch = max(2, min(37, (1 << 18) // n))
+    x = inputs.make("normal", n, batch, seed=50 + q + k)
+    y, passes = run(pkg, x, r, prec)
+    assert passes[0] == 1 and sum(passes[1:]) == k
+    check(y, x, prec)
+    yi, _ = run(pkg, x, r, prec, inverse=True)
+    check(yi, x, prec, inverse=True)
+
+
+def test_mixed_radix_in_place(pkg):
+    n = 8 * 16 ** 4
+    x = inputs.make("uniform", n, 3, seed=8)
+    y, _ = run(pkg, x, 16, 3, inplace=True)
+    check(y, x, 3)
