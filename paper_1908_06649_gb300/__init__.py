@@ -19,6 +19,8 @@ from . import _build
 
 TF32 = 1
 X3TF32 = 3
+BF16 = 4
+X3BF16 = 5
 FORWARD = -1
 INVERSE = 1
 

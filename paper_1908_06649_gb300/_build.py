@@ -13,6 +13,7 @@ HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
 UNITS = ["tcu_dft.cu", "kernels_r8.cu", "kernels_r16.cu", "kernels_r32.cu",
          "kernels_mixed_r8.cu", "kernels_mixed_r16.cu", "kernels_mixed_r32.cu",
+         "kernels_bf16_r16.cu",
          "grid_kernels.cu"]
 HEADERS = ["tcgen05.cuh", "group_kernel.cuh", "launch.h",
            "launch_impl.cuh"]

@@ -36,6 +36,8 @@
 #include <cuda.h>
 
 #include "../../include/tcu_dft.h"
+#include <cuda_bf16.h>
+
 #include "tcgen05.cuh"
 
 namespace tcu {
@@ -218,60 +220,91 @@ __device__ __forceinline__ int gswz(int p, uint32_t tabv) {
   return p ^ (int)((tabv ^ (uint32_t)(p >> 4)) & 15u);
 }
 
-// TF32 split of 8 complex values, stored as A operand columns of this
-// thread's TMEM lane.  3xTF32: hi keeps the top 10 explicit mantissa bits
-// (exactly representable in TF32) and lo = v - hi is exact in fp32.  TF32:
-// hi rounded to nearest.
+// Precision modes: 1 TF32, 3 3xTF32 (kind::tf32, K = 8 fp32 per product);
+// 4 BF16, 5 3xBF16 (kind::f16 with bf16 operands, K = 16 per product, two
+// values packed per 32-bit TMEM column).
+__host__ __device__ constexpr bool is_bf16(int PREC) { return PREC >= 4; }
+__host__ __device__ constexpr bool is_split(int PREC) { return PREC == 3 || PREC == 5; }
+// TMEM columns of the A operand for 8 complex values, and bytes of one F_r
+// image (2r x 2r elements).
+__host__ __device__ constexpr int a_cols8(int PREC) { return is_bf16(PREC) ? 8 : 16; }
+__host__ __device__ constexpr int img_bytes(int R, int PREC) {
+  return (is_bf16(PREC) ? 8 : 16) * R * R;
+}
+
+// Split of 8 complex values, stored as A operand columns of this thread's
+// TMEM lane.  3xTF32: hi keeps the top 10 explicit mantissa bits (exactly
+// representable in TF32) and lo = v - hi is exact in fp32.  TF32: hi rounded
+// to nearest.  BF16 modes: hi = bf16 rounding of v, lo = bf16 rounding of
+// v - hi (exact in fp32 before rounding), packed two per column.
 template <int PREC>
 __device__ __forceinline__ void split_store8(const float2 *x, uint32_t col_hi,
                                              uint32_t col_lo) {
-  float vh[16], vl[16];
+  if constexpr (is_bf16(PREC)) {
+    uint32_t ph[8], pl[8];
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    if (PREC == 3) {
-      const float hx = __uint_as_float(__float_as_uint(x[j].x) & 0xFFFFE000u);
-      const float hy = __uint_as_float(__float_as_uint(x[j].y) & 0xFFFFE000u);
-      vh[2 * j] = hx;
-      vh[2 * j + 1] = hy;
-      vl[2 * j] = x[j].x - hx;
-      vl[2 * j + 1] = x[j].y - hy;
-    } else {
-      vh[2 * j] = tf32_rna(x[j].x);
-      vh[2 * j + 1] = tf32_rna(x[j].y);
+    for (int j = 0; j < 8; ++j) {
+      const __nv_bfloat16 hx = __float2bfloat16_rn(x[j].x), hy = __float2bfloat16_rn(x[j].y);
+      ph[j] = (uint32_t)__bfloat16_as_ushort(hx) | ((uint32_t)__bfloat16_as_ushort(hy) << 16);
+      if (PREC == 5) {
+        const __nv_bfloat16 lx = __float2bfloat16_rn(x[j].x - __bfloat162float(hx));
+        const __nv_bfloat16 ly = __float2bfloat16_rn(x[j].y - __bfloat162float(hy));
+        pl[j] = (uint32_t)__bfloat16_as_ushort(lx) | ((uint32_t)__bfloat16_as_ushort(ly) << 16);
+      }
     }
+    tmem_st8u(col_hi, ph);
+    if (PREC == 5) tmem_st8u(col_lo, pl);
+  } else {
+    float vh[16], vl[16];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      if (PREC == 3) {
+        const float hx = __uint_as_float(__float_as_uint(x[j].x) & 0xFFFFE000u);
+        const float hy = __uint_as_float(__float_as_uint(x[j].y) & 0xFFFFE000u);
+        vh[2 * j] = hx;
+        vh[2 * j + 1] = hy;
+        vl[2 * j] = x[j].x - hx;
+        vl[2 * j + 1] = x[j].y - hy;
+      } else {
+        vh[2 * j] = tf32_rna(x[j].x);
+        vh[2 * j + 1] = tf32_rna(x[j].y);
+      }
+    }
+    tmem_st16(col_hi, vh);
+    if (PREC == 3) tmem_st16(col_lo, vl);
   }
-  tmem_st16(col_hi, vh);
-  if (PREC == 3) tmem_st16(col_lo, vl);
 }
 
 // One stage: D = A * Bf for the 128 rows of this warpgroup's slot.
-// 3xTF32: one accumulator chain over K = 6r, i.e. [A_lo | A_hi | A_hi] times
-// [Bhi; Blo; Bhi] stacked -- lo*Bhi + hi*Blo + hi*Bhi, small terms first
-// (lo*Blo is below fp32 resolution and dropped).  The three K-blocks read the
-// same TMEM columns of A_hi twice; D has N = 2r columns and needs no sum in
-// the epilogue.
+// Split modes: one accumulator chain over three K-blocks, [A_lo | A_hi |
+// A_hi] times [Bhi; Blo; Bhi] stacked -- lo*Bhi + hi*Blo + hi*Bhi, small
+// terms first (lo*Blo is dropped: below the target precision).  The
+// K-blocks read the same TMEM columns of A_hi twice; D has N = 2r columns.
+// Each product covers 32 bytes of K: 8 fp32 (kind::tf32) or 16 bf16
+// (kind::f16), i.e. 8 TMEM columns of A and two 16-byte core matrices of B.
 template <int R, int PREC>
 __device__ __forceinline__ void issue_stage_mma(uint32_t slot, uint32_t img_addr) {
   constexpr int Q = (2 * R > 32) ? 2 * R : 32;
-  constexpr int IMG = 16 * R * R, LBO = 128, SBO = 64 * R, KSTEPS = 2 * R / 8;
-  constexpr uint32_t idesc = idesc_tf32(128, 2 * R);
+  constexpr bool BF = is_bf16(PREC);
+  constexpr int IMG = img_bytes(R, PREC), LBO = 128, SBO = (BF ? 32 : 64) * R;
+  constexpr int KSTEPS = 2 * R / (BF ? 16 : 8);
+  constexpr uint32_t idesc = BF ? idesc_bf16(128, 2 * R) : idesc_tf32(128, 2 * R);
   const uint32_t ahi = slot, alo = slot + Q, d = slot + 2 * Q;
   const uint32_t ihi = img_addr, ilo = img_addr + IMG;
   uint32_t acc = 0;
-  if (PREC == 3) {
+  if (is_split(PREC)) {
 #pragma unroll
     for (int kk = 0; kk < KSTEPS; ++kk) {
-      mma_tf32_ts(d, alo + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO), idesc,
-                  acc);
+      mma_ts<BF>(d, alo + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO), idesc, acc);
       acc = 1;
     }
 #pragma unroll
     for (int kk = 0; kk < KSTEPS; ++kk)
-      mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(ilo + kk * 2 * LBO, LBO, SBO), idesc, 1);
+      mma_ts<BF>(d, ahi + 8 * kk, smem_desc_noswz(ilo + kk * 2 * LBO, LBO, SBO), idesc, 1);
   }
 #pragma unroll
   for (int kk = 0; kk < KSTEPS; ++kk) {
-    mma_tf32_ts(d, ahi + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO), idesc, acc);
+    mma_ts<BF>(d, ahi + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO), idesc, acc);
     acc = 1;
   }
 }
@@ -416,7 +449,8 @@ __device__ __forceinline__ void stage_rows(const PRun &P, const WG &w) {
     float2 row[8];
 #pragma unroll
     for (int jj = 0; jj < 8; ++jj) row[jj] = w.buf[gswz(base + ((c + jj) << SH), tabv)];
-    split_store8<PREC>(row, w.slot + w.lane_off + 2 * c, w.slot + G::Q + w.lane_off + 2 * c);
+    split_store8<PREC>(row, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
+                       w.slot + G::Q + w.lane_off + a_cols8(PREC) * c / 8);
   }
 }
 
@@ -497,7 +531,8 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
     staged_row<G>(w, x);
 #pragma unroll
     for (int c = 0; c < R; c += 8)
-      split_store8<PREC>(x + c, w.slot + w.lane_off + 2 * c, w.slot + G::Q + w.lane_off + 2 * c);
+      split_store8<PREC>(x + c, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
+                         w.slot + G::Q + w.lane_off + a_cols8(PREC) * c / 8);
   }
   tmem_wait_st();
   fence_before_sync();

@@ -159,16 +159,38 @@ float2 root(long long m, long long period, int sign) {
   return make_float2((float)cos(ang), (float)sin(ang));
 }
 
+// Round an fp32 value to bf16 (8 significant bits), nearest-even; the bits.
+uint16_t host_bf16_rne(float x) {
+  uint32_t b;
+  memcpy(&b, &x, 4);
+  if ((b & 0x7F800000u) != 0x7F800000u) b += 0x7FFFu + ((b >> 16) & 1u);
+  return (uint16_t)(b >> 16);
+}
+
+float host_bf16_value(uint16_t h) {
+  const uint32_t b = (uint32_t)h << 16;
+  float r;
+  memcpy(&r, &b, 4);
+  return r;
+}
+
+bool prec_bf16(int precision) { return precision == TCU_DFT_BF16 || precision == TCU_DFT_3XBF16; }
+
 // B operand images of the real 2r x 2r block form of F_r for one direction,
 // in the canonical no-swizzle K-major layout the MMA reads: hi, lo, and the
 // same two scaled by 2^-log2n (exact: a power of two) for the inverse's last
-// stage, which folds the 1/n normalisation into the product.
-void build_images(int r, int sign, int log2n, std::vector<float> &out) {
+// stage, which folds the 1/n normalisation into the product.  Core matrices
+// are 8 rows x 16 bytes: 4 fp32 (TF32 modes) or 8 bf16 (BF16 modes) of K;
+// the four images sit at multiples of their size (16 r^2 or 8 r^2 bytes) in
+// a buffer of 64 r^2 bytes.
+void build_images(int r, int sign, int log2n, int precision, std::vector<float> &out) {
   const int K = 2 * r, N = 2 * r;
-  const int lbo = 128, sbo = 64 * r;
-  const size_t img_floats = (size_t)16 * r * r / 4;
+  const bool bf = prec_bf16(precision);
+  const size_t lbo = 128, sbo = (bf ? 32 : 64) * (size_t)r, esz = bf ? 2 : 4;
+  const size_t img_bytes = (bf ? 8 : 16) * (size_t)r * r;
   const float sc = ldexpf(1.0f, -log2n);
-  out.assign(4 * img_floats, 0.f);
+  out.assign((size_t)16 * r * r, 0.f);  // 64 r^2 bytes
+  unsigned char *bytes = reinterpret_cast<unsigned char *>(out.data());
   for (int kr = 0; kr < K; ++kr) {
     for (int nc = 0; nc < N; ++nc) {
       const int j = kr >> 1, a = kr & 1, c = nc >> 1, b = nc & 1;
@@ -180,15 +202,21 @@ void build_images(int r, int sign, int log2n, std::vector<float> &out) {
         v = (b == 0) ? re : im;
       else
         v = (b == 0) ? -im : re;
-      const float hi = host_tf32_rna((float)v);
-      const float lo = host_tf32_rna((float)(v - (double)hi));
-      const size_t off =
-          ((size_t)(nc >> 3) * sbo + (size_t)(kr >> 2) * lbo + (nc & 7) * 16 +
-           (kr & 3) * 4) / 4;
-      out[off] = hi;
-      out[img_floats + off] = lo;
-      out[2 * img_floats + off] = hi * sc;
-      out[3 * img_floats + off] = lo * sc;
+      const int per = bf ? 8 : 4;  // K elements per core-matrix row
+      const size_t off = (size_t)(nc >> 3) * sbo + (size_t)(kr / per) * lbo + (nc & 7) * 16 +
+                         (size_t)(kr % per) * esz;
+      if (bf) {
+        const uint16_t hi = host_bf16_rne((float)v);
+        const uint16_t lo = host_bf16_rne((float)(v - (double)host_bf16_value(hi)));
+        const uint16_t vals[4] = {hi, lo, host_bf16_rne(host_bf16_value(hi) * sc),
+                                  host_bf16_rne(host_bf16_value(lo) * sc)};
+        for (int i = 0; i < 4; ++i) memcpy(bytes + i * img_bytes + off, &vals[i], 2);
+      } else {
+        const float hi = host_tf32_rna((float)v);
+        const float lo = host_tf32_rna((float)(v - (double)hi));
+        const float vals[4] = {hi, lo, hi * sc, lo * sc};
+        for (int i = 0; i < 4; ++i) memcpy(bytes + i * img_bytes + off, &vals[i], 4);
+      }
     }
   }
 }
@@ -466,6 +494,7 @@ cudaError_t pass_dispatch(int r, int prec, const PassPlan &pp, const GArgs &a, i
     if (r == 16) return launch_pass_mixed_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
     return launch_pass_mixed_r32(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   }
+  if (prec_bf16(prec)) return launch_pass_bf16_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   if (r == 8) return launch_pass_r8(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   if (r == 16) return launch_pass_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   return launch_pass_r32(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
@@ -499,7 +528,7 @@ PRun group_pass(const tcu_dft_plan_s *p, int pi, int di, const float2 *in, float
   g.tw_stage = pp.tw_stage[di];
   g.swz_tab = pp.swz_tab;
   // the inverse's last stage uses the F images scaled by 1/n
-  g.last_img = (pp.last && inverse) ? 2 * 16 * p->r * p->r : 0;
+  g.last_img = (pp.last && inverse) ? 2 * (prec_bf16(p->precision) ? 8 : 16) * p->r * p->r : 0;
   return g;
 }
 
@@ -512,7 +541,7 @@ struct DirTables {
 
 void dir_tables(const tcu_dft_plan_s *p, int d, DirTables &t) {
   const int sign = d == 0 ? -1 : 1;
-  build_images(p->r, sign, ilog2(p->n), t.img);
+  build_images(p->r, sign, ilog2(p->n), p->precision, t.img);
   for (int pi = 0; pi < p->npasses; ++pi) {
     const PassPlan &pp = p->pass[pi];
     t.stage[pi] = stage_twiddles(p->r, pp.q ? 1 : pp.s, sign);
@@ -578,7 +607,8 @@ tcu_dft_plan_t tcu_dft_plan(int64_t n, int64_t batch, int32_t sqrt_m,
 tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
                                int32_t precision, uint32_t flags) {
   g_last_error = TCU_DFT_OK;
-  if (n < 1 || batch < 1 || (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32) ||
+  if (n < 1 || batch < 1 ||
+      (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32 && !prec_bf16(precision)) ||
       (flags & ~(uint32_t)(TCU_DFT_PLAN_NO_FUSE | TCU_DFT_PLAN_FUSE)) ||
       ((flags & TCU_DFT_PLAN_NO_FUSE) && (flags & TCU_DFT_PLAN_FUSE))) {
     g_last_error = TCU_DFT_ERR_INVALID;
@@ -601,7 +631,9 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
   const bool is_mixed = m != n;
   const int npasses = is_mixed ? plan_mixed(r, n, batch, mixed)
                                : (k >= 1 ? plan_stages(r, k, st) : 0);
-  if (npasses == 0 || (long long)batch * n > (1ll << 40)) {
+  // the BF16 modes are instantiated for radix 16, r^k sizes
+  if (npasses == 0 || (long long)batch * n > (1ll << 40) ||
+      (prec_bf16(precision) && (r != 16 || is_mixed))) {
     g_last_error = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
   }
@@ -655,8 +687,8 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
   }
   if (rc == TCU_DFT_OK && npasses >= 2) {
     const PassPlan &p1 = p->pass[0], &p2 = p->pass[1];
-    p->fused = !is_mixed && npasses == 2 && p1.s >= 2 && p2.s >= 2 &&
-               (flags & TCU_DFT_PLAN_FUSE);
+    p->fused = !is_mixed && !prec_bf16(precision) && npasses == 2 && p1.s >= 2 &&
+               p2.s >= 2 && (flags & TCU_DFT_PLAN_FUSE);
     long long scratch_tf = batch;
     if (p->fused) {
       // chunks of C transforms (a power of two dividing the batch, <= 8);
@@ -829,9 +861,11 @@ int tcu_dft_pass_stages(tcu_dft_plan_t p, int i) {
 int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t precision,
                          const void *in, void *out, int dir, void *stream) {
   // ---- arguments (no CUDA call before they are known to be good)
-  if (n < 1 || batch < 1 || (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32) ||
+  if (n < 1 || batch < 1 ||
+      (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32 && !prec_bf16(precision)) ||
       !in || !out || (dir != TCU_DFT_FORWARD && dir != TCU_DFT_INVERSE))
     return TCU_DFT_ERR_INVALID;
+  if (prec_bf16(precision)) return TCU_DFT_ERR_UNSUPPORTED;
   if (sqrt_m != 8 && sqrt_m != 16 && sqrt_m != 32) return TCU_DFT_ERR_UNSUPPORTED;
   const int r = sqrt_m, log2r = ilog2(r);
   int k = 0;
@@ -1043,8 +1077,12 @@ tcu_dft2_plan_s *make_dft2(int64_t n1, int64_t n2, int64_t batch, int32_t r,
                            int32_t precision, int &rc) {
   rc = TCU_DFT_OK;
   if (n1 < 1 || n2 < 1 || batch < 1 ||
-      (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32)) {
+      (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32 && !prec_bf16(precision))) {
     rc = TCU_DFT_ERR_INVALID;
+    return nullptr;
+  }
+  if (prec_bf16(precision)) {  // the 2-D passes are instantiated for the TF32 modes
+    rc = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
   }
   int k1 = 0, k2 = 0;
@@ -1095,7 +1133,7 @@ tcu_dft2_plan_s *make_dft2(int64_t n1, int64_t n2, int64_t batch, int32_t r,
   for (int d = 0; d < 2 && rc == TCU_DFT_OK; ++d) {
     const int sign = d == 0 ? -1 : 1;
     std::vector<float> img;
-    build_images(r, sign, ilog2(n1 * n2), img);
+    build_images(r, sign, ilog2(n1 * n2), precision, img);
     rc = upload(&p->bimg[d], img);
     if (rc == TCU_DFT_OK) rc = upload(&c.tw_stage[d], stage_twiddles(r, c.s, sign));
     if (rc == TCU_DFT_OK) rc = upload(&w.tw_stage[d], stage_twiddles(r, w.s, sign));
@@ -1199,8 +1237,13 @@ int tcu_dft2_destroy(tcu_dft2_plan_t p) {
 tcu_stencil_plan_t tcu_stencil_plan(int64_t side, int32_t steps, int32_t sqrt_m,
                                     int32_t precision) {
   g_last_error = TCU_DFT_OK;
-  if (side < 1 || steps < 1 || (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32)) {
+  if (side < 1 || steps < 1 ||
+      (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32 && !prec_bf16(precision))) {
     g_last_error = TCU_DFT_ERR_INVALID;
+    return nullptr;
+  }
+  if (prec_bf16(precision)) {
+    g_last_error = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
   }
   const long long N = (sqrt_m == 8 || sqrt_m == 16 || sqrt_m == 32) ? grid_side(sqrt_m, 3ll * steps) : 0;
