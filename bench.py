@@ -323,7 +323,7 @@ def run_grid(args):
             spec = one.forward(w)
             one.check()
             step = lambda: plan.conv(x, spec, y)
-            passes, flops = 4, 2 * 5.0 * N * math.log2(N) * batch
+            passes, flops = 3, 2 * 5.0 * N * math.log2(N) * batch
         else:
             step = lambda: plan.forward(x, y)
             passes, flops = 2, 5.0 * N * math.log2(N) * batch
@@ -357,10 +357,10 @@ def run_grid(args):
             Nt *= r
         tiles = (side // k) ** 2
         points = tiles * Nt * Nt
-        passes = 4
+        passes = 3
         # weights: place, 2-D DFT (2), power, inverse (2); kernel W': place,
-        # 2-D DFT (2); tiles: gather, convolution (4), extract
-        launches = 15
+        # 2-D DFT (2); tiles: gather, convolution (3), extract
+        launches = 14
         unit = "Gupdates/s"
         metric = ("linear stencil grid-point updates/s (side^2 x steps), "
                   "%d^2 grid x %d steps, 1xGB300" % (side, k))
@@ -394,14 +394,14 @@ def run_grid(args):
     ms = t0.elapsed_time(t1) / K
     cpu = None if args.no_cpu_baseline else grid_cpu_baseline(args, g)
     if args.grid == "stencil":
-        # whole step: the four convolution passes (16 B per tile point each),
+        # whole step: the three convolution passes (16 B per tile point each),
         # the gather (tile points written, the grid read once) and the
         # extract (one tile point read and one grid point written per cell);
         # the weight and kernel-spectrum transforms are tiny
         S = float(side * side)
-        step_bytes = 64.0 * points + 8.0 * points + 4.0 * S + 8.0 * S + 4.0 * S
+        step_bytes = 48.0 * points + 8.0 * points + 4.0 * S + 8.0 * S + 4.0 * S
         achieved = step_bytes / (ms * 1e-3) / 1e9
-        kname = ("whole step (%d launches: weights, kernel spectrum, gather, 4 "
+        kname = ("whole step (%d launches: weights, kernel spectrum, gather, 3 "
                  "convolution passes, extract), %.2f GB algorithmic" % (launches, step_bytes / 1e9))
     else:
         achieved = 16.0 * points / (ms / passes * 1e-3) / 1e9

@@ -199,8 +199,8 @@ int tcu_dft2_exec(tcu_dft2_plan_t p, const void *in, void *out, int dir, void *s
 /* out = IDFT2(DFT2(in) * spectrum) for every array of the batch: the
  * circular convolution of each array with the one n1 x n2 array whose 2-D
  * DFT is `spectrum` (device, n1*n2 complex64, e.g. from tcu_dft2_exec on a
- * batch-1 plan).  Four passes: columns, rows times the spectrum, inverse
- * rows, inverse columns. */
+ * batch-1 plan).  Three passes: columns; rows transformed, multiplied by
+ * the spectrum and transformed back on chip; inverse columns. */
 int tcu_conv2_exec(tcu_dft2_plan_t p, const void *in, const void *spectrum, void *out,
                    void *stream);
 int tcu_dft2_check(tcu_dft2_plan_t p, void *stream);  /* as tcu_dft_check */
@@ -231,6 +231,20 @@ int tcu_stencil_exec(tcu_stencil_plan_t p, const float *w3x3, const float *A, fl
                      void *stream);
 int tcu_stencil_check(tcu_stencil_plan_t p, void *stream);
 int tcu_stencil_destroy(tcu_stencil_plan_t p);
+
+/* Failure-detection self-test (not a transform): runs a fused plan's
+ * schedule with its work queue started past work that then never runs, so
+ * that the dependency waits of the items it claims cannot be satisfied.
+ * Every such wait gives up after its limit (2 s of the global timer); the
+ * kernel records TCU_DFT_ERR_TIMEOUT in the plan's error word, waits
+ * (bounded) for its own copies in flight, frees its tensor memory and
+ * returns, leaving the context usable: tcu_dft_check then reports
+ * TCU_DFT_ERR_TIMEOUT and clears the word, and the plan transforms normally
+ * afterwards.  No fault, trap or unbounded wait is involved.  `out` receives
+ * partial data.  Needs a fused plan (TCU_DFT_PLAN_FUSE) with at least
+ * lag + 2 chunks of transforms (batch >= 48 for n = 16^4); ERR_INVALID
+ * otherwise.  Asynchronous on `stream`. */
+int tcu_dft_exec_stalled(tcu_dft_plan_t p, const void *in, void *out, void *stream);
 
 /* Status of the last plan call (tcu_dft_plan*, tcu_dft2_plan,
  * tcu_stencil_plan) on this thread. */

@@ -39,7 +39,7 @@ PLAN_FUSE = 2
 SYMBOLS = (
     "tcu_dft_plan", "tcu_dft_plan_ex", "tcu_dft_is_fused", "tcu_dft_exec",
     "tcu_dft_exec_dir", "tcu_dft_exec_timed",
-    "tcu_dft_exec_host", "tcu_dft_exec_noalloc",
+    "tcu_dft_exec_host", "tcu_dft_exec_noalloc", "tcu_dft_exec_stalled",
     "tcu_dft_check", "tcu_dft_destroy", "tcu_dft_num_passes",
     "tcu_dft_pass_stages", "tcu_dft_last_error", "tcu_dft_strerror",
     "tcu_dft2_plan", "tcu_dft2_exec", "tcu_conv2_exec", "tcu_dft2_check",
@@ -90,6 +90,8 @@ def lib():
     L.tcu_dft_exec_noalloc.argtypes = [i64, i64, i32, i32, vp, vp, ctypes.c_int,
                                        vp]
     L.tcu_dft_exec_noalloc.restype = ctypes.c_int
+    L.tcu_dft_exec_stalled.argtypes = [vp, vp, vp, vp]
+    L.tcu_dft_exec_stalled.restype = ctypes.c_int
     L.tcu_dft_check.argtypes = [vp, vp]
     L.tcu_dft_check.restype = ctypes.c_int
     L.tcu_dft_destroy.argtypes = [vp]

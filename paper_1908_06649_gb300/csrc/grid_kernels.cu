@@ -76,32 +76,36 @@ __global__ void place_kernel_kernel(float2 *w, long long N, const float2 *g, lon
 
 // Tile (r, c) of the side x side grid A as the N x N complex array whose
 // top-left 3k x 3k block is A'_{r,c} = A[(r-1)k .. (r+2)k)[(c-1)k .. (c+2)k)
-// (zero outside A) and whose other entries are 0.
+// (zero outside A) and whose other entries are 0.  One block per tile,
+// 32 x 8 threads: rows by threadIdx.y, columns by threadIdx.x, so reads of A
+// and writes of the tile are contiguous along the columns.
 __global__ void gather_tiles_kernel(float2 *tiles, const float *A, long long side, int k,
-                                    long long N, long long tpr) {
-  const long long count = tpr * tpr * N * N;
-  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < count;
-       e += (long long)gridDim.x * blockDim.x) {
-    const long long t = e / (N * N), ij = e % (N * N);
-    const long long i = ij / N, j = ij % N;
-    const long long gi = (t / tpr - 1) * k + i, gj = (t % tpr - 1) * k + j;
-    float v = 0.f;
-    if (i < 3 * k && j < 3 * k && gi >= 0 && gi < side && gj >= 0 && gj < side)
-      v = __ldg(A + gi * side + gj);
-    tiles[e] = make_float2(v, 0.f);
+                                    int N, long long tpr) {
+  const long long t = blockIdx.x;
+  const long long r0 = (t / tpr - 1) * k, c0 = (t % tpr - 1) * k;
+  float2 *dst = tiles + t * N * N;
+  for (int i = threadIdx.y; i < N; i += blockDim.y) {
+    const long long gi = r0 + i;
+    const bool row_in = i < 3 * k && gi >= 0 && gi < side;
+    for (int j = threadIdx.x; j < N; j += blockDim.x) {
+      const long long gj = c0 + j;
+      float v = 0.f;
+      if (row_in && j < 3 * k && gj >= 0 && gj < side) v = __ldg(A + gi * side + gj);
+      __stcs(dst + (long long)i * N + j, make_float2(v, 0.f));
+    }
   }
 }
 
-// A_k[rk + i][ck + j] = Re tile_{r,c}[k + i][k + j] for i, j < k.
+// A_k[rk + i][ck + j] = Re tile_{r,c}[k + i][k + j] for i, j < k: one block
+// per tile, contiguous along the columns.
 __global__ void extract_tiles_kernel(float *Ak, const float2 *tiles, long long side, int k,
-                                     long long N, long long tpr) {
-  const long long count = side * side;
-  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < count;
-       e += (long long)gridDim.x * blockDim.x) {
-    const long long gi = e / side, gj = e % side;
-    const long long t = (gi / k) * tpr + gj / k;
-    Ak[e] = tiles[t * N * N + (k + gi % k) * N + (k + gj % k)].x;
-  }
+                                     int N, long long tpr) {
+  const long long t = blockIdx.x;
+  const long long r0 = (t / tpr) * k, c0 = (t % tpr) * k;
+  const float2 *src = tiles + t * N * N + (long long)k * N + k;
+  for (int i = threadIdx.y; i < k; i += blockDim.y)
+    for (int j = threadIdx.x; j < k; j += blockDim.x)
+      Ak[(r0 + i) * side + c0 + j] = __ldcs(src + (long long)i * N + j).x;
 }
 
 unsigned grid_for(long long count, int num_sms) {
@@ -140,16 +144,16 @@ cudaError_t launch_place_kernel(float2 *w, long long N, const float2 *g, long lo
 cudaError_t launch_gather_tiles(float2 *tiles, const float *A, long long side, int k,
                                 long long N, int num_sms, cudaStream_t st) {
   const long long tpr = side / k;
-  gather_tiles_kernel<<<grid_for(tpr * tpr * N * N, num_sms), kBlock, 0, st>>>(tiles, A, side,
-                                                                              k, N, tpr);
+  gather_tiles_kernel<<<(unsigned)(tpr * tpr), dim3(32, 8), 0, st>>>(tiles, A, side, k, (int)N,
+                                                                    tpr);
   return cudaGetLastError();
 }
 
 cudaError_t launch_extract_tiles(float *Ak, const float2 *tiles, long long side, int k,
                                  long long N, int num_sms, cudaStream_t st) {
   const long long tpr = side / k;
-  extract_tiles_kernel<<<grid_for(side * side, num_sms), kBlock, 0, st>>>(Ak, tiles, side, k,
-                                                                         N, tpr);
+  extract_tiles_kernel<<<(unsigned)(tpr * tpr), dim3(32, 8), 0, st>>>(Ak, tiles, side, k,
+                                                                     (int)N, tpr);
   return cudaGetLastError();
 }
 

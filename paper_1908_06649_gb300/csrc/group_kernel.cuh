@@ -455,7 +455,7 @@ __device__ __forceinline__ void stage_rows(const PRun &P, const WG &w) {
 }
 
 // Last stage: D -> registers -> natural-order output.
-template <class G, int PREC, bool OUT_L2>
+template <class G, int PREC, bool OUT_L2, bool SPEC = true>
 __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, WG &w) {
   constexpr int R = 1 << G::LOG2R;
   constexpr int S = G::LOG2L / G::LOG2R;
@@ -497,7 +497,7 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, 
   const float2 *twbg = P.tw_b + (vh << G::LOG2L) + klow;
   constexpr int TBJ = 1 << (G::LOG2L - G::LOG2R);
   const float2 *sp = P.spec + ((u & P.spec_mask) << G::LOG2L) + klow;
-  const bool mul = G::MODE_LAST == kRQF && P.spec != nullptr;
+  const bool mul = SPEC && G::MODE_LAST == kRQF && P.spec != nullptr;
 #pragma unroll
   for (int j = 0; j < R; ++j) {
     float2 y = make_float2(d[2 * j], d[2 * j + 1]);
@@ -581,6 +581,126 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
   last_stage_store<G, PREC, OUT_L2>(P, item, w);
 }
 
+// Convolution row item (kSingle geometry): the forward transform of each
+// row, the product with the spectrum, and the inverse transform, all on chip.
+// The thread that holds forward outputs k = klow + j r^(S-1) of a row after
+// the last forward stage (digit-reversed row map) is the thread whose
+// inverse stage-1 row is exactly those k in the same order (natural row
+// map, same TMEM lane): it multiplies them by the spectrum and stores them
+// straight back as its A operand.  F images in SMEM: forward hi, lo at 0,
+// inverse hi, lo at 2 IMG; stage twiddles tw_f (forward), tw_i (inverse).
+template <class G, int PREC>
+__device__ __forceinline__ void conv_turn(const PRun &P, long long item, const WG &w) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  int ul, q;
+  row_of<G>(kRQF, w.rho, ul, q);
+  int klow = 0, vq = q;
+#pragma unroll
+  for (int i = 0; i < S - 1; ++i) {
+    klow = (klow << G::LOG2R) | (vq & (R - 1));
+    vq >>= G::LOG2R;
+  }
+  const long long u = (item << G::LOG2GG) + ul;
+  float d[2 * R];
+  load_d_row<G, PREC>(w, d);
+  const float2 *sp = P.spec + ((u & P.spec_mask) << G::LOG2L) + klow;
+  constexpr int JS = 1 << (G::LOG2L - G::LOG2R);
+#pragma unroll
+  for (int c = 0; c < R; c += 8) {
+    float2 x[8];
+#pragma unroll
+    for (int jj = 0; jj < 8; ++jj)
+      x[jj] = cmul(make_float2(d[2 * (c + jj)], d[2 * (c + jj) + 1]), __ldg(sp + (c + jj) * JS));
+    split_store8<PREC>(x, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
+                       w.slot + G::Q + w.lane_off + a_cols8(PREC) * c / 8);
+  }
+}
+
+// Stages 2..S of one direction after the stage-1 products were issued:
+// epilogue, transpose, next products (F images at img_off).
+template <class G, int PREC, class Mid>
+__device__ __forceinline__ bool later_stages(const PRun &P, const float2 *tws, WG &w,
+                                             uint32_t img_off, Mid &mid, bool publish) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  constexpr int S2 = S >= 2 ? 2 : S, S3 = S >= 3 ? 3 : S2;
+#pragma unroll
+  for (int t = 1; t < S; ++t) {
+    if (t == 1) stage_epilogue<G, PREC, 1>(P, tws, w);
+    if (t == 2) stage_epilogue<G, PREC, S2>(P, tws, w);
+    if (publish && t == 1 && w.rho < 32) mid.publish();
+    fence_before_sync();
+    named_bar_or(w.bar_id, 128, false);
+    if (t == 1) stage_rows<G, PREC, S2>(P, w);
+    if (t == 2) stage_rows<G, PREC, S3>(P, w);
+    tmem_wait_st();
+    fence_before_sync();
+    if (named_bar_or(w.bar_id, 128, w.fail)) {
+      w.fail = true;
+      return false;
+    }
+    if (w.rho < 32) {
+      fence_after_sync();
+      issue_stage<R, PREC>(w.slot, w.img_addr + img_off, w.bar_mma);
+    }
+    if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
+    w.ph_mma ^= 1;
+    fence_after_sync();
+  }
+  return true;
+}
+
+template <class G, int PREC, class Mid>
+__device__ __forceinline__ void process_item_conv(const PRun &P, const float2 *tw_f,
+                                                  const float2 *tw_i, long long item, WG &w,
+                                                  Mid &mid) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr uint32_t INV = 2 * img_bytes(R, PREC);
+  if (!mbar_wait_bounded(w.bar_stg, w.ph_stg)) w.fail = true;
+  w.ph_stg ^= 1;
+  {
+    float2 x[R];
+    staged_row<G>(w, x);
+#pragma unroll
+    for (int c = 0; c < R; c += 8)
+      split_store8<PREC>(x + c, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
+                         w.slot + G::Q + w.lane_off + a_cols8(PREC) * c / 8);
+  }
+  tmem_wait_st();
+  fence_before_sync();
+  if (named_bar_or(w.bar_id, 128, w.fail)) {
+    w.fail = true;
+    return;
+  }
+  if (w.rho < 32) {
+    fence_after_sync();
+    issue_stage<R, PREC>(w.slot, w.img_addr, w.bar_mma);
+    mid.issue(w);
+  }
+  if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
+  w.ph_mma ^= 1;
+  fence_after_sync();
+  if (!later_stages<G, PREC>(P, tw_f, w, 0, mid, true)) return;
+  // the turn: forward outputs times the spectrum become the inverse A rows
+  conv_turn<G, PREC>(P, item, w);
+  tmem_wait_st();
+  fence_before_sync();
+  if (named_bar_or(w.bar_id, 128, w.fail)) {
+    w.fail = true;
+    return;
+  }
+  if (w.rho < 32) {
+    fence_after_sync();
+    issue_stage<R, PREC>(w.slot, w.img_addr + INV, w.bar_mma);
+  }
+  if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
+  w.ph_mma ^= 1;
+  fence_after_sync();
+  if (!later_stages<G, PREC>(P, tw_i, w, INV, mid, false)) return;
+  last_stage_store<G, PREC, false, false>(P, item, w);
+}
+
 // Common set-up: F images and stage twiddles into SMEM, mbarriers, TMEM.
 template <int NWG, int THREADS>
 __device__ __forceinline__ uint32_t kernel_setup(const float *bimg, int img_floats,
@@ -661,19 +781,22 @@ struct StaticNext {
   __device__ void publish() {}
 };
 
-template <int R, int PREC, int S, int LO, int ROLE, int LP>
+template <int R, int PREC, int S, int LO, int ROLE, int LP, bool CONV = false>
 __global__ void __launch_bounds__(Geo<R, S, LO, ROLE, LP>::THREADS, 1)
     dft_pass_kernel(const __grid_constant__ GArgs a) {
   using G = Geo<R, S, LO, ROLE, LP>;
-  using SM = SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM, G::TWB>;
+  static_assert(!CONV || ROLE == kSingle, "convolution rows are whole transforms");
+  using SM = SmemLayout<R, G::NWG, G::TW_ENTRIES, CONV ? G::TW_ENTRIES : 0, G::TW_SMEM, G::TWB>;
   extern __shared__ __align__(1024) unsigned char smem[];
   float2 *tw = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
+  float2 *tw_inv = reinterpret_cast<float2 *>(smem + SM::OFF_TW2);
   uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + SM::OFF_BAR);
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 3 * G::NWG);
   const PRun &P = a.p[0];
+  // a convolution row pass also holds the inverse stage twiddles (p[1])
   const uint32_t tbase = kernel_setup<G::NWG, G::THREADS>(
       a.bimg, (int)(SM::IMG / 4), reinterpret_cast<float *>(smem), P.tw_stage, tw,
-      G::TW_ENTRIES, P.tw_stage, tw, 0, mbar, tmem_slot);
+      G::TW_ENTRIES, a.p[1].tw_stage, tw_inv, CONV ? G::TW_ENTRIES : 0, mbar, tmem_slot);
   WG w;
   init_wg<R, SM, G::GCOLS>(w, tbase, smem);
 
@@ -685,7 +808,10 @@ __global__ void __launch_bounds__(Geo<R, S, LO, ROLE, LP>::THREADS, 1)
   if (w.rho < 32 && item < nitems) issue_input<G>(P, &a.tm_in, item, w);
   while (item < nitems && !w.fail) {
     nx.next = item + istride;
-    process_item<G, PREC, false>(P, &a.tm_tw, tw, item, w, nx);
+    if constexpr (CONV)
+      process_item_conv<G, PREC>(P, tw, tw_inv, item, w, nx);
+    else
+      process_item<G, PREC, false>(P, &a.tm_tw, tw, item, w, nx);
     item += istride;
   }
   if (w.fail && w.rho == 0) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);

@@ -43,4 +43,13 @@ cudaError_t launch_fused_r8(int prec, int s1, int s2, const GArgs &a, int num_sm
   return cudaErrorInvalidValue;
 }
 
+cudaError_t launch_rowconv_r8(int prec, int s, const GArgs &a, int num_sms,
+                               cudaStream_t st) {
+  constexpr int R = 8;
+  TCU_ROWCONV_CASE(1)
+  TCU_ROWCONV_CASE(2)
+  TCU_ROWCONV_CASE(3)
+  return cudaErrorInvalidValue;
+}
+
 }  // namespace tcu

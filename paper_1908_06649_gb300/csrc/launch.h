@@ -17,6 +17,11 @@ cudaError_t launch_pass_r16(int prec, int s, int lo, int role, int lp, const GAr
                             int num_sms, cudaStream_t st);
 cudaError_t launch_pass_r32(int prec, int s, int lo, int role, int lp, const GArgs &a,
                             int num_sms, cudaStream_t st);
+// The row pass of a circular 2-D convolution: each row transformed,
+// multiplied by the spectrum and transformed back on chip (s stages).
+cudaError_t launch_rowconv_r8(int prec, int s, const GArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_rowconv_r16(int prec, int s, const GArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_rowconv_r32(int prec, int s, const GArgs &a, int num_sms, cudaStream_t st);
 // Both passes of a two-pass transform fused in one launch (s1, s2 >= 2).
 cudaError_t launch_fused_r8(int prec, int s1, int s2, const GArgs &a, int num_sms,
                             cudaStream_t st);

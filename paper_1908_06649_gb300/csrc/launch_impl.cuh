@@ -20,6 +20,27 @@ cudaError_t launch_pass_t(const GArgs &a, int num_sms, cudaStream_t st) {
   return cudaGetLastError();
 }
 
+// The convolution row pass (forward rows, spectrum product, inverse rows).
+template <int R, int PREC, int S>
+cudaError_t launch_rowconv_t(const GArgs &a, int num_sms, cudaStream_t st) {
+  using G = Geo<R, S, 0, kSingle>;
+  const size_t sm = SmemLayout<R, G::NWG, G::TW_ENTRIES, G::TW_ENTRIES, false, 0>::BYTES;
+  cudaError_t e = cudaFuncSetAttribute(dft_pass_kernel<R, PREC, S, 0, kSingle, 0, true>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)sm);
+  if (e != cudaSuccess) return e;
+  const long long nitems = (a.p[0].U + G::GG - 1) >> G::LOG2GG;
+  long long grid = (nitems + G::NWG - 1) / G::NWG;
+  if (grid > num_sms) grid = num_sms;
+  dft_pass_kernel<R, PREC, S, 0, kSingle, 0, true><<<(unsigned)grid, G::THREADS, sm, st>>>(a);
+  return cudaGetLastError();
+}
+
+#define TCU_ROWCONV_CASE(S)                                                         \
+  if (s == S)                                                                       \
+    return prec == 3 ? launch_rowconv_t<R, 3, S>(a, num_sms, st)                    \
+                     : launch_rowconv_t<R, 1, S>(a, num_sms, st);
+
 template <int R, int PREC, int S1, int S2>
 cudaError_t launch_fused_t(const GArgs &a, int num_sms, cudaStream_t st) {
   using G1 = Geo<R, S1, log2_radix(R) * S2, kFirst>;

@@ -729,7 +729,7 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
 }
 
 static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
-                     void *stream, void *const *events) {
+                     void *stream, void *const *events, long long queue_start = 0) {
   if (!p || !in || !out || (dir != TCU_DFT_FORWARD && dir != TCU_DFT_INVERSE))
     return TCU_DFT_ERR_INVALID;
   if (((uintptr_t)in & 15) || ((uintptr_t)out & 15)) return TCU_DFT_ERR_INVALID;
@@ -757,6 +757,14 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
     g.log2_items_per_chunk = p->log2_items_per_chunk;
     if (cudaMemsetAsync(p->counters, 0, p->counter_bytes, st) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
+    if (queue_start > 0) {
+      // failure-detection self-test: start the queue past work that then
+      // never runs (pageable source: copied before the call returns)
+      const int head = (int)queue_start;
+      if (cudaMemcpyAsync(p->counters, &head, sizeof(int), cudaMemcpyHostToDevice, st) !=
+          cudaSuccess)
+        return TCU_DFT_ERR_CUDA;
+    }
     if (events && cudaEventRecord((cudaEvent_t)events[0], st) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
     if (fused_dispatch(p->r, p->precision, p->pass[0].s, p->pass[1].s, g, p->num_sms,
@@ -802,6 +810,14 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
 int tcu_dft_exec_dir(tcu_dft_plan_t p, const void *in, void *out, int dir,
                      void *stream) {
   return exec_impl(p, in, out, dir, stream, nullptr);
+}
+
+int tcu_dft_exec_stalled(tcu_dft_plan_t p, const void *in, void *out, void *stream) {
+  // the first items claimed are the pass-2 items of chunk 0, whose pass-1
+  // items sit before the start and never run
+  if (!p || !p->fused || p->nchunks < p->lag + 2) return TCU_DFT_ERR_INVALID;
+  const long long start = (long long)(p->lag + 1) << p->log2_items_per_chunk;
+  return exec_impl(p, in, out, TCU_DFT_FORWARD, stream, nullptr, start);
 }
 
 int tcu_dft_exec_timed(tcu_dft_plan_t p, const void *in, void *out, int dir,
@@ -977,9 +993,9 @@ int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t preci
 // every column, then of every row) is two warpgroup passes: the column pass
 // (kCols: kFirst's strided geometry without a twiddle, T[b][k1][v]) and the
 // row pass (kSingle over batch * n1 rows, natural order).  A circular
-// convolution with a fixed array whose spectrum S is given is four: columns,
-// rows times S, inverse rows, inverse columns (1/(n1 n2) folded into the
-// last stage's F images).
+// convolution with a fixed array whose spectrum S is given is three:
+// columns, rows (forward, times S, inverse -- on chip, one item at a time),
+// inverse columns (1/(n1 n2) folded into the last stage's F images).
 
 }  // extern "C"
 
@@ -988,6 +1004,7 @@ struct tcu_dft2_plan_s {
   int r, precision, num_sms;
   PassPlan cols, rows;
   float *bimg[2];     // [dir index]; scaled copies by 2^-log2(n1 n2)
+  float *cimg;        // convolution rows: forward hi, lo | inverse hi, lo
   float2 *scratch;    // batch * n1 * n2
   int *err;
 };
@@ -1026,6 +1043,7 @@ void free_dft2(tcu_dft2_plan_s *p) {
     cudaFree(p->cols.tw_stage[d]);
     cudaFree(p->rows.tw_stage[d]);
   }
+  cudaFree(p->cimg);
   cudaFree(p->scratch);
   cudaFree(p->err);
   delete p;
@@ -1130,14 +1148,18 @@ tcu_dft2_plan_s *make_dft2(int64_t n1, int64_t n2, int64_t batch, int32_t r,
   w.modes[1] = kUF;
   w.modes[2] = kRQF;
   w.swz_tab = choose_swizzle(r, w.s, w.modes);
+  std::vector<float> conv_img;
   for (int d = 0; d < 2 && rc == TCU_DFT_OK; ++d) {
     const int sign = d == 0 ? -1 : 1;
     std::vector<float> img;
     build_images(r, sign, ilog2(n1 * n2), precision, img);
     rc = upload(&p->bimg[d], img);
+    // hi and lo of this direction (the first two images)
+    conv_img.insert(conv_img.end(), img.begin(), img.begin() + img.size() / 2);
     if (rc == TCU_DFT_OK) rc = upload(&c.tw_stage[d], stage_twiddles(r, c.s, sign));
     if (rc == TCU_DFT_OK) rc = upload(&w.tw_stage[d], stage_twiddles(r, w.s, sign));
   }
+  if (rc == TCU_DFT_OK) rc = upload(&p->cimg, conv_img);
   if (rc == TCU_DFT_OK &&
       (cudaMalloc((void **)&p->scratch, (size_t)(batch * n1 * n2) * sizeof(float2)) !=
            cudaSuccess ||
@@ -1206,14 +1228,23 @@ int tcu_conv2_exec(tcu_dft2_plan_t p, const void *in, const void *spectrum, void
   int rc = check_buffers(in, out, bytes);
   if (rc != TCU_DFT_OK) return rc;
   cudaStream_t st = (cudaStream_t)stream;
-  float2 *o = (float2 *)out;
-  // in -> scratch -> out -> scratch -> out (in is read by the first pass only)
+  // columns: in -> scratch; rows forward, times the spectrum and inverse on
+  // chip: scratch -> scratch (an item reads its rows before writing them);
+  // inverse columns with 1/(n1 n2): scratch -> out
   rc = run_dft2_pass(p, p->cols, 0, (const float2 *)in, p->scratch, false, nullptr, st);
-  if (rc == TCU_DFT_OK)
-    rc = run_dft2_pass(p, p->rows, 0, p->scratch, o, false, (const float2 *)spectrum, st);
-  if (rc == TCU_DFT_OK) rc = run_dft2_pass(p, p->rows, 1, o, p->scratch, false, nullptr, st);
-  if (rc == TCU_DFT_OK) rc = run_dft2_pass(p, p->cols, 1, p->scratch, o, true, nullptr, st);
-  return rc;
+  if (rc != TCU_DFT_OK) return rc;
+  GArgs g;
+  memset(&g, 0, sizeof(g));
+  g.p[0] = dft2_pass(p, p->rows, 0, p->scratch, p->scratch, false, (const float2 *)spectrum);
+  g.p[1].tw_stage = p->rows.tw_stage[1];
+  g.bimg = p->cimg;
+  g.err = p->err;
+  cudaError_t e;
+  if (p->r == 8) e = launch_rowconv_r8(p->precision, p->rows.s, g, p->num_sms, st);
+  else if (p->r == 16) e = launch_rowconv_r16(p->precision, p->rows.s, g, p->num_sms, st);
+  else e = launch_rowconv_r32(p->precision, p->rows.s, g, p->num_sms, st);
+  if (e != cudaSuccess) return TCU_DFT_ERR_CUDA;
+  return run_dft2_pass(p, p->cols, 1, p->scratch, (float2 *)out, true, nullptr, st);
 }
 
 int tcu_dft2_check(tcu_dft2_plan_t p, void *stream) {

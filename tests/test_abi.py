@@ -57,6 +57,7 @@ def test_strerror_and_null_handling(lib):
     assert lib.tcu_dft_exec_dir(None, None, None, -1, None) == pkg.ERR_INVALID
     assert lib.tcu_dft_exec_host(None, None, None, None, -1, None) == pkg.ERR_INVALID
     assert lib.tcu_dft_check(None, None) == pkg.ERR_INVALID
+    assert lib.tcu_dft_exec_stalled(None, None, None, None) == pkg.ERR_INVALID
     assert lib.tcu_dft_num_passes(None) == -1
     assert lib.tcu_dft_is_fused(None) == -1
     assert not lib.tcu_dft_plan_ex(256, 4, 16, 3, 4)   # unknown flag bit
