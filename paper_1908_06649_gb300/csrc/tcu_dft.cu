@@ -51,6 +51,7 @@ using namespace tcu;
 namespace {
 
 constexpr int kMaxPasses = 3;
+constexpr int kHostChunks = 16;  // pipeline depth of the host-buffer path
 
 struct PassPlan {
   int s;            // stages
@@ -102,6 +103,10 @@ struct tcu_dft_plan_s {
   size_t counter_bytes;
   int *err;
   int device;
+  // host-buffer path: copy streams and per-chunk events (created by the plan)
+  cudaStream_t copy_in, copy_out;
+  cudaEvent_t ev_start, ev_in[kHostChunks], ev_done[kHostChunks], ev_out[kHostChunks];
+  bool has_copy_streams;
 };
 
 namespace {
@@ -464,14 +469,26 @@ bool twiddle_map(CUtensorMap *m, const float2 *A, int r, const PassPlan &pp) {
 
 // TMA map of a strided pass's input: sequences of M = L n2 points, batch *
 // r^sp of them, seen as [sequence][row a][column v].
-bool input_map(CUtensorMap *m, const void *in, const tcu_dft_plan_s *p, const PassPlan &pp) {
+bool input_map(CUtensorMap *m, const void *in, const tcu_dft_plan_s *p, const PassPlan &pp,
+               long long batch) {
   const long long L = 1ll << pp.log2L, n2 = 1ll << pp.lo, pre = 1ll << pp.lp;
   const long long gg = (128ll * p->r) >> pp.log2L;
-  return encode_map(m, in, n2, L, p->batch * pre, L * n2, (int)gg, L < 256 ? (int)L : 256);
+  return encode_map(m, in, n2, L, batch * pre, L * n2, (int)gg, L < 256 ? (int)L : 256);
 }
 
 void free_plan(tcu_dft_plan_s *p) {
   if (!p) return;
+  if (p->has_copy_streams) {
+    // null handles (creation failed part-way) are skipped
+    if (p->copy_in) cudaStreamSynchronize(p->copy_in), cudaStreamDestroy(p->copy_in);
+    if (p->copy_out) cudaStreamSynchronize(p->copy_out), cudaStreamDestroy(p->copy_out);
+    if (p->ev_start) cudaEventDestroy(p->ev_start);
+    for (int i = 0; i < kHostChunks; ++i) {
+      if (p->ev_in[i]) cudaEventDestroy(p->ev_in[i]);
+      if (p->ev_done[i]) cudaEventDestroy(p->ev_done[i]);
+      if (p->ev_out[i]) cudaEventDestroy(p->ev_out[i]);
+    }
+  }
   for (int d = 0; d < 2; ++d) {
     cudaFree(p->bimg[d]);
     for (int i = 0; i < kMaxPasses; ++i) {
@@ -514,7 +531,7 @@ bool overlaps(const void *a, const void *b, size_t bytes) {
 
 // Warpgroup-kernel description of pass `pi` between buffers `in` and `out`.
 PRun group_pass(const tcu_dft_plan_s *p, int pi, int di, const float2 *in, float2 *out,
-                long long in_bmask, long long out_bmask, bool inverse) {
+                long long in_bmask, long long out_bmask, bool inverse, long long batch) {
   const PassPlan &pp = p->pass[pi];
   PRun g;
   memset(&g, 0, sizeof(g));
@@ -522,7 +539,7 @@ PRun group_pass(const tcu_dft_plan_s *p, int pi, int di, const float2 *in, float
   g.out = out;
   g.in_bmask = in_bmask;
   g.out_bmask = out_bmask;
-  g.U = pp.U;
+  g.U = batch * (p->n >> pp.log2L);
   g.tw_out = pp.tw_a[di];
   g.tw_b = pp.tw_b[di];
   g.tw_stage = pp.tw_stage[di];
@@ -720,6 +737,20 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
         rc = TCU_DFT_ERR_OOM;
       }
   }
+  if (rc == TCU_DFT_OK) {
+    bool ok = cudaStreamCreateWithFlags(&p->copy_in, cudaStreamNonBlocking) == cudaSuccess &&
+              cudaStreamCreateWithFlags(&p->copy_out, cudaStreamNonBlocking) == cudaSuccess &&
+              cudaEventCreateWithFlags(&p->ev_start, cudaEventDisableTiming) == cudaSuccess;
+    for (int i = 0; i < kHostChunks && ok; ++i)
+      ok = cudaEventCreateWithFlags(&p->ev_in[i], cudaEventDisableTiming) == cudaSuccess &&
+           cudaEventCreateWithFlags(&p->ev_done[i], cudaEventDisableTiming) == cudaSuccess &&
+           cudaEventCreateWithFlags(&p->ev_out[i], cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) {
+      cudaGetLastError();
+      rc = TCU_DFT_ERR_CUDA;
+    }
+    p->has_copy_streams = true;  // whatever was created is freed with the plan
+  }
   if (rc != TCU_DFT_OK) {
     free_plan(p);
     g_last_error = rc;
@@ -728,12 +759,20 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
   return p;
 }
 
+// The transform of transforms [b0, b0 + count) of the plan's batch (in and
+// out point at transform b0; count < 0: the whole batch).  The intermediates
+// of that range sit at the same offset in the plan's scratch, so disjoint
+// ranges may run concurrently on different streams (not fused plans).
 static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
-                     void *stream, void *const *events, long long queue_start = 0) {
+                     void *stream, void *const *events, long long queue_start = 0,
+                     long long b0 = 0, long long count = -1) {
   if (!p || !in || !out || (dir != TCU_DFT_FORWARD && dir != TCU_DFT_INVERSE))
     return TCU_DFT_ERR_INVALID;
   if (((uintptr_t)in & 15) || ((uintptr_t)out & 15)) return TCU_DFT_ERR_INVALID;
-  const size_t bytes = (size_t)p->batch * p->n * sizeof(float2);
+  if (count < 0) count = p->batch;
+  if (b0 < 0 || b0 + count > p->batch || (p->fused && count != p->batch))
+    return TCU_DFT_ERR_INVALID;
+  const size_t bytes = (size_t)count * p->n * sizeof(float2);
   if (in != out && overlaps(in, out, bytes)) return TCU_DFT_ERR_INVALID;
   cudaStream_t st = (cudaStream_t)stream;
   const int di = dir_index(dir);
@@ -742,9 +781,11 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
     GArgs g;
     memset(&g, 0, sizeof(g));
     const long long ring_mask = ((long long)p->ring_chunks << p->log2C) - 1;
-    g.p[0] = group_pass(p, 0, di, (const float2 *)in, p->scratch[0], -1, ring_mask, inverse);
-    g.p[1] = group_pass(p, 1, di, p->scratch[0], (float2 *)out, ring_mask, -1, inverse);
-    if (!input_map(&g.tm_in, in, p, p->pass[0])) return TCU_DFT_ERR_CUDA;
+    g.p[0] = group_pass(p, 0, di, (const float2 *)in, p->scratch[0], -1, ring_mask, inverse,
+                        p->batch);
+    g.p[1] = group_pass(p, 1, di, p->scratch[0], (float2 *)out, ring_mask, -1, inverse,
+                        p->batch);
+    if (!input_map(&g.tm_in, in, p, p->pass[0], p->batch)) return TCU_DFT_ERR_CUDA;
     g.tm_tw = p->pass[0].tw_map[di];
     g.bimg = p->bimg[di];
     g.err = p->err;
@@ -778,23 +819,24 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
   }
 
   // in -> scratch[0] -> scratch[1] -> out
+  const long long off = b0 * p->n;
   for (int pi = 0; pi < p->npasses; ++pi) {
     const PassPlan &pp = p->pass[pi];
-    const float2 *src = (pi == 0) ? (const float2 *)in : p->scratch[pi - 1];
-    float2 *dst = pp.last ? (float2 *)out : p->scratch[pi];
+    const float2 *src = (pi == 0) ? (const float2 *)in : p->scratch[pi - 1] + off;
+    float2 *dst = pp.last ? (float2 *)out : p->scratch[pi] + off;
     if (events && cudaEventRecord((cudaEvent_t)events[pi], st) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
     if (pp.q) {
-      if (launch_radix_q(pp.q, src, dst, p->batch, pp.lo, pp.tw_a[di], pp.tw_b[di],
+      if (launch_radix_q(pp.q, src, dst, count, pp.lo, pp.tw_a[di], pp.tw_b[di],
                          pp.roots[di], p->num_sms, st) != cudaSuccess)
         return TCU_DFT_ERR_CUDA;
       continue;
     }
     GArgs g;
     memset(&g, 0, sizeof(g));
-    g.p[0] = group_pass(p, pi, di, src, dst, -1, -1, inverse);
+    g.p[0] = group_pass(p, pi, di, src, dst, -1, -1, inverse, count);
     if (pp.role == kFirst) {
-      if (!input_map(&g.tm_in, src, p, pp)) return TCU_DFT_ERR_CUDA;
+      if (!input_map(&g.tm_in, src, p, pp, count)) return TCU_DFT_ERR_CUDA;
       g.tm_tw = pp.tw_map[di];
     }
     g.bimg = p->bimg[di];
@@ -834,17 +876,57 @@ int tcu_dft_exec(tcu_dft_plan_t p, const void *in, void *out, void *stream) {
 
 int tcu_dft_exec_host(tcu_dft_plan_t p, const void *h_in, void *h_out, void *d_work,
                       int dir, void *stream) {
-  if (!p || !h_in || !h_out || !d_work) return TCU_DFT_ERR_INVALID;
+  if (!p || !h_in || !h_out || !d_work || (dir != TCU_DFT_FORWARD && dir != TCU_DFT_INVERSE))
+    return TCU_DFT_ERR_INVALID;
   if ((uintptr_t)d_work & 15) return TCU_DFT_ERR_INVALID;
   const size_t bytes = (size_t)p->batch * p->n * sizeof(float2);
   cudaStream_t st = (cudaStream_t)stream;
-  if (cudaMemcpyAsync(d_work, h_in, bytes, cudaMemcpyHostToDevice, st) != cudaSuccess)
+  if (p->fused || !p->has_copy_streams || p->batch < 2) {
+    if (cudaMemcpyAsync(d_work, h_in, bytes, cudaMemcpyHostToDevice, st) != cudaSuccess)
+      return TCU_DFT_ERR_CUDA;
+    const int rc = tcu_dft_exec_dir(p, d_work, d_work, dir, stream);
+    if (rc != TCU_DFT_OK) return rc;
+    if (cudaMemcpyAsync(h_out, d_work, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess)
+      return TCU_DFT_ERR_CUDA;
+    return TCU_DFT_OK;
+  }
+  // Pipelined over up to kHostChunks chunks of transforms: chunk c's host->device
+  // copy (copy_in stream), its transform (the caller's stream) and its
+  // device->host copy (copy_out stream) overlap with the neighbouring
+  // chunks'; events order each chunk's three steps and join the copy
+  // streams to the caller's stream at both ends.
+  const long long C = p->batch < kHostChunks ? p->batch : kHostChunks;
+  const long long per = (p->batch + C - 1) / C;
+  float2 *d = (float2 *)d_work;
+  const float2 *hin = (const float2 *)h_in;
+  float2 *hout = (float2 *)h_out;
+  if (cudaEventRecord(p->ev_start, st) != cudaSuccess ||
+      cudaStreamWaitEvent(p->copy_in, p->ev_start, 0) != cudaSuccess ||
+      cudaStreamWaitEvent(p->copy_out, p->ev_start, 0) != cudaSuccess)
     return TCU_DFT_ERR_CUDA;
-  const int rc = tcu_dft_exec_dir(p, d_work, d_work, dir, stream);
-  if (rc != TCU_DFT_OK) return rc;
-  if (cudaMemcpyAsync(h_out, d_work, bytes, cudaMemcpyDeviceToHost, st) != cudaSuccess)
-    return TCU_DFT_ERR_CUDA;
-  return TCU_DFT_OK;
+  int last = 0;
+  for (long long c = 0; c < C; ++c) {
+    const long long b0 = c * per;
+    if (b0 >= p->batch) break;
+    const long long cnt = (b0 + per <= p->batch) ? per : p->batch - b0;
+    const size_t off = (size_t)(b0 * p->n), cb = (size_t)cnt * p->n * sizeof(float2);
+    if (cudaMemcpyAsync(d + off, hin + off, cb, cudaMemcpyHostToDevice, p->copy_in) !=
+            cudaSuccess ||
+        cudaEventRecord(p->ev_in[c], p->copy_in) != cudaSuccess ||
+        cudaStreamWaitEvent(st, p->ev_in[c], 0) != cudaSuccess)
+      return TCU_DFT_ERR_CUDA;
+    const int rc = exec_impl(p, d + off, d + off, dir, stream, nullptr, 0, b0, cnt);
+    if (rc != TCU_DFT_OK) return rc;
+    if (cudaEventRecord(p->ev_done[c], st) != cudaSuccess ||
+        cudaStreamWaitEvent(p->copy_out, p->ev_done[c], 0) != cudaSuccess ||
+        cudaMemcpyAsync(hout + off, d + off, cb, cudaMemcpyDeviceToHost, p->copy_out) !=
+            cudaSuccess ||
+        cudaEventRecord(p->ev_out[c], p->copy_out) != cudaSuccess)
+      return TCU_DFT_ERR_CUDA;
+    last = (int)c;
+  }
+  return cudaStreamWaitEvent(st, p->ev_out[last], 0) == cudaSuccess ? TCU_DFT_OK
+                                                                     : TCU_DFT_ERR_CUDA;
 }
 
 int tcu_dft_check(tcu_dft_plan_t p, void *stream) {

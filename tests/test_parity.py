@@ -340,3 +340,24 @@ def test_bf16_modes(pkg, k, batch, prec):
     yi, _ = run(pkg, x, 16, prec, inverse=True)
     erri = oracle.rel_l2(yi, oracle.dft(x, inverse=True, threads=8))
     assert erri.max() <= BF16_TOL[prec], erri.max()
+
+
+@pytest.mark.parametrize("n,batch,r", [(8 ** 4, 13, 8), (16 ** 5, 5, 16), (2 * 16 ** 4, 3, 16),
+                                       (32 ** 3, 9, 32)])
+def test_exec_host_pipelined(pkg, n, batch, r):
+    # host buffers in chunks of transforms: copies on two internal streams
+    # overlap the transforms of neighbouring chunks (ragged last chunk)
+    import torch
+    x = inputs.make("normal", n, batch, seed=70)
+    plan = pkg.Plan(n, batch, r, 3)
+    h_in = torch.from_numpy(x).pin_memory()
+    h_out = torch.empty_like(h_in).pin_memory()
+    work = torch.empty(batch * n, dtype=torch.complex64, device="cuda")
+    for _ in range(2):  # twice in a row: the second reuses the streams
+        plan.exec_host(h_in, h_out, work)
+        plan.check()
+        check(h_out.numpy().reshape(batch, n), x, 3)
+    plan.exec_host(h_in, h_out, work, pkg.INVERSE)
+    plan.check()
+    check(h_out.numpy().reshape(batch, n), x, 3, inverse=True)
+    plan.destroy()
