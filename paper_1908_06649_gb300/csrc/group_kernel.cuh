@@ -49,7 +49,7 @@ __host__ __device__ constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 
 // Warpgroups per CTA: TMEM holds 512 columns, a warpgroup's slot 3 Q of
 // them; a first (strided) pass also stages its inter-pass twiddles in SMEM,
 // which leaves room for four.
-constexpr int pass_nwg(int R, int ROLE) { return R == 32 ? 2 : (ROLE == 1 ? 4 : 5); }
+__host__ __device__ constexpr int pass_nwg(int R, int ROLE) { return R == 32 ? 2 : (ROLE == 1 ? 4 : 5); }
 
 // Compile-time geometry of one pass: S stages of radix R.  A transform of
 // length n is computed in up to three passes (the four-step split applied
@@ -66,12 +66,23 @@ constexpr int pass_nwg(int R, int ROLE) { return R == 32 ? 2 : (ROLE == 1 ? 4 : 
 //            x[b n + a n2 + v] -> X[b n + k n2 + v]
 //   kSecond: last of several passes, n1 = 2^LO points before it per row:
 //            T[b n + v L + a] -> y[b n + v + k n1]
-template <int R, int S, int LO, int ROLE, int LP = 0, int NWG_ = pass_nwg(R, ROLE)>
+//
+// An item is the work of a team of TW warpgroups: 128 TW data rows, each
+// warpgroup's 128 rows one M = 128 product per stage into its own TMEM slot;
+// the team shares the item's SMEM staging and transpose buffers and
+// synchronises on one named barrier.  TW > 1 lets an item hold sub-transforms
+// longer than 128 rows, or more columns of a strided pass.
+template <int R, int S, int LO, int ROLE, int LP = 0, int NWG_ = pass_nwg(R, ROLE),
+          int TW_ = 1>
 struct Geo {
   static constexpr int LOG2R = log2_radix(R);
   static constexpr int NWG = NWG_;
+  static constexpr int TW = TW_;
+  static constexpr int LOG2TW = TW == 1 ? 0 : (TW == 2 ? 1 : 2);
+  static constexpr int NTEAM = NWG / TW;
+  static constexpr int ROWS = 128 * TW;
   static constexpr int THREADS = 128 * NWG;
-  static constexpr int LOG2GPTS = 7 + LOG2R;   // 128 rows of R points
+  static constexpr int LOG2GPTS = 7 + LOG2TW + LOG2R;   // ROWS rows of R points
   static constexpr int GPTS = 1 << LOG2GPTS;
   static constexpr int LOG2L = LOG2R * S;
   static constexpr int L = 1 << LOG2L;
@@ -108,6 +119,7 @@ struct Geo {
   static_assert(LOG2GG <= LOG2VL || !TW_OUT, "an item spans one twiddle column block");
   static_assert(LOG2GG <= LOG2UPER || !STRIDED, "an item spans columns of one sequence");
   static_assert(NWG * GCOLS <= 512, "TMEM budget");
+  static_assert(NTEAM * TW == NWG && (TW == 1 || TW == 2 || TW == 4), "team size");
 };
 
 // Runtime part of a pass.
@@ -158,19 +170,20 @@ __host__ __device__ constexpr int tw_stage_offset(int t) {
 // transpose buffer, input staging and twiddle staging | mbarriers (3 per
 // warpgroup: products, input staging, twiddle staging) | TMEM slot |
 // scheduler mailboxes.
-template <int R, int NWG, int TW1, int TW2, bool TWS, int TWB = 0>
+template <int R, int NWG, int TW1, int TW2, bool TWS, int TWB = 0, int TEAM = 1>
 struct SmemLayout {
+  static constexpr int NTEAM = NWG / TEAM;
   static constexpr size_t IMG = 4 * 16 * R * R;
   static constexpr size_t OFF_TW1 = IMG;
   static constexpr size_t OFF_TW2 = OFF_TW1 + (size_t)TW1 * 8;
-  static constexpr size_t PTS = 128 * R;  // points per item
+  static constexpr size_t PTS = 128 * (size_t)TEAM * R;  // points per item
   static constexpr size_t OFF_BUF = (OFF_TW2 + (size_t)TW2 * 8 + 127) / 128 * 128;
-  static constexpr size_t OFF_STG = OFF_BUF + (size_t)NWG * PTS * 8;
-  static constexpr size_t OFF_TWS = OFF_STG + (size_t)NWG * PTS * 8;
-  static constexpr size_t TWS_BYTES = TWS ? (size_t)NWG * PTS * 8 : 0;
+  static constexpr size_t OFF_STG = OFF_BUF + (size_t)NTEAM * PTS * 8;
+  static constexpr size_t OFF_TWS = OFF_STG + (size_t)NTEAM * PTS * 8;
+  static constexpr size_t TWS_BYTES = TWS ? (size_t)NTEAM * PTS * 8 : 0;
   static constexpr size_t OFF_TWB = OFF_TWS + TWS_BYTES;  // [k] row of table B
-  static constexpr size_t TWB_PER_WG = TWB;
-  static constexpr size_t TWB_BYTES = (size_t)NWG * TWB * 8;
+  static constexpr size_t TWB_PER_WG = TWB;               // per team
+  static constexpr size_t TWB_BYTES = (size_t)NTEAM * TWB * 8;
   static constexpr size_t OFF_BAR = OFF_TWB + TWB_BYTES;
   static constexpr size_t OFF_SCHED = OFF_BAR + 8 * 3 * NWG + 8;
   static constexpr size_t BYTES = OFF_SCHED + 32 * NWG;
@@ -185,8 +198,11 @@ struct WG {
   uint32_t bar_mma;   // mbarrier: products done
   uint32_t bar_stg;   // mbarrier: input staging full
   uint32_t bar_tws;   // mbarrier: twiddle staging full
-  int bar_id;         // named barrier id
-  int rho;            // this thread's row within the item (0..127)
+  int bar_id;         // named barrier id (one per team)
+  int bar_count;      // threads of the team
+  int rho;            // this thread's row within the item (0 .. 128 TW - 1)
+  bool wg_lead;       // warp 0 of its warpgroup: issues the warpgroup's products
+  bool team_lead;     // warp 0 of the team: issues copies, runs the schedule
   float2 *buf;        // SMEM transpose buffer
   float2 *stg;        // SMEM input staging (one item)
   float2 *tws;        // SMEM twiddle staging (one item)
@@ -536,14 +552,16 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
   }
   tmem_wait_st();
   fence_before_sync();
-  if (named_bar_or(w.bar_id, 128, w.fail)) {
+  if (named_bar_or(w.bar_id, w.bar_count, w.fail)) {
     w.fail = true;
     return;
   }
   // staging is free again: the next item's copy may land there
-  if (w.rho < 32) {
+  if (w.wg_lead) {
     fence_after_sync();
     issue_stage<R, PREC>(w.slot, w.img_addr + (S == 1 ? P.last_img : 0), w.bar_mma);
+  }
+  if (w.team_lead) {
     if (G::TW_SMEM) {
       issue_twiddles<G>(P, tm_tw, item, w);
       w.tws_inflight = true;
@@ -558,18 +576,18 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
   for (int t = 1; t < S; ++t) {
     if (t == 1) stage_epilogue<G, PREC, 1>(P, tws, w);
     if (t == 2) stage_epilogue<G, PREC, S2>(P, tws, w);
-    if (t == 1 && w.rho < 32) mid.publish();
+    if (t == 1 && w.team_lead) mid.publish();
     fence_before_sync();
-    named_bar_or(w.bar_id, 128, false);
+    named_bar_or(w.bar_id, w.bar_count, false);
     if (t == 1) stage_rows<G, PREC, S2>(P, w);
     if (t == 2) stage_rows<G, PREC, S3>(P, w);
     tmem_wait_st();
     fence_before_sync();
-    if (named_bar_or(w.bar_id, 128, w.fail)) {
+    if (named_bar_or(w.bar_id, w.bar_count, w.fail)) {
       w.fail = true;
       return;
     }
-    if (w.rho < 32) {
+    if (w.wg_lead) {
       fence_after_sync();
       issue_stage<R, PREC>(w.slot, w.img_addr + (t + 1 == S ? P.last_img : 0), w.bar_mma);
     }
@@ -577,7 +595,7 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
     w.ph_mma ^= 1;
     fence_after_sync();
   }
-  if (S == 1 && w.rho < 32) mid.publish();
+  if (S == 1 && w.team_lead) mid.publish();
   last_stage_store<G, PREC, OUT_L2>(P, item, w);
 }
 
@@ -629,18 +647,18 @@ __device__ __forceinline__ bool later_stages(const PRun &P, const float2 *tws, W
   for (int t = 1; t < S; ++t) {
     if (t == 1) stage_epilogue<G, PREC, 1>(P, tws, w);
     if (t == 2) stage_epilogue<G, PREC, S2>(P, tws, w);
-    if (publish && t == 1 && w.rho < 32) mid.publish();
+    if (publish && t == 1 && w.team_lead) mid.publish();
     fence_before_sync();
-    named_bar_or(w.bar_id, 128, false);
+    named_bar_or(w.bar_id, w.bar_count, false);
     if (t == 1) stage_rows<G, PREC, S2>(P, w);
     if (t == 2) stage_rows<G, PREC, S3>(P, w);
     tmem_wait_st();
     fence_before_sync();
-    if (named_bar_or(w.bar_id, 128, w.fail)) {
+    if (named_bar_or(w.bar_id, w.bar_count, w.fail)) {
       w.fail = true;
       return false;
     }
-    if (w.rho < 32) {
+    if (w.wg_lead) {
       fence_after_sync();
       issue_stage<R, PREC>(w.slot, w.img_addr + img_off, w.bar_mma);
     }
@@ -669,15 +687,15 @@ __device__ __forceinline__ void process_item_conv(const PRun &P, const float2 *t
   }
   tmem_wait_st();
   fence_before_sync();
-  if (named_bar_or(w.bar_id, 128, w.fail)) {
+  if (named_bar_or(w.bar_id, w.bar_count, w.fail)) {
     w.fail = true;
     return;
   }
-  if (w.rho < 32) {
+  if (w.wg_lead) {
     fence_after_sync();
     issue_stage<R, PREC>(w.slot, w.img_addr, w.bar_mma);
-    mid.issue(w);
   }
+  if (w.team_lead) mid.issue(w);
   if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
   w.ph_mma ^= 1;
   fence_after_sync();
@@ -686,11 +704,11 @@ __device__ __forceinline__ void process_item_conv(const PRun &P, const float2 *t
   conv_turn<G, PREC>(P, item, w);
   tmem_wait_st();
   fence_before_sync();
-  if (named_bar_or(w.bar_id, 128, w.fail)) {
+  if (named_bar_or(w.bar_id, w.bar_count, w.fail)) {
     w.fail = true;
     return;
   }
-  if (w.rho < 32) {
+  if (w.wg_lead) {
     fence_after_sync();
     issue_stage<R, PREC>(w.slot, w.img_addr + INV, w.bar_mma);
   }
@@ -745,23 +763,27 @@ __device__ __forceinline__ void kernel_teardown(uint32_t tbase, const WG &w, boo
   }
 }
 
-template <int R, class SM, int GCOLS>
+template <int R, class SM, int GCOLS, int TW = 1>
 __device__ __forceinline__ void init_wg(WG &w, uint32_t tbase, unsigned char *smem) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int wg = warp >> 2;
+  const int wg = warp >> 2, team = wg / TW, wt = wg % TW;
   uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + SM::OFF_BAR);
-  w.rho = (warp & 3) * 32 + lane;
+  w.rho = (wt * 4 + (warp & 3)) * 32 + lane;
+  w.wg_lead = (warp & 3) == 0;
+  w.team_lead = w.wg_lead && wt == 0;
   w.slot = tbase + wg * GCOLS;
   w.lane_off = (uint32_t)((warp & 3) * 32) << 16;
   w.img_addr = smem_u32(smem);
   w.bar_mma = smem_u32(mbar + 3 * wg);
-  w.bar_stg = smem_u32(mbar + 3 * wg + 1);
-  w.bar_tws = smem_u32(mbar + 3 * wg + 2);
-  w.bar_id = 1 + wg;
-  w.buf = reinterpret_cast<float2 *>(smem + SM::OFF_BUF) + wg * SM::PTS;
-  w.stg = reinterpret_cast<float2 *>(smem + SM::OFF_STG) + wg * SM::PTS;
-  w.tws = reinterpret_cast<float2 *>(smem + SM::OFF_TWS) + (SM::TWS_BYTES ? wg * SM::PTS : 0);
-  w.twb = reinterpret_cast<float2 *>(smem + SM::OFF_TWB) + wg * SM::TWB_PER_WG;
+  // the team's copies complete on its first warpgroup's staging barriers
+  w.bar_stg = smem_u32(mbar + 3 * (team * TW) + 1);
+  w.bar_tws = smem_u32(mbar + 3 * (team * TW) + 2);
+  w.bar_id = 1 + team;
+  w.bar_count = 128 * TW;
+  w.buf = reinterpret_cast<float2 *>(smem + SM::OFF_BUF) + team * SM::PTS;
+  w.stg = reinterpret_cast<float2 *>(smem + SM::OFF_STG) + team * SM::PTS;
+  w.tws = reinterpret_cast<float2 *>(smem + SM::OFF_TWS) + (SM::TWS_BYTES ? team * SM::PTS : 0);
+  w.twb = reinterpret_cast<float2 *>(smem + SM::OFF_TWB) + team * SM::TWB_PER_WG;
   w.ph_mma = w.ph_stg = w.ph_tws = 0;
   w.fail = false;
   w.tws_inflight = false;
@@ -781,12 +803,14 @@ struct StaticNext {
   __device__ void publish() {}
 };
 
-template <int R, int PREC, int S, int LO, int ROLE, int LP, bool CONV = false>
-__global__ void __launch_bounds__(Geo<R, S, LO, ROLE, LP>::THREADS, 1)
+template <int R, int PREC, int S, int LO, int ROLE, int LP, bool CONV = false, int TW = 1>
+__global__ void __launch_bounds__(
+    Geo<R, S, LO, ROLE, LP, TW == 1 ? pass_nwg(R, ROLE) : 4, TW>::THREADS, 1)
     dft_pass_kernel(const __grid_constant__ GArgs a) {
-  using G = Geo<R, S, LO, ROLE, LP>;
+  using G = Geo<R, S, LO, ROLE, LP, TW == 1 ? pass_nwg(R, ROLE) : 4, TW>;
   static_assert(!CONV || ROLE == kSingle, "convolution rows are whole transforms");
-  using SM = SmemLayout<R, G::NWG, G::TW_ENTRIES, CONV ? G::TW_ENTRIES : 0, G::TW_SMEM, G::TWB>;
+  using SM = SmemLayout<R, G::NWG, G::TW_ENTRIES, CONV ? G::TW_ENTRIES : 0, G::TW_SMEM, G::TWB,
+                        TW>;
   extern __shared__ __align__(1024) unsigned char smem[];
   float2 *tw = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
   float2 *tw_inv = reinterpret_cast<float2 *>(smem + SM::OFF_TW2);
@@ -798,14 +822,14 @@ __global__ void __launch_bounds__(Geo<R, S, LO, ROLE, LP>::THREADS, 1)
       a.bimg, (int)(SM::IMG / 4), reinterpret_cast<float *>(smem), P.tw_stage, tw,
       G::TW_ENTRIES, a.p[1].tw_stage, tw_inv, CONV ? G::TW_ENTRIES : 0, mbar, tmem_slot);
   WG w;
-  init_wg<R, SM, G::GCOLS>(w, tbase, smem);
+  init_wg<R, SM, G::GCOLS, TW>(w, tbase, smem);
 
-  const int wg = threadIdx.x >> 7;
+  const int team = (threadIdx.x >> 7) / TW;
   const long long nitems = (P.U + G::GG - 1) >> G::LOG2GG;
-  const long long istride = (long long)gridDim.x * G::NWG;
-  long long item = (long long)blockIdx.x * G::NWG + wg;
+  const long long istride = (long long)gridDim.x * G::NTEAM;
+  long long item = (long long)blockIdx.x * G::NTEAM + team;
   StaticNext<G> nx{P, &a.tm_in, item, nitems, false};
-  if (w.rho < 32 && item < nitems) issue_input<G>(P, &a.tm_in, item, w);
+  if (w.team_lead && item < nitems) issue_input<G>(P, &a.tm_in, item, w);
   while (item < nitems && !w.fail) {
     nx.next = item + istride;
     if constexpr (CONV)
@@ -1029,7 +1053,7 @@ __global__ void __launch_bounds__(Geo<R, S1, log2_radix(R) * S2, kFirst>::THREAD
   // first item: claim it, wait for its dependencies, issue its copy; claim
   // the one after and start reading its dependency (warp 0)
   bool f = false;
-  if (w.rho < 32) {
+  if (w.team_lead) {
     const QItem first = nx.decode(__shfl_sync(0xffffffffu, nx.claim(), 0));
     if (first.valid) {
       if (!nx.wait_deps(first)) f = true;
@@ -1044,7 +1068,7 @@ __global__ void __launch_bounds__(Geo<R, S1, log2_radix(R) * S2, kFirst>::THREAD
     nx.n1 = nx.decode(__shfl_sync(0xffffffffu, nx.claim(), 0));
     nx.read_dep(nx.n1);
   }
-  if (named_bar_or(w.bar_id, 128, f)) w.fail = true;
+  if (named_bar_or(w.bar_id, w.bar_count, f)) w.fail = true;
 
   bool stg_pending = false;
   while (!w.fail) {
@@ -1056,14 +1080,14 @@ __global__ void __launch_bounds__(Geo<R, S1, log2_radix(R) * S2, kFirst>::THREAD
       // its dependency was not ready at issue time: publish our own last
       // completion (it may be what it waits for; the barrier orders every
       // thread's stores of it first), wait, then copy
-      bool ff = named_bar_or(w.bar_id, 128, false);
-      if (w.rho < 32) {
+      bool ff = named_bar_or(w.bar_id, w.bar_count, false);
+      if (w.team_lead) {
         nx.publish_pending();
         const QItem q{item, pass, chunk, true};
         if (!nx.wait_deps(q)) ff = true;
         else nx.issue_copy(q, w);
       }
-      if (named_bar_or(w.bar_id, 128, ff)) {
+      if (named_bar_or(w.bar_id, w.bar_count, ff)) {
         w.fail = true;
         break;
       }
@@ -1076,13 +1100,13 @@ __global__ void __launch_bounds__(Geo<R, S1, log2_radix(R) * S2, kFirst>::THREAD
     if (w.fail) break;
     // the mailbox now names the next item; its completion is published
     // during the next item (after its first barrier), or below
-    if (w.rho < 32)
+    if (w.team_lead)
       nx.pend_flag = (pass == 0) ? a.counters + 1 + ((item << G1::LOG2GG) >> G1::LOG2UPER)
                                  : a.counters + 1 + a.batch + chunk;
   }
   // all stores of this warpgroup are issued: publish the last completion
-  named_bar_or(w.bar_id, 128, false);
-  if (w.rho < 32) nx.publish_pending();
+  named_bar_or(w.bar_id, w.bar_count, false);
+  if (w.team_lead) nx.publish_pending();
   if (w.rho == 0 && w.fail) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);
   kernel_teardown(tbase, w, w.fail && stg_pending, w.fail && w.tws_inflight);
 }

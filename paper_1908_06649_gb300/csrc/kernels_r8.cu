@@ -36,6 +36,21 @@ cudaError_t launch_pass_r8(int prec, int s, int lo, int role, int lp, const GArg
   return cudaErrorInvalidValue;
 }
 
+// Team passes (items of tw warpgroups) for the 3-stage radix-8 passes of
+// two-pass transforms: 8^5 = 2 + 3, 8^6 = 3 + 3.
+cudaError_t launch_team_r8(int prec, int s, int lo, int role, int lp, int tw, const GArgs &a,
+                           int num_sms, cudaStream_t st) {
+  constexpr int R = 8;
+  TCU_PASS_CASE(2, 3, kFirst, 0)   // 8^5: the 2-stage strided pass (one warpgroup)
+  TCU_TEAM_CASE(3, 2, kSecond, 0, 2)
+  TCU_TEAM_CASE(3, 2, kSecond, 0, 4)
+  TCU_TEAM_CASE(3, 3, kFirst, 0, 2)  // 8^6
+  TCU_TEAM_CASE(3, 3, kFirst, 0, 4)
+  TCU_TEAM_CASE(3, 3, kSecond, 0, 2)
+  TCU_TEAM_CASE(3, 3, kSecond, 0, 4)
+  return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_fused_r8(int prec, int s1, int s2, const GArgs &a, int num_sms,
                             cudaStream_t st) {
   constexpr int R = 8;

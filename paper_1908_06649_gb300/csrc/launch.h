@@ -22,6 +22,9 @@ cudaError_t launch_pass_r32(int prec, int s, int lo, int role, int lp, const GAr
 cudaError_t launch_rowconv_r8(int prec, int s, const GArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_rowconv_r16(int prec, int s, const GArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_rowconv_r32(int prec, int s, const GArgs &a, int num_sms, cudaStream_t st);
+// Radix-8 passes whose items are teams of tw warpgroups (kernels_r8.cu).
+cudaError_t launch_team_r8(int prec, int s, int lo, int role, int lp, int tw, const GArgs &a,
+                           int num_sms, cudaStream_t st);
 // Both passes of a two-pass transform fused in one launch (s1, s2 >= 2).
 cudaError_t launch_fused_r8(int prec, int s1, int s2, const GArgs &a, int num_sms,
                             cudaStream_t st);

@@ -20,6 +20,31 @@ cudaError_t launch_pass_t(const GArgs &a, int num_sms, cudaStream_t st) {
   return cudaGetLastError();
 }
 
+// A team pass: items of TW warpgroups (128 TW rows), four warpgroups a CTA.
+template <int R, int PREC, int S, int LO, int ROLE, int LP, int TW>
+cudaError_t launch_team_t(const GArgs &a, int num_sms, cudaStream_t st) {
+  using G = Geo<R, S, LO, ROLE, LP, 4, TW>;
+  const size_t sm = SmemLayout<R, 4, G::TW_ENTRIES, 0, G::TW_SMEM, G::TWB, TW>::BYTES;
+  cudaError_t e = cudaFuncSetAttribute(dft_pass_kernel<R, PREC, S, LO, ROLE, LP, false, TW>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       (int)sm);
+  if (e != cudaSuccess) return e;
+  const long long nitems = (a.p[0].U + G::GG - 1) >> G::LOG2GG;
+  long long grid = (nitems + G::NTEAM - 1) / G::NTEAM;
+  if (grid > num_sms) grid = num_sms;
+  dft_pass_kernel<R, PREC, S, LO, ROLE, LP, false, TW>
+      <<<(unsigned)grid, G::THREADS, sm, st>>>(a);
+  return cudaGetLastError();
+}
+
+#define TCU_TEAM_CASE(S, SO, ROLE, SP, TW)                                               \
+  if (s == S && lo == log2_radix(R) * (SO) && role == ROLE && lp == log2_radix(R) * (SP) && \
+      tw == TW)                                                                           \
+    return prec == 3 ? launch_team_t<R, 3, S, log2_radix(R) * (SO), ROLE,               \
+                                     log2_radix(R) * (SP), TW>(a, num_sms, st)           \
+                     : launch_team_t<R, 1, S, log2_radix(R) * (SO), ROLE,               \
+                                     log2_radix(R) * (SP), TW>(a, num_sms, st);
+
 // The convolution row pass (forward rows, spectrum product, inverse rows).
 template <int R, int PREC, int S>
 cudaError_t launch_rowconv_t(const GArgs &a, int num_sms, cudaStream_t st) {

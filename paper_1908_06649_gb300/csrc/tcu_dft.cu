@@ -75,6 +75,7 @@ struct PassPlan {
   int q;
   RootsQ roots[2];
   bool mixed;
+  int tw;           // warpgroups per item (teams for the 3-stage radix-8 passes)
 };
 
 thread_local int g_last_error = TCU_DFT_OK;
@@ -250,17 +251,17 @@ int stage_mode(const int modes[3], int t, int S) {
 // Shared-memory wavefronts per warp-wide 8-byte access of the warpgroup
 // kernel's transposes (1.0 = conflict free), for swizzle table `tab`:
 // phys(P) = P ^ ((tab[ul & 15] ^ (P >> 4)) & 15).
-double swizzle_cost(int r, int S, const int modes[3], unsigned long long tab) {
+double swizzle_cost(int r, int S, const int modes[3], unsigned long long tab, int team) {
   const int log2r = ilog2(r);
   const int L = 1 << (log2r * S);
-  const int rps = L / r, gg = 128 * r / L;
+  const int rps = L / r, gg = 128 * team * r / L;
   long long waves = 0, accesses = 0;
   for (int t = 1; t < S; ++t) {
     for (int side = 0; side < 2; ++side) {  // epilogue write of t, read of t+1
       const int tt = t + side;
       const int mode = stage_mode(modes, tt, S);
       const int sl = log2r * (S - tt);
-      for (int w = 0; w < 4; ++w)
+      for (int w = 0; w < 4 * team; ++w)
         for (int j = 0; j < r; ++j)
           for (int h = 0; h < 2; ++h) {
             int seen = 0, count = 0;
@@ -300,7 +301,7 @@ double swizzle_cost(int r, int S, const int modes[3], unsigned long long tab) {
   return accesses ? (double)waves / (double)accesses : 1.0;
 }
 
-unsigned long long choose_swizzle(int r, int S, const int modes[3]) {
+unsigned long long choose_swizzle(int r, int S, const int modes[3], int team) {
   std::vector<unsigned long long> cands;
   for (int c = 0; c < 4; ++c) {
     unsigned long long t = 0;
@@ -317,7 +318,7 @@ unsigned long long choose_swizzle(int r, int S, const int modes[3]) {
   unsigned long long best = cands[0];
   double bc = 1e30;
   for (unsigned long long t : cands) {
-    const double c = swizzle_cost(r, S, modes, t);
+    const double c = swizzle_cost(r, S, modes, t, team);
     if (c < bc - 1e-9) {
       bc = c;
       best = t;
@@ -349,6 +350,13 @@ int plan_stages(int r, int k, int st[kMaxPasses]) {
   if (k <= sg) {
     st[0] = k;
     return 1;
+  }
+  if (r == 8 && k <= 6) {
+    // two passes of 2 + 3 or 3 + 3: the 3-stage passes run on teams of
+    // warpgroups (team_size), whose items span 8 adjacent columns
+    st[0] = k / 2;
+    st[1] = k - st[0];
+    return 2;
   }
   int P = (k + 1) / 2;
   if (P > kMaxPasses) P = kMaxPasses;
@@ -408,9 +416,17 @@ int plan_mixed(int r, long long n, long long batch, PassPlan pass[kMaxPasses]) {
     pp.modes[0] = pp.role == kFirst ? kUF : kQF;
     pp.modes[1] = kUF;
     pp.modes[2] = kUF;
-    pp.swz_tab = choose_swizzle(r, pp.s, pp.modes);
+    pp.tw = 1;
+    pp.swz_tab = choose_swizzle(r, pp.s, pp.modes, 1);
   }
   return 1 + tc;
+}
+
+// Warpgroups per item of pass pp: 4 for the 3-stage radix-8 passes of
+// two-pass transforms (an item of 512 rows holds 8 sub-transforms of 512
+// points, so the strided side moves 64-byte runs), else 1.
+int team_size(int r, int npasses, const PassPlan &pp) {
+  return (r == 8 && npasses == 2 && pp.s == 3 && pp.role != kCols) ? 4 : 1;
 }
 
 // Role, neighbouring stage counts, size and row maps of pass `pi`.
@@ -439,7 +455,8 @@ void pass_geometry(PassPlan &pp, int pi, int P, const int st[kMaxPasses], int k,
   pp.modes[0] = pp.role == kFirst ? kUF : kQF;
   pp.modes[1] = kUF;
   pp.modes[2] = pp.role == kSingle ? kRQF : kUF;
-  pp.swz_tab = choose_swizzle(r, pp.s, pp.modes);
+  pp.tw = team_size(r, P, pp);
+  pp.swz_tab = choose_swizzle(r, pp.s, pp.modes, pp.tw);
 }
 
 // Inter-pass twiddles of a strided pass: w_M^{k v}, k < L, v < n2, M = L n2;
@@ -463,7 +480,7 @@ void pass_twiddles(long long L, long long n2, int sign, std::vector<float2> &A,
 bool twiddle_map(CUtensorMap *m, const float2 *A, int r, const PassPlan &pp) {
   const long long L = 1ll << pp.log2L, n2 = 1ll << pp.lo;
   const long long VL = n2 > 256 ? 256 : n2;
-  const long long gg = (128ll * r) >> pp.log2L;
+  const long long gg = (128ll * pp.tw * r) >> pp.log2L;
   return encode_map(m, A, VL, L, 1, L * VL, (int)gg, L < 256 ? (int)L : 256);
 }
 
@@ -472,7 +489,7 @@ bool twiddle_map(CUtensorMap *m, const float2 *A, int r, const PassPlan &pp) {
 bool input_map(CUtensorMap *m, const void *in, const tcu_dft_plan_s *p, const PassPlan &pp,
                long long batch) {
   const long long L = 1ll << pp.log2L, n2 = 1ll << pp.lo, pre = 1ll << pp.lp;
-  const long long gg = (128ll * p->r) >> pp.log2L;
+  const long long gg = (128ll * pp.tw * p->r) >> pp.log2L;
   return encode_map(m, in, n2, L, batch * pre, L * n2, (int)gg, L < 256 ? (int)L : 256);
 }
 
@@ -505,13 +522,15 @@ void free_plan(tcu_dft_plan_s *p) {
 
 // ---------------------------------------------------------------- launches
 cudaError_t pass_dispatch(int r, int prec, const PassPlan &pp, const GArgs &a, int num_sms,
-                          cudaStream_t st) {
+                          cudaStream_t st, bool team_plan = false) {
   if (pp.mixed) {
     if (r == 8) return launch_pass_mixed_r8(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
     if (r == 16) return launch_pass_mixed_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
     return launch_pass_mixed_r32(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   }
   if (prec_bf16(prec)) return launch_pass_bf16_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
+  if (r == 8 && team_plan)
+    return launch_team_r8(prec, pp.s, pp.lo, pp.role, pp.lp, pp.tw, a, num_sms, st);
   if (r == 8) return launch_pass_r8(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   if (r == 16) return launch_pass_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   return launch_pass_r32(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
@@ -704,8 +723,9 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
   }
   if (rc == TCU_DFT_OK && npasses >= 2) {
     const PassPlan &p1 = p->pass[0], &p2 = p->pass[1];
-    p->fused = !is_mixed && !prec_bf16(precision) && npasses == 2 && p1.s >= 2 &&
-               p2.s >= 2 && (flags & TCU_DFT_PLAN_FUSE);
+    // fused kernels are instantiated for 2 + 2 stages
+    p->fused = !is_mixed && !prec_bf16(precision) && npasses == 2 && p1.s == 2 &&
+               p2.s == 2 && (flags & TCU_DFT_PLAN_FUSE);
     long long scratch_tf = batch;
     if (p->fused) {
       // chunks of C transforms (a power of two dividing the batch, <= 8);
@@ -841,7 +861,8 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
     }
     g.bimg = p->bimg[di];
     g.err = p->err;
-    if (pass_dispatch(p->r, p->precision, pp, g, p->num_sms, st) != cudaSuccess)
+    const bool team_plan = p->npasses == 2 && (p->pass[0].tw > 1 || p->pass[1].tw > 1);
+    if (pass_dispatch(p->r, p->precision, pp, g, p->num_sms, st, team_plan) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
   }
   if (events && cudaEventRecord((cudaEvent_t)events[p->npasses], st) != cudaSuccess)
@@ -1220,7 +1241,8 @@ tcu_dft2_plan_s *make_dft2(int64_t n1, int64_t n2, int64_t batch, int32_t r,
   c.log2L = log2r * k1;
   c.U = batch * n2;
   c.modes[0] = c.modes[1] = c.modes[2] = kUF;
-  c.swz_tab = choose_swizzle(r, c.s, c.modes);
+  c.tw = 1;
+  c.swz_tab = choose_swizzle(r, c.s, c.modes, 1);
   w.s = k2;
   w.role = kSingle;
   w.so = w.sp = w.lo = w.lp = 0;
@@ -1229,7 +1251,8 @@ tcu_dft2_plan_s *make_dft2(int64_t n1, int64_t n2, int64_t batch, int32_t r,
   w.modes[0] = kQF;
   w.modes[1] = kUF;
   w.modes[2] = kRQF;
-  w.swz_tab = choose_swizzle(r, w.s, w.modes);
+  w.tw = 1;
+  w.swz_tab = choose_swizzle(r, w.s, w.modes, 1);
   std::vector<float> conv_img;
   for (int d = 0; d < 2 && rc == TCU_DFT_OK; ++d) {
     const int sign = d == 0 ? -1 : 1;

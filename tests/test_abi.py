@@ -114,7 +114,7 @@ def test_python_plan_raises(lib):
     ((256, 1, 12, 3, -1), 2),          # radix
     ((48, 1, 16, 3, -1), 2),           # not a power of the radix
     ((16 ** 5, 1, 16, 3, -1), 6),      # three passes
-    ((8 ** 5, 1, 8, 3, -1), 6),
+    ((8 ** 7, 1, 8, 3, -1), 6),
     ((32 ** 4, 1, 32, 3, -1), 6),      # n beyond the fixed twiddle table
     ((65536, 65, 16, 3, -1), 6),       # batch*n beyond the fixed intermediate
 ])

@@ -80,8 +80,8 @@ def test_single_pass(pkg, r, k, prec):
 @pytest.mark.parametrize("r,k,batch,stages", [
     (16, 3, 7, [1, 2]), (16, 4, 5, [2, 2]), (16, 4, 40, [2, 2]), (8, 4, 6, [2, 2]),
     (32, 3, 3, [1, 2]), (32, 4, 1, [2, 2]),
-    (16, 5, 2, [1, 2, 2]), (16, 6, 1, [2, 2, 2]), (8, 5, 3, [1, 2, 2]),
-    (8, 6, 2, [2, 2, 2]), (8, 7, 1, [2, 2, 3]), (8, 8, 1, [2, 3, 3]),
+    (16, 5, 2, [1, 2, 2]), (16, 6, 1, [2, 2, 2]), (8, 5, 3, [2, 3]),
+    (8, 6, 2, [3, 3]), (8, 5, 41, [2, 3]), (8, 7, 1, [2, 2, 3]), (8, 8, 1, [2, 3, 3]),
     (32, 5, 1, [1, 2, 2])])
 @pytest.mark.parametrize("prec", [3, 1])
 def test_multi_pass(pkg, r, k, batch, stages, prec):
