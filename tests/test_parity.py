@@ -361,3 +361,28 @@ def test_exec_host_pipelined(pkg, n, batch, r):
     plan.check()
     check(h_out.numpy().reshape(batch, n), x, 3, inverse=True)
     plan.destroy()
+
+
+@pytest.mark.parametrize("n,batch,r", [(4096, 64, 16), (8 ** 5, 6, 8), (16 ** 5, 2, 16)])
+def test_exec_captures_into_a_cuda_graph(pkg, n, batch, r):
+    # exec allocates nothing and synchronises nothing, so it can be captured
+    # once into a CUDA graph and replayed
+    import torch
+    x = torch.from_numpy(inputs.make("uniform", n, batch, seed=80)).cuda()
+    y = torch.empty_like(x)
+    plan = pkg.Plan(n, batch, r, 3)
+    s = torch.cuda.Stream()
+    with torch.cuda.stream(s):
+        plan.forward(x, y)
+    torch.cuda.synchronize()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        plan.forward(x, y)
+    y.zero_()
+    torch.cuda.synchronize()
+    for _ in range(2):
+        g.replay()
+    torch.cuda.synchronize()
+    plan.check()
+    check(y.cpu().numpy().reshape(batch, n), x.cpu().numpy().reshape(batch, n), 3)
+    plan.destroy()
