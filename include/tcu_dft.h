@@ -143,6 +143,13 @@ int tcu_dft_check(tcu_dft_plan_t p, void *stream);
  * Destroying NULL is a no-op returning OK. */
 int tcu_dft_destroy(tcu_dft_plan_t p);
 
+/* The pass grouping tcu_dft_plan would choose for n and sqrt_m, without
+ * creating a plan or touching the GPU: returns the number of HBM passes (0
+ * if n is not supported) and writes the stages of each pass to stages[0 ..
+ * passes) (caller array of 3; the q-point pass of a mixed-radix n counts
+ * as one stage). */
+int tcu_dft_plan_passes(int64_t n, int32_t sqrt_m, int32_t *stages);
+
 /* Plan introspection: number of HBM passes, and stages in pass i (0-based);
  * -1 for a NULL plan or an index out of range. */
 int tcu_dft_num_passes(tcu_dft_plan_t p);

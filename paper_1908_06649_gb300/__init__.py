@@ -41,7 +41,8 @@ SYMBOLS = (
     "tcu_dft_exec_dir", "tcu_dft_exec_timed",
     "tcu_dft_exec_host", "tcu_dft_exec_noalloc", "tcu_dft_exec_stalled",
     "tcu_dft_check", "tcu_dft_destroy", "tcu_dft_num_passes",
-    "tcu_dft_pass_stages", "tcu_dft_last_error", "tcu_dft_strerror",
+    "tcu_dft_pass_stages", "tcu_dft_plan_passes", "tcu_dft_last_error",
+    "tcu_dft_strerror",
     "tcu_dft2_plan", "tcu_dft2_exec", "tcu_conv2_exec", "tcu_dft2_check",
     "tcu_dft2_destroy", "tcu_stencil_plan", "tcu_stencil_weights",
     "tcu_stencil_exec", "tcu_stencil_check", "tcu_stencil_destroy",
@@ -98,6 +99,8 @@ def lib():
     L.tcu_dft_destroy.restype = ctypes.c_int
     L.tcu_dft_num_passes.argtypes = [vp]
     L.tcu_dft_num_passes.restype = ctypes.c_int
+    L.tcu_dft_plan_passes.argtypes = [i64, i32, ctypes.POINTER(ctypes.c_int32)]
+    L.tcu_dft_plan_passes.restype = ctypes.c_int
     L.tcu_dft_pass_stages.argtypes = [vp, ctypes.c_int]
     L.tcu_dft_pass_stages.restype = ctypes.c_int
     L.tcu_dft_last_error.argtypes = []
@@ -125,6 +128,14 @@ def lib():
         getattr(L, nm).restype = ctypes.c_int
     _lib = L
     return L
+
+
+def plan_passes(n: int, sqrt_m: int = 16):
+    """Stages per HBM pass that a plan for (n, sqrt_m) would use ([] if n is
+    not supported); no GPU needed."""
+    st = (ctypes.c_int32 * 3)()
+    np_ = lib().tcu_dft_plan_passes(int(n), int(sqrt_m), st)
+    return [int(st[i]) for i in range(np_)]
 
 
 def strerror(status: int) -> str:

@@ -968,6 +968,29 @@ int tcu_dft_destroy(tcu_dft_plan_t p) {
   return TCU_DFT_OK;
 }
 
+int tcu_dft_plan_passes(int64_t n, int32_t sqrt_m, int32_t *stages) {
+  if (n < 1 || !stages || (sqrt_m != 8 && sqrt_m != 16 && sqrt_m != 32)) return 0;
+  const int r = sqrt_m;
+  int k = 0;
+  long long m = 1;
+  while (m < n) {
+    m *= r;
+    ++k;
+  }
+  int st[kMaxPasses] = {0, 0, 0};
+  int np = 0;
+  if (m == n) {
+    np = k >= 1 ? plan_stages(r, k, st) : 0;
+  } else {
+    PassPlan mixed[kMaxPasses];
+    memset(mixed, 0, sizeof(mixed));
+    np = plan_mixed(r, n, 1, mixed);
+    for (int i = 0; i < np; ++i) st[i] = mixed[i].s;
+  }
+  for (int i = 0; i < np; ++i) stages[i] = st[i];
+  return np;
+}
+
 int tcu_dft_num_passes(tcu_dft_plan_t p) { return p ? p->npasses : -1; }
 
 int tcu_dft_is_fused(tcu_dft_plan_t p) { return p ? (p->fused ? 1 : 0) : -1; }

@@ -164,3 +164,22 @@ def test_grid_null_handling(lib):
     assert lib.tcu_conv2_exec(None, None, None, None, None) == pkg.ERR_INVALID
     assert lib.tcu_stencil_exec(None, None, None, None, None) == pkg.ERR_INVALID
     assert lib.tcu_dft2_check(None, None) == pkg.ERR_INVALID
+
+
+@pytest.mark.parametrize("n,r,stages", [
+    (16, 16, [1]), (256, 16, [2]), (4096, 16, [1, 2]), (65536, 16, [2, 2]),
+    (16 ** 5, 16, [1, 2, 2]), (16 ** 6, 16, [2, 2, 2]), (16 ** 7, 16, []),
+    (8, 8, [1]), (512, 8, [3]), (8 ** 4, 8, [2, 2]), (8 ** 5, 8, [2, 3]), (8 ** 6, 8, [3, 3]),
+    (8 ** 7, 8, [2, 2, 3]), (8 ** 8, 8, [2, 3, 3]), (8 ** 9, 8, [3, 3, 3]), (8 ** 10, 8, []),
+    (32 ** 2, 32, [2]), (32 ** 3, 32, [1, 2]), (32 ** 4, 32, [2, 2]), (32 ** 5, 32, [1, 2, 2]),
+    (32 ** 6, 32, [2, 2, 2]), (32 ** 7, 32, []),
+    # mixed final radix n = q r^k: the q-point pass first
+    (2 * 256, 16, [1, 2]), (8 * 4096, 16, [1, 1, 2]), (4 * 65536, 16, [1, 2, 2]),
+    (2 * 64, 8, [1, 2]), (4 * 512, 8, [1, 3]), (2 * 4096, 8, [1, 2, 2]),
+    (16 * 1024, 32, [1, 2]), (2 * 32 ** 3, 32, [1, 1, 2]),
+    (2 * 16, 16, []), (3 * 256, 16, []), (2 * 16 ** 5, 16, []), (0, 16, [])])
+def test_plan_grouping(n, r, stages):
+    # the documented grouping, computed on the host without a GPU
+    import paper_1908_06649_gb300 as pkg
+    pkg.lib()
+    assert pkg.plan_passes(n, r) == stages
