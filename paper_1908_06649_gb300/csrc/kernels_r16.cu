@@ -9,8 +9,6 @@ cudaError_t launch_pass_r16(int prec, int s, int lo, int role, int lp, const GAr
   constexpr int R = 16;
   TCU_PASS_CASE(1, 0, kSingle, 0)
   TCU_PASS_CASE(2, 0, kSingle, 0)
-  TCU_PASS_CASE(1, 2, kFirst, 0)   // n = 16^3: 1 + 2
-  TCU_PASS_CASE(2, 1, kSecond, 0)
   TCU_PASS_CASE(2, 2, kFirst, 0)   // n = 16^4: 2 + 2
   TCU_PASS_CASE(2, 2, kSecond, 0)
   TCU_PASS_CASE(1, 4, kFirst, 0)   // n = 16^5: 1 + 2 + 2
@@ -22,6 +20,14 @@ cudaError_t launch_pass_r16(int prec, int s, int lo, int role, int lp, const GAr
   TCU_PASS_CASE(1, 2, kCols, 0)   // 2-D DFT column passes: n1 = R^s, n2 = R^so
   TCU_PASS_CASE(2, 1, kCols, 0)
   TCU_PASS_CASE(2, 2, kCols, 0)
+  return cudaErrorInvalidValue;
+}
+
+// Team passes: 16^3 in one pass on items of two warpgroups.
+cudaError_t launch_team_r16(int prec, int s, int lo, int role, int lp, int tw, const GArgs &a,
+                            int num_sms, cudaStream_t st) {
+  constexpr int R = 16;
+  TCU_TEAM_CASE(3, 0, kSingle, 0, 2)
   return cudaErrorInvalidValue;
 }
 

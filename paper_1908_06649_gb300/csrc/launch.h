@@ -25,6 +25,9 @@ cudaError_t launch_rowconv_r32(int prec, int s, const GArgs &a, int num_sms, cud
 // Radix-8 passes whose items are teams of tw warpgroups (kernels_r8.cu).
 cudaError_t launch_team_r8(int prec, int s, int lo, int role, int lp, int tw, const GArgs &a,
                            int num_sms, cudaStream_t st);
+// Radix-16 team passes (kernels_r16.cu).
+cudaError_t launch_team_r16(int prec, int s, int lo, int role, int lp, int tw, const GArgs &a,
+                            int num_sms, cudaStream_t st);
 // Both passes of a two-pass transform fused in one launch (s1, s2 >= 2).
 cudaError_t launch_fused_r8(int prec, int s1, int s2, const GArgs &a, int num_sms,
                             cudaStream_t st);
@@ -57,8 +60,8 @@ cudaError_t launch_radix_q(int q, const float2 *x, float2 *out, long long batch,
                            const float2 *twA, const float2 *twB, const RootsQ &roots,
                            int num_sms, cudaStream_t st);
 // BF16-mode (precision 4, 5) radix-16 passes (kernels_bf16_r16.cu).
-cudaError_t launch_pass_bf16_r16(int prec, int s, int lo, int role, int lp, const GArgs &a,
-                                 int num_sms, cudaStream_t st);
+cudaError_t launch_pass_bf16_r16(int prec, int s, int lo, int role, int lp, int tw,
+                                 const GArgs &a, int num_sms, cudaStream_t st);
 // Mixed-radix warpgroup passes (kernels_mixed_r*.cu): same arguments as
 // launch_pass_r*.
 cudaError_t launch_pass_mixed_r8(int prec, int s, int lo, int role, int lp, const GArgs &a,

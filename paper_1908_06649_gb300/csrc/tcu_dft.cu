@@ -347,7 +347,8 @@ int upload(T **dst, const std::vector<T> &src) {
 // wider TMA rows.  Returns the number of passes, 0 if n is too long.
 int plan_stages(int r, int k, int st[kMaxPasses]) {
   const int sg = r == 8 ? 3 : 2;
-  if (k <= sg) {
+  if (k <= sg || (r == 16 && k == 3)) {
+    // 16^3 in one pass on items of two warpgroups (one 4096-point transform)
     st[0] = k;
     return 1;
   }
@@ -426,6 +427,7 @@ int plan_mixed(int r, long long n, long long batch, PassPlan pass[kMaxPasses]) {
 // two-pass transforms (an item of 512 rows holds 8 sub-transforms of 512
 // points, so the strided side moves 64-byte runs), else 1.
 int team_size(int r, int npasses, const PassPlan &pp) {
+  if (r == 16 && npasses == 1 && pp.s == 3) return 2;
   return (r == 8 && npasses == 2 && pp.s == 3 && pp.role != kCols) ? 4 : 1;
 }
 
@@ -528,9 +530,12 @@ cudaError_t pass_dispatch(int r, int prec, const PassPlan &pp, const GArgs &a, i
     if (r == 16) return launch_pass_mixed_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
     return launch_pass_mixed_r32(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   }
-  if (prec_bf16(prec)) return launch_pass_bf16_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
+  if (prec_bf16(prec))
+    return launch_pass_bf16_r16(prec, pp.s, pp.lo, pp.role, pp.lp, pp.tw, a, num_sms, st);
   if (r == 8 && team_plan)
     return launch_team_r8(prec, pp.s, pp.lo, pp.role, pp.lp, pp.tw, a, num_sms, st);
+  if (r == 16 && pp.tw > 1)
+    return launch_team_r16(prec, pp.s, pp.lo, pp.role, pp.lp, pp.tw, a, num_sms, st);
   if (r == 8) return launch_pass_r8(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   if (r == 16) return launch_pass_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   return launch_pass_r32(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
@@ -592,7 +597,7 @@ void dir_tables(const tcu_dft_plan_s *p, int d, DirTables &t) {
 constexpr long long kNaMaxPoints = 1ll << 22;      // two-pass intermediate
 constexpr long long kNaMaxN = 1ll << 18;           // longest transform
 constexpr int kNaImgFloats = 4 * 16 * 32 * 32 / 4;  // 4 F_r images, r <= 32
-constexpr int kNaStageTw = 1024;                    // stage twiddles of a pass
+constexpr int kNaStageTw = 4608;  // stage twiddles of a pass (16^3 + 16^2 = 4352 for 3 stages)
 static __device__ __align__(256) float2 g_na_scratch[kNaMaxPoints];
 static __device__ __align__(256) float g_na_img[2][kNaImgFloats];
 static __device__ __align__(256) float2 g_na_tw_stage[2][2][kNaStageTw];
@@ -861,7 +866,8 @@ static int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
     }
     g.bimg = p->bimg[di];
     g.err = p->err;
-    const bool team_plan = p->npasses == 2 && (p->pass[0].tw > 1 || p->pass[1].tw > 1);
+    bool team_plan = false;
+    for (int i = 0; i < p->npasses; ++i) team_plan |= p->pass[i].tw > 1;
     if (pass_dispatch(p->r, p->precision, pp, g, p->num_sms, st, team_plan) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
   }
@@ -1074,6 +1080,8 @@ int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t preci
   DirTables t[2];
   for (int d = 0; d < 2; ++d) {
     dir_tables(&p, d, t[d]);
+    for (int pi = 0; pi < npasses; ++pi)
+      if (t[d].stage[pi].size() > (size_t)kNaStageTw) return TCU_DFT_ERR_TOO_LARGE;
     if (npasses == 2) {
       p.pass[0].tw_a[d] = D.tw_out + (size_t)d * kNaMaxN;
       if (!t[d].B[0].empty()) p.pass[0].tw_b[d] = p.pass[0].tw_a[d] + t[d].A[0].size();

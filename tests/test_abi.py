@@ -167,7 +167,7 @@ def test_grid_null_handling(lib):
 
 
 @pytest.mark.parametrize("n,r,stages", [
-    (16, 16, [1]), (256, 16, [2]), (4096, 16, [1, 2]), (65536, 16, [2, 2]),
+    (16, 16, [1]), (256, 16, [2]), (4096, 16, [3]), (65536, 16, [2, 2]),
     (16 ** 5, 16, [1, 2, 2]), (16 ** 6, 16, [2, 2, 2]), (16 ** 7, 16, []),
     (8, 8, [1]), (512, 8, [3]), (8 ** 4, 8, [2, 2]), (8 ** 5, 8, [2, 3]), (8 ** 6, 8, [3, 3]),
     (8 ** 7, 8, [2, 2, 3]), (8 ** 8, 8, [2, 3, 3]), (8 ** 9, 8, [3, 3, 3]), (8 ** 10, 8, []),
