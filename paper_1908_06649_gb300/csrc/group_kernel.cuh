@@ -1,31 +1,36 @@
 // group_kernel.cuh -- warpgroup kernels for passes whose sub-transforms fit
-// in 128 data rows (L = r^S <= 128 r).
+// in one item of 128 TW data rows (L = r^S <= 128 TW r, TW = 1, 2 or 4
+// warpgroups per item).
 //
-// A CTA (one per SM, persistent) holds NWG independent warpgroups.  A
-// warpgroup owns one TMEM slot (A_hi | A_lo | D for 128 rows), SMEM staging
-// and transpose buffers and its mbarriers, and processes work items; an item
-// is GG = 128 r / L consecutive sub-transforms, i.e. exactly 128 data rows per
-// stage, so every stage of an item is ONE M=128 tall-left tcgen05 product
-// with F_r (the (m,l)-TCU call of Sec. 3 / Theorem 7) and the transposition
-// between stages stays inside the warpgroup.
+// A CTA (one per SM, persistent) holds NWG warpgroups grouped into teams of
+// TW.  A warpgroup owns one TMEM slot (A_hi | A_lo | D for its 128 rows) and
+// its product mbarrier; a team owns SMEM staging and transpose buffers, the
+// staging mbarriers and one named barrier, and processes work items; an item
+// is GG = 128 TW r / L consecutive sub-transforms, i.e. exactly 128 TW data
+// rows per stage, so every stage of an item is one M=128 tall-left tcgen05
+// product with F_r per warpgroup (the (m,l)-TCU call of Sec. 3 / Theorem 7)
+// and the transposition between stages stays inside the team.
 //
 // Per item: the item's input block arrives in SMEM by TMA (a 1-D bulk copy
-// when it is contiguous, a 3-D tensor box for the strided first pass of a
-// four-step split), issued by one thread a whole item ahead; every thread
-// reads its stage-1 row from there, splits it into TF32 hi/lo parts and
-// stores them into TMEM as the A operand; one thread issues the products; the
+// when it is contiguous, a 3-D tensor box for a strided pass), issued by an
+// elected lane of the team's first warp a whole item ahead; every thread
+// reads its stage-1 row from there, splits it into hi/lo parts (TF32, or
+// BF16 packed two per column) and stores them into TMEM as the A operand;
+// an elected lane of each warpgroup's first warp issues its products; the
 // epilogue reads D from TMEM, multiplies by the stage twiddles w_L^{k_t c_t}
 // and writes the transposed rows of the next stage to SMEM; the last stage's
 // outputs go straight from registers to global memory in natural order, with
-// the inter-pass twiddle w_n^{b k} of the four-step split (also staged by
-// TMA) applied on the way.  The inverse's 1/n is folded, exactly, into a
-// 2^-log2(n)-scaled copy of F_r used by the last stage.
+// the inter-pass twiddle w_M^{k v} of a strided pass (staged by TMA from two
+// small tables) applied on the way.  The inverse's 1/n is folded, exactly,
+// into a 2^-log2(n)-scaled copy of F_r used by the last stage.
 //
-// The whole geometry of a pass (radix, stage counts of both passes, role) is
-// a template parameter, so every stride is a compile-time constant.
+// The whole geometry of a pass (radix, stages, other-side size, role, prefix,
+// team) is a template parameter, so every stride is a compile-time constant.
 //
-// Two kernels share the item routine:
-//   dft_pass_kernel   -- one pass, items assigned round-robin;
+// Kernels sharing the item routines:
+//   dft_pass_kernel   -- one pass, items assigned round-robin; with CONV, the
+//     row pass of a circular 2-D convolution (forward stages, spectrum
+//     product, inverse stages of every row, on chip);
 //   dft_fused_kernel  -- both passes of a two-pass (four-step) transform in
 //     ONE launch: a work queue interleaves the passes by chunks of C
 //     transforms, pass-1 items write their output to a small ring of chunks

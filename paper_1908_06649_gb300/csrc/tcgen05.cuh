@@ -1,6 +1,7 @@
 // tcgen05.cuh -- inline-PTX building blocks for sm_103a: shared-memory and
 // tensor-memory addressing, mbarriers with bounded waits, TMEM allocation,
-// tcgen05.mma (kind::tf32, A in tensor memory), tcgen05.ld/st, descriptors.
+// tcgen05.mma (kind::tf32 and kind::f16, A in tensor memory), tcgen05.ld/st,
+// descriptors, elected-lane issue.
 #pragma once
 #include <cuda_runtime.h>
 #include <stdint.h>
