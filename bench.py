@@ -206,11 +206,21 @@ def cpu_baseline(wl, seconds=10.0, sample=32):
         el = time.perf_counter() - t0
         if el >= seconds:
             break
+    # one core on a 1/64 subset of the sample, scaled to the same unit
+    x1 = x[:max(1, sample // 64)]
+    done1, t1 = 0, time.perf_counter()
+    while time.perf_counter() - t1 < min(3.0, seconds / 3):
+        oracle.fft_radix2_timed(x1, threads=1)
+        done1 += x1.shape[0]
+    el1 = time.perf_counter() - t1
     return {"value": dft_flops(n, done) / el / 1e9, "unit": UNIT,
             "cores": used, "kind": "oracle",
             "sample": "%d transforms (first %d of the workload, repeated) of "
                       "n=%d through the fp64 recursive radix-2 FFT, %.1f s "
-                      "wall" % (done, sample, n, el)}
+                      "wall" % (done, sample, n, el),
+            "one_core": {"value": dft_flops(n, done1) / el1 / 1e9, "unit": UNIT,
+                         "sample": "%d transforms of n=%d on 1 core, %.1f s"
+                                   % (done1, n, el1)}}
 
 
 def run_reference(args, wl):
