@@ -11,12 +11,13 @@ import subprocess
 
 HERE = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(HERE, "csrc")
-UNITS = ["tcu_dft.cu", "kernels_r8.cu", "kernels_r16.cu", "kernels_r32.cu",
+UNITS = ["tcu_dft.cu", "host_tables.cu", "noalloc.cu", "grid_plan.cu",
+         "kernels_r8.cu", "kernels_r16.cu", "kernels_r32.cu",
          "kernels_mixed_r8.cu", "kernels_mixed_r16.cu", "kernels_mixed_r32.cu",
          "kernels_bf16_r16.cu",
          "grid_kernels.cu"]
 HEADERS = ["tcgen05.cuh", "group_kernel.cuh", "launch.h",
-           "launch_impl.cuh"]
+           "launch_impl.cuh", "host_plan.h"]
 HDR = os.path.join(os.path.dirname(HERE), "include", "tcu_dft.h")
 LIB_PATH = os.path.join(HERE, "libtcu_dft.so")
 BUILD_DIR = os.path.join(HERE, "_build")
