@@ -237,8 +237,17 @@ __device__ __forceinline__ void row_of(int mode, int rho, int &ul, int &q) {
   }
 }
 
+// Swizzle of the transpose buffer: the 8-byte slot (p mod 16) of index p is
+// XORed with the table value of its sub-transform column and with bits 4-7
+// of p; for sub-transforms longer than 256 points (WIDE) also with bits
+// 8-11, where the leading digit of a 16^3 or 8^3 row lives.  A bijection on
+// every 16-entry block; the host picks the table by a bank-conflict cost
+// model of the same function.
+template <bool WIDE>
 __device__ __forceinline__ int gswz(int p, uint32_t tabv) {
-  return p ^ (int)((tabv ^ (uint32_t)(p >> 4)) & 15u);
+  uint32_t h = tabv ^ (uint32_t)(p >> 4);
+  if (WIDE) h ^= (uint32_t)(p >> 8);
+  return p ^ (int)(h & 15u);
 }
 
 // Precision modes: 1 TF32, 3 3xTF32 (kind::tf32, K = 8 fp32 per product);
@@ -450,7 +459,7 @@ __device__ __forceinline__ void stage_epilogue(const PRun &P, const float2 *tws,
 #pragma unroll
   for (int j = 0; j < R; ++j) {
     const float2 y = cmul(make_float2(d[2 * j], d[2 * j + 1]), twrow[j << SH]);
-    w.buf[gswz(base + (j << SH), tabv)] = y;
+    w.buf[gswz<(G::LOG2L > 8)>(base + (j << SH), tabv)] = y;
   }
 }
 
@@ -469,7 +478,7 @@ __device__ __forceinline__ void stage_rows(const PRun &P, const WG &w) {
   for (int c = 0; c < R; c += 8) {
     float2 row[8];
 #pragma unroll
-    for (int jj = 0; jj < 8; ++jj) row[jj] = w.buf[gswz(base + ((c + jj) << SH), tabv)];
+    for (int jj = 0; jj < 8; ++jj) row[jj] = w.buf[gswz<(G::LOG2L > 8)>(base + ((c + jj) << SH), tabv)];
     split_store8<PREC>(row, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
                        w.slot + G::Q + w.lane_off + a_cols8(PREC) * c / 8);
   }

@@ -165,7 +165,8 @@ int stage_mode(const int modes[3], int t, int S) {
 
 // Shared-memory wavefronts per warp-wide 8-byte access of the warpgroup
 // kernel's transposes (1.0 = conflict free), for swizzle table `tab`:
-// phys(P) = P ^ ((tab[ul & 15] ^ (P >> 4)) & 15).
+// phys(P) = P ^ ((tab[ul & 15] ^ (P >> 4)) & 15), and for sub-transforms
+// longer than 256 points also ^ ((P >> 8) & 15) (gswz in group_kernel.cuh).
 double swizzle_cost(int r, int S, const int modes[3], unsigned long long tab, int team) {
   const int log2r = ilog2(r);
   const int L = 1 << (log2r * S);
@@ -201,7 +202,9 @@ double swizzle_cost(int r, int S, const int modes[3], unsigned long long tab, in
               const int hi = q >> sl, lo = q & ((1 << sl) - 1);
               const int P = ul * L + (hi << (sl + log2r)) + (j << sl) + lo;
               const unsigned tv = (unsigned)(tab >> (4 * (ul & 15))) & 15u;
-              const int ph = P ^ (int)((tv ^ (unsigned)(P >> 4)) & 15u);
+              unsigned hsw = tv ^ (unsigned)(P >> 4);
+              if (log2r * S > 8) hsw ^= (unsigned)(P >> 8);
+              const int ph = P ^ (int)(hsw & 15u);
               const int slot = ph & 15;
               if (!(seen & (1 << slot))) {
                 seen |= 1 << slot;
