@@ -27,6 +27,21 @@
  * Threading: plans are independent objects; one plan must not be executed
  * concurrently on two streams (its scratch is shared).  tcu_dft_last_error()
  * is thread-local.
+ *
+ * Diagnostics (environment, read at each call):
+ *   TCU_DFT_DEBUG=1       every exec call synchronises its stream and returns
+ *                         the plan's error word (as the *_check calls)
+ *                         instead of returning once the launches are queued.
+ *   TCU_DFT_FAIL_ALLOC=k  host-side fault injection for tests: the k-th
+ *                         device allocation of each plan call (k >= 1) fails
+ *                         as if the device were out of memory; the plan call
+ *                         then frees what it had and returns NULL with
+ *                         ERR_OOM.
+ * Each pass's launches sit in an NVTX range ("tcu_dft pass 1", ...; the 2-D
+ * calls "tcu_dft2", "tcu_conv2", "tcu_stencil").  The library is also built
+ * with every shared-memory, tensor-memory and global index of the pass
+ * kernels checked (libtcu_dft_checked.so, -DTCU_DFT_CHECKED): an index out
+ * of range skips the access and records ERR_BOUNDS in the plan's error word.
  */
 #ifndef TCU_DFT_H
 #define TCU_DFT_H
@@ -62,7 +77,8 @@ enum {
   TCU_DFT_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed, or no sm_103 device */
   TCU_DFT_ERR_OOM = 4,         /* device allocation failed */
   TCU_DFT_ERR_TIMEOUT = 5,     /* a device-side wait hit its iteration limit */
-  TCU_DFT_ERR_TOO_LARGE = 6    /* beyond the fixed memory of tcu_dft_exec_noalloc */
+  TCU_DFT_ERR_TOO_LARGE = 6,   /* beyond the fixed memory of tcu_dft_exec_noalloc */
+  TCU_DFT_ERR_BOUNDS = 7       /* checked build: a kernel index was out of range */
 };
 
 /* Build a plan for `batch` forward/inverse DFTs of length n with radix
@@ -135,7 +151,8 @@ int tcu_dft_exec_host(tcu_dft_plan_t p, const void *h_in, void *h_out,
                       void *d_work, int dir, void *stream);
 
 /* Synchronise `stream` and report whether any device-side wait of this
- * plan's kernels gave up (ERR_TIMEOUT), then clear the flag.  OK otherwise;
+ * plan's kernels gave up (ERR_TIMEOUT) or, in the checked build, an index
+ * was out of range (ERR_BOUNDS), then clear the flag.  OK otherwise;
  * ERR_CUDA if the synchronisation itself failed. */
 int tcu_dft_check(tcu_dft_plan_t p, void *stream);
 

@@ -31,6 +31,7 @@ ERR_CUDA = 3
 ERR_OOM = 4
 ERR_TIMEOUT = 5
 ERR_TOO_LARGE = 6
+ERR_BOUNDS = 7
 
 PLAN_DEFAULT = 0
 PLAN_NO_FUSE = 1
@@ -58,19 +59,24 @@ class TcuDftError(RuntimeError):
 
 
 def lib_path() -> str:
+    """The library this process uses: libtcu_dft.so, or the bounds-checked
+    libtcu_dft_checked.so when TCU_DFT_CHECKED=1 is set before the first
+    ``lib()`` call."""
+    if os.environ.get("TCU_DFT_CHECKED") == "1":
+        return _build.CHECKED_LIB_PATH
     return _build.LIB_PATH
 
 
 def lib():
-    """Load libtcu_dft.so (built in-tree by ``_build.build()``)."""
+    """Load the library (built in-tree by ``_build.build()``)."""
     global _lib
     if _lib is not None:
         return _lib
-    path = _build.LIB_PATH
+    path = lib_path()
     if not os.path.exists(path):
         raise ImportError(
-            "libtcu_dft.so is not built (%s); run "
-            "paper_1908_06649_gb300._build.build() first" % path)
+            "%s is not built; run paper_1908_06649_gb300._build.build_all() "
+            "first" % path)
     L = ctypes.CDLL(path)
     vp, i64, i32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_int32
     L.tcu_dft_plan.argtypes = [i64, i64, i32, i32]

@@ -191,9 +191,9 @@ tcu_dft2_plan_s *make_dft2(int64_t n1, int64_t n2, int64_t batch, int32_t r,
   }
   if (rc == TCU_DFT_OK) rc = upload(&p->cimg, conv_img);
   if (rc == TCU_DFT_OK &&
-      (cudaMalloc((void **)&p->scratch, (size_t)(batch * n1 * n2) * sizeof(float2)) !=
+      (dev_malloc((void **)&p->scratch, (size_t)(batch * n1 * n2) * sizeof(float2)) !=
            cudaSuccess ||
-       cudaMalloc((void **)&p->err, sizeof(int)) != cudaSuccess ||
+       dev_malloc((void **)&p->err, sizeof(int)) != cudaSuccess ||
        cudaMemset(p->err, 0, sizeof(int)) != cudaSuccess)) {
     cudaGetLastError();
     rc = TCU_DFT_ERR_OOM;
@@ -232,6 +232,7 @@ extern "C" {
 tcu_dft2_plan_t tcu_dft2_plan(int64_t n1, int64_t n2, int64_t batch, int32_t sqrt_m,
                               int32_t precision) {
   int rc;
+  arm_alloc_faults();
   tcu_dft2_plan_s *p = make_dft2(n1, n2, batch, sqrt_m, precision, rc);
   g_last_error = rc;
   return p;
@@ -244,11 +245,14 @@ int tcu_dft2_exec(tcu_dft2_plan_t p, const void *in, void *out, int dir, void *s
   if (rc != TCU_DFT_OK) return rc;
   cudaStream_t st = (cudaStream_t)stream;
   const int di = dir_index(dir);
-  rc = run_dft2_pass(p, p->cols, di, (const float2 *)in, p->scratch, false, nullptr, st);
-  if (rc == TCU_DFT_OK)
-    rc = run_dft2_pass(p, p->rows, di, p->scratch, (float2 *)out, dir == TCU_DFT_INVERSE,
-                       nullptr, st);
-  return rc;
+  {
+    const NvtxRange range("tcu_dft2");
+    rc = run_dft2_pass(p, p->cols, di, (const float2 *)in, p->scratch, false, nullptr, st);
+    if (rc == TCU_DFT_OK)
+      rc = run_dft2_pass(p, p->rows, di, p->scratch, (float2 *)out, dir == TCU_DFT_INVERSE,
+                         nullptr, st);
+  }
+  return rc == TCU_DFT_OK && debug_exec() ? tcu_dft2_check(p, stream) : rc;
 }
 
 int tcu_conv2_exec(tcu_dft2_plan_t p, const void *in, const void *spectrum, void *out,
@@ -258,6 +262,7 @@ int tcu_conv2_exec(tcu_dft2_plan_t p, const void *in, const void *spectrum, void
   int rc = check_buffers(in, out, bytes);
   if (rc != TCU_DFT_OK) return rc;
   cudaStream_t st = (cudaStream_t)stream;
+  const NvtxRange range("tcu_conv2");
   // columns: in -> scratch; rows forward, times the spectrum and inverse on
   // chip: scratch -> scratch (an item reads its rows before writing them);
   // inverse columns with 1/(n1 n2): scratch -> out
@@ -274,7 +279,8 @@ int tcu_conv2_exec(tcu_dft2_plan_t p, const void *in, const void *spectrum, void
   else if (p->r == 16) e = launch_rowconv_r16(p->precision, p->rows.s, g, p->num_sms, st);
   else e = launch_rowconv_r32(p->precision, p->rows.s, g, p->num_sms, st);
   if (e != cudaSuccess) return TCU_DFT_ERR_CUDA;
-  return run_dft2_pass(p, p->cols, 1, p->scratch, (float2 *)out, true, nullptr, st);
+  rc = run_dft2_pass(p, p->cols, 1, p->scratch, (float2 *)out, true, nullptr, st);
+  return rc == TCU_DFT_OK && debug_exec() ? tcu_dft2_check(p, stream) : rc;
 }
 
 int tcu_dft2_check(tcu_dft2_plan_t p, void *stream) {
@@ -283,11 +289,8 @@ int tcu_dft2_check(tcu_dft2_plan_t p, void *stream) {
   int flag = 0;
   if (cudaMemcpy(&flag, p->err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
     return TCU_DFT_ERR_CUDA;
-  if (flag) {
-    cudaMemset(p->err, 0, sizeof(int));
-    return TCU_DFT_ERR_TIMEOUT;
-  }
-  return TCU_DFT_OK;
+  if (flag) cudaMemset(p->err, 0, sizeof(int));
+  return word_status(flag);
 }
 
 int tcu_dft2_destroy(tcu_dft2_plan_t p) {
@@ -298,6 +301,7 @@ int tcu_dft2_destroy(tcu_dft2_plan_t p) {
 tcu_stencil_plan_t tcu_stencil_plan(int64_t side, int32_t steps, int32_t sqrt_m,
                                     int32_t precision) {
   g_last_error = TCU_DFT_OK;
+  arm_alloc_faults();
   if (side < 1 || steps < 1 ||
       (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32 && !prec_bf16(precision))) {
     g_last_error = TCU_DFT_ERR_INVALID;
@@ -329,10 +333,10 @@ tcu_stencil_plan_t tcu_stencil_plan(int64_t side, int32_t steps, int32_t sqrt_m,
   if (rc == TCU_DFT_OK) p->wpow = make_dft2(Nw, Nw, 1, sqrt_m, precision, rc);
   if (rc == TCU_DFT_OK) {
     p->num_sms = p->conv->num_sms;
-    if (cudaMalloc((void **)&p->tile_buf, (size_t)(p->tiles * N * N) * sizeof(float2)) !=
+    if (dev_malloc((void **)&p->tile_buf, (size_t)(p->tiles * N * N) * sizeof(float2)) !=
             cudaSuccess ||
-        cudaMalloc((void **)&p->wgrid, (size_t)(Nw * Nw) * sizeof(float2)) != cudaSuccess ||
-        cudaMalloc((void **)&p->wker, (size_t)(N * N) * sizeof(float2)) != cudaSuccess) {
+        dev_malloc((void **)&p->wgrid, (size_t)(Nw * Nw) * sizeof(float2)) != cudaSuccess ||
+        dev_malloc((void **)&p->wker, (size_t)(N * N) * sizeof(float2)) != cudaSuccess) {
       cudaGetLastError();
       rc = TCU_DFT_ERR_OOM;
     }
@@ -375,6 +379,7 @@ int tcu_stencil_exec(tcu_stencil_plan_t p, const float *w3x3, const float *A, fl
   const size_t bytes = (size_t)(p->side * p->side) * sizeof(float);
   if (A != Ak && overlaps(A, Ak, bytes)) return TCU_DFT_ERR_INVALID;
   cudaStream_t st = (cudaStream_t)stream;
+  const NvtxRange range("tcu_stencil");
   // W (Lemma 2), the kernel W' and its spectrum
   int rc = stencil_weight_grid(p, w3x3, st);
   if (rc != TCU_DFT_OK) return rc;
@@ -387,10 +392,10 @@ int tcu_stencil_exec(tcu_stencil_plan_t p, const float *w3x3, const float *A, fl
     return TCU_DFT_ERR_CUDA;
   rc = tcu_conv2_exec(p->conv, p->tile_buf, p->wker, p->tile_buf, st);
   if (rc != TCU_DFT_OK) return rc;
-  return launch_extract_tiles(Ak, p->tile_buf, p->side, p->k, p->N, p->num_sms, st) ==
-                 cudaSuccess
-             ? TCU_DFT_OK
-             : TCU_DFT_ERR_CUDA;
+  if (launch_extract_tiles(Ak, p->tile_buf, p->side, p->k, p->N, p->num_sms, st) !=
+      cudaSuccess)
+    return TCU_DFT_ERR_CUDA;
+  return debug_exec() ? tcu_stencil_check(p, stream) : TCU_DFT_OK;
 }
 
 int tcu_stencil_check(tcu_stencil_plan_t p, void *stream) {

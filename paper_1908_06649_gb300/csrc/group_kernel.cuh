@@ -215,7 +215,27 @@ struct WG {
   uint32_t ph_mma, ph_stg, ph_tws;
   bool fail;
   bool tws_inflight;  // warp 0: a twiddle copy has not been waited on
+#ifdef TCU_DFT_CHECKED
+  int *err;           // error word: index violations are recorded at once
+#endif
 };
+
+// Bounds-checked build (-DTCU_DFT_CHECKED): false when index i is outside
+// [0, n), with TCU_DFT_ERR_BOUNDS recorded in the error word; the caller
+// then skips the access (no trap, no fault).  The constant true otherwise,
+// so the normal build is unchanged.
+__device__ __forceinline__ bool in_range(const WG &w, long long i, long long n) {
+#ifdef TCU_DFT_CHECKED
+  if (i >= 0 && i < n) return true;
+  atomicCAS(w.err, 0, TCU_DFT_ERR_BOUNDS);
+  return false;
+#else
+  (void)w;
+  (void)i;
+  (void)n;
+  return true;
+#endif
+}
 
 template <class G>
 __device__ __forceinline__ void row_of(int mode, int rho, int &ul, int &q) {
@@ -377,10 +397,15 @@ __device__ __forceinline__ void issue_input(const PRun &P, const CUtensorMap *tm
     const uint32_t bytes = (uint32_t)(rem << G::LOG2L) * 8u;
     const long long b = u0 >> G::LOG2UPER;
     const long long v = u0 & ((1ll << G::LOG2UPER) - 1);
-    const float2 *src = P.in + ((b & P.in_bmask) << G::LOG2N) + (v << G::LOG2L);
+    const long long off = ((b & P.in_bmask) << G::LOG2N) + (v << G::LOG2L);
+    const float2 *src = P.in + off;
+    const long long in_elems =
+        P.in_bmask == -1 ? (P.U << G::LOG2L) : ((P.in_bmask + 1) << G::LOG2N);
+    const bool ok = in_range(w, off + (rem << G::LOG2L) - 1, in_elems);
     if (elect_one()) {
-      mbar_expect_tx(w.bar_stg, bytes);
-      tma_load_1d(dst, src, bytes, w.bar_stg);
+      // a skipped copy still completes the phase (no bytes expected)
+      mbar_expect_tx(w.bar_stg, ok ? bytes : 0u);
+      if (ok) tma_load_1d(dst, src, bytes, w.bar_stg);
     }
   }
   __syncwarp();
@@ -397,14 +422,15 @@ __device__ __forceinline__ void issue_twiddles(const PRun &P, const CUtensorMap 
     const long long v0 = u0 & ((1ll << G::LOG2UPER) - 1);
     const int vl0 = (int)(v0 & ((1 << G::LOG2VL) - 1));
     const uint32_t dst = smem_u32(w.tws);
+    const long long boff = (v0 >> G::LOG2VL) << G::LOG2L;
+    const bool ok =
+        !G::TW2L || in_range(w, boff + G::L - 1, (1ll << (G::LOG2UPER - G::LOG2VL)) << G::LOG2L);
     if (elect_one()) {
-      mbar_expect_tx(w.bar_tws, G::GPTS * 8 + (G::TW2L ? G::L * 8 : 0));
+      mbar_expect_tx(w.bar_tws, G::GPTS * 8 + (G::TW2L && ok ? G::L * 8 : 0));
 #pragma unroll
       for (int k0 = 0; k0 < G::L; k0 += G::TMA_ROWS)
         tma_load_3d(dst + k0 * G::GG * 8, tm, 2 * vl0, k0, 0, w.bar_tws);
-      if (G::TW2L)
-        tma_load_1d(smem_u32(w.twb), P.tw_b + ((v0 >> G::LOG2VL) << G::LOG2L), G::L * 8,
-                    w.bar_tws);
+      if (G::TW2L && ok) tma_load_1d(smem_u32(w.twb), P.tw_b + boff, G::L * 8, w.bar_tws);
     }
     __syncwarp();
   }
@@ -429,14 +455,18 @@ __device__ __forceinline__ void staged_row(const WG &w, float2 *x) {
   int ul, q;
   row_of<G>(G::MODE_FIRST, w.rho, ul, q);
   constexpr int JS = 1 << (G::LOG2L - G::LOG2R);  // a = j * R^(S-1) + q
+  const float2 zero = make_float2(0.f, 0.f);
   if (G::MODE_FIRST == kUF) {
-    const float2 *p = w.stg + q * G::GG + ul;  // staging [a][ul]
+    const int i0 = q * G::GG + ul;  // staging [a][ul]
+    const float2 *p = w.stg + i0;
 #pragma unroll
-    for (int j = 0; j < R; ++j) x[j] = p[j * JS * G::GG];
+    for (int j = 0; j < R; ++j)
+      x[j] = in_range(w, i0 + j * JS * G::GG, G::GPTS) ? p[j * JS * G::GG] : zero;
   } else {
-    const float2 *p = w.stg + (ul << G::LOG2L) + q;  // staging [ul][a]
+    const int i0 = (ul << G::LOG2L) + q;  // staging [ul][a]
+    const float2 *p = w.stg + i0;
 #pragma unroll
-    for (int j = 0; j < R; ++j) x[j] = p[j * JS];
+    for (int j = 0; j < R; ++j) x[j] = in_range(w, i0 + j * JS, G::GPTS) ? p[j * JS] : zero;
   }
 }
 
@@ -458,8 +488,11 @@ __device__ __forceinline__ void stage_epilogue(const PRun &P, const float2 *tws,
   load_d_row<G, PREC>(w, d);
 #pragma unroll
   for (int j = 0; j < R; ++j) {
-    const float2 y = cmul(make_float2(d[2 * j], d[2 * j + 1]), twrow[j << SH]);
-    w.buf[gswz<(G::LOG2L > 8)>(base + (j << SH), tabv)] = y;
+    const float2 t = in_range(w, TWOFF + lo + (j << SH), G::TW_ENTRIES) ? twrow[j << SH]
+                                                                         : make_float2(1.f, 0.f);
+    const float2 y = cmul(make_float2(d[2 * j], d[2 * j + 1]), t);
+    const int bi = gswz<(G::LOG2L > 8)>(base + (j << SH), tabv);
+    if (in_range(w, bi, G::GPTS)) w.buf[bi] = y;
   }
 }
 
@@ -478,7 +511,10 @@ __device__ __forceinline__ void stage_rows(const PRun &P, const WG &w) {
   for (int c = 0; c < R; c += 8) {
     float2 row[8];
 #pragma unroll
-    for (int jj = 0; jj < 8; ++jj) row[jj] = w.buf[gswz<(G::LOG2L > 8)>(base + ((c + jj) << SH), tabv)];
+    for (int jj = 0; jj < 8; ++jj) {
+      const int bi = gswz<(G::LOG2L > 8)>(base + ((c + jj) << SH), tabv);
+      row[jj] = in_range(w, bi, G::GPTS) ? w.buf[bi] : make_float2(0.f, 0.f);
+    }
     split_store8<PREC>(row, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
                        w.slot + G::Q + w.lane_off + a_cols8(PREC) * c / 8);
   }
@@ -526,22 +562,49 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, 
   const float2 *twbs = w.twb + klow;
   const float2 *twbg = P.tw_b + (vh << G::LOG2L) + klow;
   constexpr int TBJ = 1 << (G::LOG2L - G::LOG2R);
-  const float2 *sp = P.spec + ((u & P.spec_mask) << G::LOG2L) + klow;
+  const long long soff = ((u & P.spec_mask) << G::LOG2L) + klow;
+  const float2 *sp = P.spec + soff;
   const bool mul = SPEC && G::MODE_LAST == kRQF && P.spec != nullptr;
+  // index bounds of the checked build (element offsets from each base)
+  const long long doff = dst - P.out;
+  const long long out_elems =
+      P.out_bmask == -1 ? (P.U << G::LOG2L) : ((P.out_bmask + 1) << G::LOG2NT);
+  const long long toff = klow * G::GG + ul, goff = ((long long)klow << G::LOG2VL) + vl;
+  const long long gboff = (vh << G::LOG2L) + klow;
+  const float2 one = make_float2(1.f, 0.f);
 #pragma unroll
   for (int j = 0; j < R; ++j) {
     float2 y = make_float2(d[2 * j], d[2 * j + 1]);
-    if (G::MODE_LAST == kRQF && mul) y = cmul(y, __ldg(sp + j * JS));
+    if (G::MODE_LAST == kRQF && mul)
+      y = cmul(y, in_range(w, soff + j * JS, (P.spec_mask + 1) << G::LOG2L) ? __ldg(sp + j * JS)
+                                                                          : one);
     if (G::TW_SMEM) {
-      y = G::TW2L ? cmul(y, cmul(tws[j * TJS], twbs[j * TBJ])) : cmul(y, tws[j * TJS]);
+      const float2 ta = in_range(w, toff + j * TJS, G::GPTS) ? tws[j * TJS] : one;
+      if (G::TW2L) {
+        const float2 tb = in_range(w, klow + j * TBJ, G::L) ? twbs[j * TBJ] : one;
+        y = cmul(y, cmul(ta, tb));
+      } else {
+        y = cmul(y, ta);
+      }
     } else if (G::TW_OUT) {
-      y = G::TW2L ? cmul(y, cmul(__ldg(twg + j * TWG), __ldg(twbg + j * TBJ)))
-                  : cmul(y, __ldg(twg + j * TWG));
+      const float2 ta =
+          in_range(w, goff + j * TWG, (long long)G::L << G::LOG2VL) ? __ldg(twg + j * TWG) : one;
+      if (G::TW2L) {
+        const float2 tb =
+            in_range(w, gboff + j * TBJ, (1ll << (G::LOG2UPER - G::LOG2VL)) << G::LOG2L)
+                ? __ldg(twbg + j * TBJ)
+                : one;
+        y = cmul(y, cmul(ta, tb));
+      } else {
+        y = cmul(y, ta);
+      }
     }
-    if (OUT_L2)
-      __stcg(dst + j * JS, y);
-    else
-      __stcs(dst + j * JS, y);
+    if (in_range(w, doff + j * JS, out_elems)) {
+      if (OUT_L2)
+        __stcg(dst + j * JS, y);
+      else
+        __stcs(dst + j * JS, y);
+    }
   }
 }
 
@@ -642,8 +705,16 @@ __device__ __forceinline__ void conv_turn(const PRun &P, long long item, const W
   for (int c = 0; c < R; c += 8) {
     float2 x[8];
 #pragma unroll
-    for (int jj = 0; jj < 8; ++jj)
-      x[jj] = cmul(make_float2(d[2 * (c + jj)], d[2 * (c + jj) + 1]), __ldg(sp + (c + jj) * JS));
+    for (int jj = 0; jj < 8; ++jj) {
+#ifdef TCU_DFT_CHECKED
+      const float2 s = in_range(w, (sp - P.spec) + (c + jj) * JS, (P.spec_mask + 1) << G::LOG2L)
+                           ? __ldg(sp + (c + jj) * JS)
+                           : make_float2(0.f, 0.f);
+#else
+      const float2 s = __ldg(sp + (c + jj) * JS);
+#endif
+      x[jj] = cmul(make_float2(d[2 * (c + jj)], d[2 * (c + jj) + 1]), s);
+    }
     split_store8<PREC>(x, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
                        w.slot + G::Q + w.lane_off + a_cols8(PREC) * c / 8);
   }
@@ -837,6 +908,9 @@ __global__ void __launch_bounds__(
       G::TW_ENTRIES, a.p[1].tw_stage, tw_inv, CONV ? G::TW_ENTRIES : 0, mbar, tmem_slot);
   WG w;
   init_wg<R, SM, G::GCOLS, TW>(w, tbase, smem);
+#ifdef TCU_DFT_CHECKED
+  w.err = a.err;
+#endif
 
   const int team = (threadIdx.x >> 7) / TW;
   const long long nitems = (P.U + G::GG - 1) >> G::LOG2GG;
@@ -852,7 +926,7 @@ __global__ void __launch_bounds__(
       process_item<G, PREC, false>(P, &a.tm_tw, tw, item, w, nx);
     item += istride;
   }
-  if (w.fail && w.rho == 0) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);
+  if (w.fail && w.rho == 0) atomicCAS(a.err, 0, TCU_DFT_ERR_TIMEOUT);
   // on failure a copy issued for the next item may still be landing
   kernel_teardown(tbase, w, w.fail && nx.issued, w.fail && w.tws_inflight);
 }
@@ -1057,6 +1131,9 @@ __global__ void __launch_bounds__(Geo<R, S1, log2_radix(R) * S2, kFirst>::THREAD
       G1::TW_ENTRIES, a.p[1].tw_stage, tw2, G2::TW_ENTRIES, mbar, tmem_slot);
   WG w;
   init_wg<R, SM, G1::GCOLS>(w, tbase, smem);
+#ifdef TCU_DFT_CHECKED
+  w.err = a.err;
+#endif
   const int wg = threadIdx.x >> 7;
   FusedSched *box = boxes + wg;
 
@@ -1121,7 +1198,7 @@ __global__ void __launch_bounds__(Geo<R, S1, log2_radix(R) * S2, kFirst>::THREAD
   // all stores of this warpgroup are issued: publish the last completion
   named_bar_or(w.bar_id, w.bar_count, false);
   if (w.team_lead) nx.publish_pending();
-  if (w.rho == 0 && w.fail) atomicExch(a.err, TCU_DFT_ERR_TIMEOUT);
+  if (w.rho == 0 && w.fail) atomicCAS(a.err, 0, TCU_DFT_ERR_TIMEOUT);
   kernel_teardown(tbase, w, w.fail && stg_pending, w.fail && w.tws_inflight);
 }
 

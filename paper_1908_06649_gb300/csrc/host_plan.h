@@ -10,6 +10,8 @@
 
 #include <vector>
 
+#include <nvtx3/nvToolsExt.h>
+
 #include "../../include/tcu_dft.h"
 #include "launch.h"
 
@@ -102,9 +104,35 @@ struct DirTables {
   std::vector<float2> stage[kMaxPasses], A[kMaxPasses], B[kMaxPasses];
 };
 
+// Device allocation of the plans (cudaMalloc), with a host-side fault
+// injector for the tests of the plans' error paths: with TCU_DFT_FAIL_ALLOC=k
+// (k >= 1) in the environment, the k-th allocation after arm_alloc_faults()
+// on this thread fails as if the device were out of memory.  No GPU fault is
+// involved: the allocation is simply not made.
+void arm_alloc_faults();
+cudaError_t dev_malloc(void **ptr, size_t bytes);
+
+// TCU_DFT_DEBUG=1 in the environment: every exec call synchronises its
+// stream and returns the plan's error word (as tcu_dft_check) instead of
+// returning as soon as the launches are queued.
+bool debug_exec();
+
+// An NVTX range over the launches of one pass (host side; seen by nsys and
+// by ncu's --nvtx filters, free when no tool is attached).
+struct NvtxRange {
+  explicit NvtxRange(const char *name) { nvtxRangePushA(name); }
+  ~NvtxRange() { nvtxRangePop(); }
+  NvtxRange(const NvtxRange &) = delete;
+  NvtxRange &operator=(const NvtxRange &) = delete;
+};
+
+// Status recorded in a plan's error word (0: none): the kernels write
+// TCU_DFT_ERR_TIMEOUT, the bounds-checked build also TCU_DFT_ERR_BOUNDS.
+int word_status(int flag);
+
 template <typename T>
 int upload(T **dst, const std::vector<T> &src) {
-  if (cudaMalloc((void **)dst, src.size() * sizeof(T)) != cudaSuccess) {
+  if (dev_malloc((void **)dst, src.size() * sizeof(T)) != cudaSuccess) {
     cudaGetLastError();
     *dst = nullptr;
     return TCU_DFT_ERR_OOM;

@@ -29,6 +29,34 @@ int ilog2(long long v) {
 
 int dir_index(int dir) { return dir == TCU_DFT_INVERSE ? 1 : 0; }
 
+namespace {
+thread_local int g_alloc_seq = 0, g_alloc_fail_at = 0;
+}  // namespace
+
+void arm_alloc_faults() {
+  const char *v = getenv("TCU_DFT_FAIL_ALLOC");
+  g_alloc_fail_at = v ? atoi(v) : 0;
+  g_alloc_seq = 0;
+}
+
+cudaError_t dev_malloc(void **ptr, size_t bytes) {
+  if (g_alloc_fail_at > 0 && ++g_alloc_seq == g_alloc_fail_at) {
+    *ptr = nullptr;
+    return cudaErrorMemoryAllocation;
+  }
+  return cudaMalloc(ptr, bytes);
+}
+
+bool debug_exec() {
+  const char *v = getenv("TCU_DFT_DEBUG");
+  return v && v[0] == '1';
+}
+
+int word_status(int flag) {
+  if (flag == 0) return TCU_DFT_OK;
+  return flag == TCU_DFT_ERR_BOUNDS ? TCU_DFT_ERR_BOUNDS : TCU_DFT_ERR_TIMEOUT;
+}
+
 // cuTensorMapEncodeTiled from the driver, through the runtime (no -lcuda).
 PFN_cuTensorMapEncodeTiled_v12000 tensor_map_encoder() {
   static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;

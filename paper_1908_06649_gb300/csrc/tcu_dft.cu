@@ -305,6 +305,7 @@ int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
     }
     if (events && cudaEventRecord((cudaEvent_t)events[0], st) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
+    const NvtxRange range("tcu_dft fused passes");
     if (fused_dispatch(p->r, p->precision, p->pass[0].s, p->pass[1].s, g, p->num_sms,
                        st) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
@@ -317,7 +318,10 @@ int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
 
   // in -> scratch[0] -> scratch[1] -> out
   const long long off = b0 * p->n;
+  static const char *const kRange[kMaxPasses] = {"tcu_dft pass 1", "tcu_dft pass 2",
+                                                 "tcu_dft pass 3"};
   for (int pi = 0; pi < p->npasses; ++pi) {
+    const NvtxRange range(kRange[pi]);
     const PassPlan &pp = p->pass[pi];
     const float2 *src = (pi == 0) ? (const float2 *)in : p->scratch[pi - 1] + off;
     float2 *dst = pp.last ? (float2 *)out : p->scratch[pi] + off;
@@ -363,6 +367,7 @@ const char *tcu_dft_strerror(int status) {
     case TCU_DFT_ERR_TIMEOUT: return "device wait timed out";
     case TCU_DFT_ERR_TOO_LARGE:
       return "size exceeds the fixed memory of tcu_dft_exec_noalloc";
+    case TCU_DFT_ERR_BOUNDS: return "index out of range (checked build)";
     default: return "unknown status";
   }
 }
@@ -377,6 +382,7 @@ tcu_dft_plan_t tcu_dft_plan(int64_t n, int64_t batch, int32_t sqrt_m,
 tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
                                int32_t precision, uint32_t flags) {
   g_last_error = TCU_DFT_OK;
+  arm_alloc_faults();
   if (n < 1 || batch < 1 ||
       (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32 && !prec_bf16(precision)) ||
       (flags & ~(uint32_t)(TCU_DFT_PLAN_NO_FUSE | TCU_DFT_PLAN_FUSE)) ||
@@ -449,7 +455,7 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
     }
   }
   if (rc == TCU_DFT_OK) {
-    if (cudaMalloc((void **)&p->err, sizeof(int)) != cudaSuccess ||
+    if (dev_malloc((void **)&p->err, sizeof(int)) != cudaSuccess ||
         cudaMemset(p->err, 0, sizeof(int)) != cudaSuccess) {
       cudaGetLastError();
       rc = TCU_DFT_ERR_OOM;
@@ -479,13 +485,13 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
       p->log2_items_per_chunk = ilog2(n2 / gg1) + log2C;
       scratch_tf = (long long)p->ring_chunks << log2C;
       p->counter_bytes = (size_t)(1 + batch + p->nchunks) * sizeof(int);
-      if (rc == TCU_DFT_OK && cudaMalloc((void **)&p->counters, p->counter_bytes) != cudaSuccess) {
+      if (rc == TCU_DFT_OK && dev_malloc((void **)&p->counters, p->counter_bytes) != cudaSuccess) {
         cudaGetLastError();
         rc = TCU_DFT_ERR_OOM;
       }
     }
     for (int i = 0; i < npasses - 1 && rc == TCU_DFT_OK; ++i)
-      if (cudaMalloc((void **)&p->scratch[i], (size_t)scratch_tf * n * sizeof(float2)) !=
+      if (dev_malloc((void **)&p->scratch[i], (size_t)scratch_tf * n * sizeof(float2)) !=
           cudaSuccess) {
         cudaGetLastError();
         rc = TCU_DFT_ERR_OOM;
@@ -516,7 +522,8 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
 
 int tcu_dft_exec_dir(tcu_dft_plan_t p, const void *in, void *out, int dir,
                      void *stream) {
-  return exec_impl(p, in, out, dir, stream, nullptr);
+  const int rc = exec_impl(p, in, out, dir, stream, nullptr);
+  return rc == TCU_DFT_OK && debug_exec() ? tcu_dft_check(p, stream) : rc;
 }
 
 int tcu_dft_exec_stalled(tcu_dft_plan_t p, const void *in, void *out, void *stream) {
@@ -532,7 +539,8 @@ int tcu_dft_exec_timed(tcu_dft_plan_t p, const void *in, void *out, int dir,
   if (!events) return TCU_DFT_ERR_INVALID;
   for (int i = 0; p && i <= p->npasses; ++i)
     if (!events[i]) return TCU_DFT_ERR_INVALID;
-  return exec_impl(p, in, out, dir, stream, events);
+  const int rc = exec_impl(p, in, out, dir, stream, events);
+  return rc == TCU_DFT_OK && debug_exec() ? tcu_dft_check(p, stream) : rc;
 }
 
 int tcu_dft_exec(tcu_dft_plan_t p, const void *in, void *out, void *stream) {
@@ -600,11 +608,8 @@ int tcu_dft_check(tcu_dft_plan_t p, void *stream) {
   int flag = 0;
   if (cudaMemcpy(&flag, p->err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
     return TCU_DFT_ERR_CUDA;
-  if (flag) {
-    cudaMemset(p->err, 0, sizeof(int));
-    return TCU_DFT_ERR_TIMEOUT;
-  }
-  return TCU_DFT_OK;
+  if (flag) cudaMemset(p->err, 0, sizeof(int));
+  return word_status(flag);
 }
 
 int tcu_dft_destroy(tcu_dft_plan_t p) {

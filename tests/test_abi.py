@@ -43,6 +43,16 @@ def test_every_declared_symbol_is_exported(lib):
         assert getattr(lib, name) is not None
 
 
+def test_checked_variant_exports_the_same_symbols():
+    """The bounds-checked build (-DTCU_DFT_CHECKED) is the same boundary."""
+    _build.build(checked=True)
+    out = subprocess.run(["nm", "-D", "--defined-only", _build.CHECKED_LIB_PATH],
+                         capture_output=True, text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (\w+)", out))
+    for name in declared_functions():
+        assert name in exported, name
+
+
 def test_binding_lists_every_symbol():
     import paper_1908_06649_gb300 as pkg
     assert sorted(pkg.SYMBOLS) == declared_functions()
@@ -52,6 +62,7 @@ def test_strerror_and_null_handling(lib):
     import paper_1908_06649_gb300 as pkg
     assert lib.tcu_dft_strerror(0) == b"ok"
     assert lib.tcu_dft_strerror(pkg.ERR_TIMEOUT) == b"device wait timed out"
+    assert b"out of range" in lib.tcu_dft_strerror(pkg.ERR_BOUNDS)
     assert lib.tcu_dft_destroy(None) == pkg.OK
     assert lib.tcu_dft_exec(None, None, None, None) == pkg.ERR_INVALID
     assert lib.tcu_dft_exec_dir(None, None, None, -1, None) == pkg.ERR_INVALID
