@@ -5,7 +5,9 @@ Default workload: n = 65536 (= 16^4, sqrt_m = 16), batch = 1024, N(0,1)
 inputs from seed 1, forward, 3xTF32.  One "step" is one complete forward
 transform of the whole batch (every stage of every pass), inputs resident in
 HBM (512 MiB, larger than the 129 MB L2, so no flush is needed between
-steps).
+steps; a workload whose buffers are smaller than twice the L2 gets an
+untimed 512 MiB write before every step, and its step time is the sum of
+the steps' own events).
 
 Prints ONE JSON line on stdout (rank 0).  Logs go to stderr.
 
@@ -191,17 +193,20 @@ def dist_setup():
     return world, rank, local
 
 
-def cpu_baseline(wl, seconds=10.0, sample=32):
+def cpu_baseline(wl, seconds=10.0, sample=32, y_gpu=None, tol=None):
     """The fp64 oracle (radix-2 FFT) on a bounded sample of the workload,
-    using every host core; returns the metric in GFLOP/s."""
+    using every host core; returns the metric in GFLOP/s.  With y_gpu (the
+    GPU's outputs for the same first `sample` transforms) it also returns
+    their per-transform relative L2 error against the oracle's outputs."""
     import oracle
     n = wl["n"]
     x = inputs.make(wl["kind"], n, wl["batch"], wl["seed"], first=0,
                     count=sample)
     threads = oracle.default_threads()
     done, used, t0 = 0, 1, time.perf_counter()
+    ref = None
     while True:
-        _, used = oracle.fft_radix2_timed(x, threads=threads)
+        ref, used = oracle.fft_radix2_timed(x, threads=threads)
         done += sample
         el = time.perf_counter() - t0
         if el >= seconds:
@@ -213,7 +218,14 @@ def cpu_baseline(wl, seconds=10.0, sample=32):
         oracle.fft_radix2_timed(x1, threads=1)
         done1 += x1.shape[0]
     el1 = time.perf_counter() - t1
-    return {"value": dft_flops(n, done) / el / 1e9, "unit": UNIT,
+    acc = None
+    if y_gpu is not None:
+        err = oracle.rel_l2(y_gpu.reshape(sample, n), ref)
+        acc = {"max_rel_l2": float(err.max()), "median_rel_l2": float(np.median(err)),
+               "transforms": sample, "tolerance": tol,
+               "ok": bool(tol is None or err.max() <= tol),
+               "against": "fp64 oracle outputs of the cpu_baseline sample"}
+    return acc, {"value": dft_flops(n, done) / el / 1e9, "unit": UNIT,
             "cores": used, "kind": "oracle",
             "sample": "%d transforms (first %d of the workload, repeated) of "
                       "n=%d through the fp64 recursive radix-2 FFT, %.1f s "
@@ -352,7 +364,8 @@ def run_grid(args):
                                   n1, n2, batch, g["seed"],
                                   "3xTF32" if args.precision == 3 else "TF32"),
                   "n1": n1, "n2": n2, "batch": batch, "sqrt_m": r,
-                  "l2": "inputs larger than L2, no flush"}
+                  "l2": "inputs larger than L2 (%d MiB per buffer), no flush"
+                        % (points * 8 >> 20)}
         value_of = lambda ms: flops / (ms * 1e-3) / 1e9
         bytes_min = 16.0 * points
     else:
@@ -380,7 +393,9 @@ def run_grid(args):
                                   side, side, k, tiles, Nt, Nt,
                                   "3xTF32" if args.precision == 3 else "TF32"),
                   "side": side, "steps": k, "sqrt_m": r, "tile": Nt,
-                  "l2": "inputs larger than L2, no flush"}
+                  "l2": "grid %d MiB, but every step streams the %d MiB tile "
+                        "batch through HBM three times, which evicts it; no "
+                        "flush" % (side * side * 4 >> 20, points * 8 >> 20)}
         value_of = lambda ms: side * side * k / (ms * 1e-3) / 1e9
         bytes_min = 8.0 * side * side
     for _ in range(max(3, args.warmup)):
@@ -436,6 +451,15 @@ def run_grid(args):
     return 0
 
 
+L2_BYTES = 129 << 20           # GB300 L2
+L2_FLUSH_BYTES = 512 << 20     # > 2 x L2
+
+
+def needs_flush(wl):
+    """Buffers smaller than twice the L2 would stay cached between steps."""
+    return wl["n"] * wl["batch"] * 8 < 2 * L2_BYTES
+
+
 def workload_config(wl, args):
     return {"workload": "batched complex64 forward DFT n=%d (=%d^%d) x batch "
                         "%d, %s inputs seed %d, %s" % (
@@ -445,8 +469,12 @@ def workload_config(wl, args):
                             "3xTF32" if args.precision == 3 else "TF32"),
             "n": wl["n"], "batch": wl["batch"], "sqrt_m": wl["sqrt_m"],
             "precision": "3xTF32" if args.precision == 3 else "TF32",
-            "l2": "inputs larger than L2 (%d MiB per buffer), no flush"
-                  % (wl["n"] * wl["batch"] * 8 >> 20),
+            "l2": (("inputs larger than L2 (%d MiB per buffer), no flush"
+                   % (wl["n"] * wl["batch"] * 8 >> 20))
+                   if not needs_flush(wl) else
+                   ("L2 flushed before every step (%d MiB write, untimed); "
+                    "%d MiB per buffer" % (L2_FLUSH_BYTES >> 20,
+                                           wl["n"] * wl["batch"] * 8 >> 20))),
             "parallelism": "replica/batch shard x%d" % args.gpus}
 
 
@@ -531,8 +559,13 @@ def main():
     if dist is not None:
         dist.barrier()
     torch.cuda.synchronize()
+    flush = needs_flush(wl)
+    l2buf = (torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+             if flush else None)
     t_start.record(stream)
     for i in range(K):
+        if flush:
+            l2buf.fill_(float(i))  # untimed: outside ev[i][0] .. ev[i][npass]
         plan.exec_timed(x, y, ev[i])
     t_end.record(stream)
     torch.cuda.synchronize()
@@ -540,7 +573,11 @@ def main():
         dist.barrier()
     clk = clocks.stop() if clocks else None
     plan.check()
-    elapsed_ms = t_start.elapsed_time(t_end)
+    if flush:
+        # the step is its own events, first pass to last, without the flush
+        elapsed_ms = sum(ev[i][0].elapsed_time(ev[i][npass]) for i in range(K))
+    else:
+        elapsed_ms = t_start.elapsed_time(t_end)
     pass_ms = [[ev[i][p].elapsed_time(ev[i][p + 1]) for i in range(K)]
                for p in range(npass)]
     elapsed_ms = max_over_ranks(elapsed_ms, dist, dev)
@@ -600,10 +637,16 @@ def main():
                "steps": args.e2e_steps}
 
     plan_fused = plan.fused
+    # GPU outputs of the first transforms, for the accuracy check of the
+    # CPU-baseline leg
+    sample = min(32, batch)
+    y_head = y.reshape(-1)[:sample * n].cpu().numpy()
     plan.destroy()
-    cpu = None
+    cpu = acc = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        cpu = cpu_baseline(wl, seconds=args.cpu_seconds)
+        acc, cpu = cpu_baseline(wl, seconds=args.cpu_seconds, sample=sample,
+                                y_gpu=y_head,
+                                tol=1e-5 if args.precision == 3 else 3e-3)
 
     if rank == 0:
         line = {
@@ -627,6 +670,8 @@ def main():
                                                   % (peak_kind, NOMINAL_TF32,
                                                      NOMINAL_BF16)},
             "cpu_baseline": cpu, "e2e": e2e,
+            "accuracy": acc,
+            "gpu": torch.cuda.get_device_name(dev),
             "gpu_launches": K * launches,
             "clocks": clk,
         }
