@@ -58,10 +58,10 @@ typedef struct tcu_dft_plan_s *tcu_dft_plan_t;
  *   TCU_DFT_TF32    -- one TF32 product, operands rounded to TF32 (~1e-3
  *                      rel. L2)
  *   TCU_DFT_3XTF32  -- hi*hi + lo*hi + hi*lo TF32 split products (fp32-level)
- *   TCU_DFT_BF16    -- one BF16 product (kind::f16; ~1e-2 rel. L2), radix 16
- *                      and n = 16^k only
- *   TCU_DFT_3XBF16  -- the same three split products in BF16 (~1e-4), radix
- *                      16 and n = 16^k only
+ *   TCU_DFT_BF16    -- one BF16 product (kind::f16; ~1e-2 rel. L2), n = r^k
+ *                      only (no mixed radix, no 2-D plans)
+ *   TCU_DFT_3XBF16  -- the same three split products in BF16 (~1e-4), n = r^k
+ *                      only
  * The BF16 modes are the low-precision variant (Sec. 4.5 cites half-precision
  * tensor-core FFTs): half the products of the TF32 modes per stage. */
 enum { TCU_DFT_TF32 = 1, TCU_DFT_3XTF32 = 3, TCU_DFT_BF16 = 4, TCU_DFT_3XBF16 = 5 };

@@ -16,7 +16,7 @@ CSRC = os.path.join(HERE, "csrc")
 UNITS = ["tcu_dft.cu", "host_tables.cu", "noalloc.cu", "grid_plan.cu",
          "kernels_r8.cu", "kernels_r16.cu", "kernels_r32.cu",
          "kernels_mixed_r8.cu", "kernels_mixed_r16.cu", "kernels_mixed_r32.cu",
-         "kernels_bf16_r16.cu",
+         "kernels_bf16_r8.cu", "kernels_bf16_r16.cu", "kernels_bf16_r32.cu",
          "grid_kernels.cu"]
 HEADERS = ["tcgen05.cuh", "group_kernel.cuh", "launch.h",
            "launch_impl.cuh", "host_plan.h"]

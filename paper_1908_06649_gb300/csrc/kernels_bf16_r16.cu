@@ -4,16 +4,10 @@
 
 namespace tcu {
 
-#define TCU_BF16_CASE(S, SO, ROLE, SP)                                                     \
-  if (s == S && lo == 4 * (SO) && role == ROLE && lp == 4 * (SP) && tw == 1)               \
-    return prec == 5 ? launch_pass_t<16, 5, S, 4 * (SO), ROLE, 4 * (SP)>(a, num_sms, st)  \
-                     : launch_pass_t<16, 4, S, 4 * (SO), ROLE, 4 * (SP)>(a, num_sms, st);
-
 cudaError_t launch_pass_bf16_r16(int prec, int s, int lo, int role, int lp, int tw,
                                  const GArgs &a, int num_sms, cudaStream_t st) {
-  if (s == 3 && lo == 0 && role == kSingle && lp == 0 && tw == 2)  // 16^3, one pass
-    return prec == 5 ? launch_team_t<16, 5, 3, 0, kSingle, 0, 2>(a, num_sms, st)
-                     : launch_team_t<16, 4, 3, 0, kSingle, 0, 2>(a, num_sms, st);
+  constexpr int R = 16;
+  TCU_BF16_TEAM_CASE(3, 0, kSingle, 0, 2)  // 16^3 in one pass
   TCU_BF16_CASE(1, 0, kSingle, 0)
   TCU_BF16_CASE(2, 0, kSingle, 0)
   TCU_BF16_CASE(2, 2, kFirst, 0)   // n = 16^4: 2 + 2

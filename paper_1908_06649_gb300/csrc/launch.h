@@ -59,7 +59,11 @@ struct RootsQ {
 cudaError_t launch_radix_q(int q, const float2 *x, float2 *out, long long batch, int log2n2,
                            const float2 *twA, const float2 *twB, const RootsQ &roots,
                            int num_sms, cudaStream_t st);
-// BF16-mode (precision 4, 5) radix-16 passes (kernels_bf16_r16.cu).
+// BF16-mode (precision 4, 5) passes of n = r^k (kernels_bf16_r{8,16,32}.cu).
+cudaError_t launch_pass_bf16_r8(int prec, int s, int lo, int role, int lp, int tw,
+                                const GArgs &a, int num_sms, cudaStream_t st);
+cudaError_t launch_pass_bf16_r32(int prec, int s, int lo, int role, int lp, int tw,
+                                 const GArgs &a, int num_sms, cudaStream_t st);
 cudaError_t launch_pass_bf16_r16(int prec, int s, int lo, int role, int lp, int tw,
                                  const GArgs &a, int num_sms, cudaStream_t st);
 // Mixed-radix warpgroup passes (kernels_mixed_r*.cu): same arguments as

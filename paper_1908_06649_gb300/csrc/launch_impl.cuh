@@ -92,6 +92,22 @@ cudaError_t launch_fused_t(const GArgs &a, int num_sms, cudaStream_t st) {
                      : launch_pass_t<R, 1, S, LO, ROLE, LP>(a, num_sms, st);
 #define TCU_PASS_CASE(S, SO, ROLE, SP) \
   TCU_PASS_CASE_L(S, log2_radix(R) * (SO), ROLE, log2_radix(R) * (SP))
+// The BF16 modes (precision 4: BF16, 5: 3xBF16; tcgen05 kind::f16) of a
+// pass or a team pass (items of TW warpgroups).
+#define TCU_BF16_CASE(S, SO, ROLE, SP)                                                  \
+  if (s == S && lo == log2_radix(R) * (SO) && role == ROLE &&                           \
+      lp == log2_radix(R) * (SP) && tw == 1)                                            \
+    return prec == 5 ? launch_pass_t<R, 5, S, log2_radix(R) * (SO), ROLE,               \
+                                     log2_radix(R) * (SP)>(a, num_sms, st)              \
+                     : launch_pass_t<R, 4, S, log2_radix(R) * (SO), ROLE,               \
+                                     log2_radix(R) * (SP)>(a, num_sms, st);
+#define TCU_BF16_TEAM_CASE(S, SO, ROLE, SP, TW)                                         \
+  if (s == S && lo == log2_radix(R) * (SO) && role == ROLE &&                           \
+      lp == log2_radix(R) * (SP) && tw == TW)                                           \
+    return prec == 5 ? launch_team_t<R, 5, S, log2_radix(R) * (SO), ROLE,               \
+                                     log2_radix(R) * (SP), TW>(a, num_sms, st)          \
+                     : launch_team_t<R, 4, S, log2_radix(R) * (SO), ROLE,               \
+                                     log2_radix(R) * (SP), TW>(a, num_sms, st);
 #define TCU_FUSED_CASE(S1, S2)                                                      \
   if (s1 == S1 && s2 == S2)                                                         \
     return prec == 3 ? launch_fused_t<R, 3, S1, S2>(a, num_sms, st)                 \

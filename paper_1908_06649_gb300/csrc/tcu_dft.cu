@@ -212,8 +212,12 @@ cudaError_t pass_dispatch(int r, int prec, const PassPlan &pp, const GArgs &a, i
     if (r == 16) return launch_pass_mixed_r16(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
     return launch_pass_mixed_r32(prec, pp.s, pp.lo, pp.role, pp.lp, a, num_sms, st);
   }
-  if (prec_bf16(prec))
-    return launch_pass_bf16_r16(prec, pp.s, pp.lo, pp.role, pp.lp, pp.tw, a, num_sms, st);
+  if (prec_bf16(prec)) {
+    if (r == 8) return launch_pass_bf16_r8(prec, pp.s, pp.lo, pp.role, pp.lp, pp.tw, a, num_sms, st);
+    if (r == 16)
+      return launch_pass_bf16_r16(prec, pp.s, pp.lo, pp.role, pp.lp, pp.tw, a, num_sms, st);
+    return launch_pass_bf16_r32(prec, pp.s, pp.lo, pp.role, pp.lp, pp.tw, a, num_sms, st);
+  }
   if (r == 8 && team_plan)
     return launch_team_r8(prec, pp.s, pp.lo, pp.role, pp.lp, pp.tw, a, num_sms, st);
   if (r == 16 && pp.tw > 1)
@@ -407,9 +411,9 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
   const bool is_mixed = m != n;
   const int npasses = is_mixed ? plan_mixed(r, n, batch, mixed)
                                : (k >= 1 ? plan_stages(r, k, st) : 0);
-  // the BF16 modes are instantiated for radix 16, r^k sizes
+  // the BF16 modes are instantiated for n = r^k (no mixed radix)
   if (npasses == 0 || (long long)batch * n > (1ll << 40) ||
-      (prec_bf16(precision) && (r != 16 || is_mixed))) {
+      (prec_bf16(precision) && is_mixed)) {
     g_last_error = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
   }

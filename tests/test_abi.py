@@ -83,7 +83,7 @@ def test_strerror_and_null_handling(lib):
     (16, 0, 16, 3, 1),       # batch < 1
     (16, 1, 16, 2, 1),       # precision not 1 or 3
     (16, 1, 16, 6, 1),       # precision not 1, 3, 4 or 5
-    (64, 1, 8, 4, 2),        # BF16 modes: radix 16 only
+    (128, 1, 8, 4, 2),       # BF16 modes: no mixed radix (2 x 8^2)
     (512, 1, 16, 5, 2),      # BF16 modes: no mixed radix
     (16, 1, 4, 3, 2),        # radix not in {8, 16, 32}
     (16, 1, 64, 3, 2),

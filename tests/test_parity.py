@@ -319,25 +319,28 @@ def test_mixed_radix_in_place(pkg):
     check(y, x, 3)
 
 
-# ---- the low-precision variant: BF16 operands on kind::f16 (radix 16).
+# ---- the low-precision variant: BF16 operands on kind::f16 (every radix).
 # Tolerance from the arithmetic: bf16 keeps 8 significant bits (unit
 # roundoff u = 2^-9 after rounding to nearest); one product per stage leaves
 # ~sqrt(2) u per real operand pair, growing ~sqrt(k) over k stages, so the
 # single product is held to 1e-2 and the hi/lo split (16 significant bits,
-# u^2-level terms dropped) to 1e-4 for k <= 6.
+# u^2-level terms dropped) to 1e-4 for up to 7 stages.
 BF16_TOL = {4: 1e-2, 5: 1e-4}
 
 
-@pytest.mark.parametrize("k,batch", [(1, 64), (2, 37), (3, 9), (4, 3), (5, 2), (6, 1)])
+@pytest.mark.parametrize("r,k,batch", [
+    (16, 1, 64), (16, 2, 37), (16, 3, 9), (16, 4, 3), (16, 5, 2), (16, 6, 1),
+    (8, 1, 64), (8, 2, 37), (8, 3, 11), (8, 4, 5), (8, 5, 3), (8, 6, 2), (8, 7, 1),
+    (32, 1, 64), (32, 2, 9), (32, 3, 3), (32, 4, 1)])
 @pytest.mark.parametrize("prec", [5, 4])
-def test_bf16_modes(pkg, k, batch, prec):
-    n = 16 ** k
-    x = inputs.make("normal", n, batch, seed=60 + k)
-    y, passes = run(pkg, x, 16, prec)
+def test_bf16_modes(pkg, r, k, batch, prec):
+    n = r ** k
+    x = inputs.make("normal", n, batch, seed=60 + k + r)
+    y, passes = run(pkg, x, r, prec)
     assert sum(passes) == k
     err = oracle.rel_l2(y, oracle.dft(x, threads=8))
     assert np.all(np.isfinite(err)) and err.max() <= BF16_TOL[prec], err.max()
-    yi, _ = run(pkg, x, 16, prec, inverse=True)
+    yi, _ = run(pkg, x, r, prec, inverse=True)
     erri = oracle.rel_l2(yi, oracle.dft(x, inverse=True, threads=8))
     assert erri.max() <= BF16_TOL[prec], erri.max()
 
