@@ -227,6 +227,17 @@ def cpu_baseline(wl, seconds=10.0, sample=32, y_gpu=None, tol=None):
         oracle.fft_radix2_timed(x1, threads=1)
         done1 += x1.shape[0]
     el1 = time.perf_counter() - t1
+    direct = None
+    if n <= 4096:
+        # the definition itself (O(n^2) per transform), for the small workload
+        nd, t2 = 0, time.perf_counter()
+        while time.perf_counter() - t2 < min(3.0, seconds / 3):
+            oracle.dft_direct(x, threads=threads)
+            nd += sample
+        el2 = time.perf_counter() - t2
+        direct = {"value": dft_flops(n, nd) / el2 / 1e9, "unit": UNIT,
+                  "sample": "%d transforms of n=%d by the direct O(n^2) "
+                            "definition, %d threads, %.1f s" % (nd, n, threads, el2)}
     acc = None
     if y_gpu is not None:
         err = oracle.rel_l2(y_gpu.reshape(sample, n), ref)
@@ -241,7 +252,8 @@ def cpu_baseline(wl, seconds=10.0, sample=32, y_gpu=None, tol=None):
                       "wall" % (done, sample, n, el),
             "one_core": {"value": dft_flops(n, done1) / el1 / 1e9, "unit": UNIT,
                          "sample": "%d transforms of n=%d on 1 core, %.1f s"
-                                   % (done1, n, el1)}}
+                                   % (done1, n, el1)},
+            "direct": direct}
 
 
 def run_reference(args, wl):
