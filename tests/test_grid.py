@@ -47,10 +47,10 @@ def test_dft2(pkg, r, n1, n2, batch, prec):
     back = plan.inverse(y)
     plan.check()
     yh = y.cpu().numpy().reshape(batch, n1, n2)
-    ref = grid.dft2(x)
+    ref = grid.dft2(x, threads=8)
     assert _rel(yh, ref).max() <= TOL[prec]
     bh = back.cpu().numpy().reshape(batch, n1, n2)
-    assert _rel(bh, grid.dft2(yh, inverse=True)).max() <= TOL[prec]
+    assert _rel(bh, grid.dft2(yh, inverse=True, threads=8)).max() <= TOL[prec]
     plan.destroy()
 
 

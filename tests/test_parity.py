@@ -259,6 +259,53 @@ def test_full_size_long_transforms(pkg):
     _sampled_full_size(pkg, x, 16, whole=(2,))
 
 
+def test_maximum_size_radix8(pkg):
+    # n = 8^9 = 2^27, the longest radix-8 plan: three passes of three stages,
+    # whole transform against the oracle, and back
+    n = 8 ** 9
+    x = inputs.make("normal", n, 1, seed=90)
+    y, passes = run(pkg, x, 8, 3)
+    assert passes == [3, 3, 3]
+    check(y, x, 3)
+    back, _ = run(pkg, y, 8, 3, inverse=True)
+    assert np.linalg.norm(back - x) / np.linalg.norm(x) <= 1e-5
+
+
+def _sumsq(v, chunk=1 << 24):
+    """sum |v|^2 in fp64, chunk by chunk (v complex64, up to 2^30 entries)."""
+    tot = 0.0
+    for a in range(0, v.shape[0], chunk):
+        seg = v[a:a + chunk].astype(np.complex128)
+        tot += float(np.sum(seg.real ** 2 + seg.imag ** 2))
+    return tot
+
+
+def test_maximum_size_radix32_closed_forms(pkg):
+    # n = 32^6 = 2^30, the longest radix-32 plan (three passes).  A whole
+    # transform would cost the oracle 16 GB and minutes, so the check is by
+    # closed forms at full size: DFT(delta_s)_k = w^{ks} on sampled k and
+    # Parseval; DFT(e^{+2 pi i f j / n}) = n delta_f over the whole output.
+    n = 32 ** 6
+    s, f = 123456789, 987654321 % n
+    x = np.zeros((2, n), np.complex64)
+    x[0, s] = 1.0
+    C = 1 << 24
+    for a in range(0, n, C):
+        j = np.arange(a, a + C, dtype=np.int64)
+        x[1, a:a + C] = np.exp(2j * np.pi * ((j * f) % n) / n)
+    y, passes = run(pkg, x, 32, 3)
+    assert passes == [2, 2, 2]
+    rng = np.random.default_rng(5)
+    ks = np.concatenate([[0, 1, n - 1, f], rng.integers(0, n, 4096)])
+    w = np.exp(-2j * np.pi * ((ks * s) % n) / n)
+    assert np.max(np.abs(y[0, ks] - w)) <= 1e-5
+    assert abs(_sumsq(y[0]) / n - 1.0) <= 1e-5
+    peak = complex(y[1, f])
+    assert abs(peak - n) / n <= 1e-5
+    rest = _sumsq(y[1]) - abs(peak) ** 2        # everything off the peak
+    assert np.sqrt(max(rest, 0.0)) / n <= 1e-5
+
+
 def test_exec_host_path(pkg):
     import torch
     n, batch = 4096, 64
