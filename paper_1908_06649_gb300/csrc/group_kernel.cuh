@@ -52,9 +52,11 @@ enum Role { kSingle = 0, kFirst = 1, kSecond = 2, kCols = 3 };
 
 __host__ __device__ constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 16 ? 4 : 5); }
 // Warpgroups per CTA: TMEM holds 512 columns, a warpgroup's slot 3 Q of
-// them; a first (strided) pass also stages its inter-pass twiddles in SMEM,
-// which leaves room for four.
-__host__ __device__ constexpr int pass_nwg(int R, int ROLE) { return R == 32 ? 2 : (ROLE == 1 ? 4 : 5); }
+// them; a radix-16 first (strided) pass also stages its inter-pass twiddles
+// in SMEM, which leaves room for four.
+__host__ __device__ constexpr int pass_nwg(int R, int ROLE) {
+  return R == 32 ? 2 : (ROLE == 1 && R == 16 ? 4 : 5);
+}
 
 // Compile-time geometry of one pass: S stages of radix R.  A transform of
 // length n is computed in up to three passes (the four-step split applied
@@ -107,7 +109,11 @@ struct Geo {
   static constexpr int MODE_MID = kUF;
   static constexpr int MODE_LAST = ROLE == kSingle ? kRQF : kUF;
   static constexpr bool TW_OUT = ROLE == kFirst;
-  static constexpr bool TW_SMEM = TW_OUT && R != 32;  // twiddles staged by TMA
+  // inter-pass twiddles staged by TMA per item (else read from the
+  // L2-resident tables): measured faster for radix 16 and for the radix-8
+  // team items; the one-warpgroup radix-8 items run faster with five
+  // warpgroups and global reads, radix 32 has no SMEM to spare
+  static constexpr bool TW_SMEM = TW_OUT && (R == 16 || (R == 8 && TW > 1));
   // w_M^{k v} with v = vh 2^VL + vl: table A [k][vl] and, for more than 256
   // columns, table B [vh][k] (two-level, so that no table exceeds L * 256)
   static constexpr int LOG2VL = (TW_OUT && LOG2UPER > 8) ? 8 : LOG2UPER;
