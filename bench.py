@@ -66,6 +66,36 @@ def dft_flops(n, batch):
     return 5.0 * n * math.log2(n) * batch
 
 
+def measure_tf32_tflops(dev, size=8192, reps=10):
+    """Dense TF32 tensor throughput of this GPU (TFLOP/s): the best of
+    `reps` cuBLAS GEMMs of size^3 with TF32 enabled; None on any failure."""
+    import torch
+    prev = torch.backends.cuda.matmul.allow_tf32
+    try:
+        torch.backends.cuda.matmul.allow_tf32 = True
+        a = torch.randn(size, size, device=dev)
+        b = torch.randn(size, size, device=dev)
+        c = torch.empty(size, size, device=dev)
+        for _ in range(3):
+            torch.matmul(a, b, out=c)
+        best = None
+        for _ in range(reps):
+            e0 = torch.cuda.Event(enable_timing=True)
+            e1 = torch.cuda.Event(enable_timing=True)
+            e0.record()
+            torch.matmul(a, b, out=c)
+            e1.record()
+            torch.cuda.synchronize()
+            ms = e0.elapsed_time(e1)
+            best = ms if best is None else min(best, ms)
+        del a, b, c
+        return 2.0 * size ** 3 / (best * 1e-3) / 1e12
+    except Exception:
+        return None
+    finally:
+        torch.backends.cuda.matmul.allow_tf32 = prev
+
+
 def load_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     try:
@@ -625,13 +655,6 @@ def main():
     if not plan.fused:
         kname = "pass kernel %d of %d (%d stages)" % (dom + 1, npass, stages[dom])
     achieved = bytes_launch / (avg[dom] * 1e-3) / 1e9
-    # whole-step roofline: min HBM bytes vs tensor flops at tf32 peak
-    p_tf32 = float(peaks["bf16_tflops"]) * NOMINAL_TF32 / NOMINAL_BF16
-    k = sum(stages)
-    tensor_flops = 8.0 * r * n * batch * k * args.precision
-    t_roof = max(bytes_launch / (hbm * 1e9), tensor_flops / (p_tf32 * 1e12))
-    frac_step = t_roof / (ms_per_step * 1e-3)
-
     e2e = None
     if args.e2e_steps > 0:
         h_in = torch.from_numpy(x_host).pin_memory()
@@ -656,6 +679,21 @@ def main():
                "unit": UNIT, "h2d_bytes_per_step": n * batch * 8,
                "d2h_bytes_per_step": n * batch * 8,
                "steps": args.e2e_steps}
+
+    # whole-step roofline: min HBM bytes vs tensor flops at the TF32 peak,
+    # measured here (cuBLAS TF32 GEMM, after every timed region) or, if that
+    # fails, the measured bf16 peak times the nominal TF32/BF16 ratio
+    p_tf32 = measure_tf32_tflops(dev) if rank == 0 else None
+    if p_tf32:
+        tf32_source = "measured in this run: cuBLAS TF32 GEMM 8192^3, best of 10"
+    else:
+        p_tf32 = float(peaks["bf16_tflops"]) * NOMINAL_TF32 / NOMINAL_BF16
+        tf32_source = "%s bf16 x %.2f/%.2f nominal" % (peak_kind, NOMINAL_TF32,
+                                                       NOMINAL_BF16)
+    k = sum(stages)
+    tensor_flops = 8.0 * r * n * batch * k * args.precision
+    t_roof = max(bytes_launch / (hbm * 1e9), tensor_flops / (p_tf32 * 1e12))
+    frac_step = t_roof / (ms_per_step * 1e-3)
 
     plan_fused = plan.fused
     # GPU outputs of the first transforms, for the accuracy check of the
@@ -687,9 +725,7 @@ def main():
                               "hbm_bytes_min": bytes_launch,
                               "tensor_flops": tensor_flops,
                               "tf32_peak_tflops": p_tf32,
-                              "tf32_peak_source": "%s bf16 x %.2f/%.2f nominal"
-                                                  % (peak_kind, NOMINAL_TF32,
-                                                     NOMINAL_BF16)},
+                              "tf32_peak_source": tf32_source},
             "cpu_baseline": cpu, "e2e": e2e,
             "accuracy": acc,
             "gpu": torch.cuda.get_device_name(dev),
