@@ -85,7 +85,7 @@ bool cols_map(CUtensorMap *m, const void *in, const tcu_dft2_plan_s *p) {
 }
 
 PRun dft2_pass(const tcu_dft2_plan_s *p, const PassPlan &pp, int di, const float2 *in,
-               float2 *out, bool scaled, const float2 *spec) {
+               float2 *out, bool scaled, const float2 *spec, int reverse = 0) {
   PRun g;
   memset(&g, 0, sizeof(g));
   g.in = in;
@@ -97,6 +97,7 @@ PRun dft2_pass(const tcu_dft2_plan_s *p, const PassPlan &pp, int di, const float
   g.last_img = scaled ? 2 * 16 * p->r * p->r : 0;
   g.spec = spec;
   g.spec_mask = p->n1 - 1;
+  g.reverse = reverse;
   return g;
 }
 
@@ -104,7 +105,8 @@ int run_dft2_pass(const tcu_dft2_plan_s *p, const PassPlan &pp, int di, const fl
                   float2 *out, bool scaled, const float2 *spec, cudaStream_t st) {
   GArgs g;
   memset(&g, 0, sizeof(g));
-  g.p[0] = dft2_pass(p, pp, di, in, out, scaled, spec);
+  // the row pass follows the column pass: items last to first (L2 reuse)
+  g.p[0] = dft2_pass(p, pp, di, in, out, scaled, spec, pp.role == kCols ? 0 : 1);
   if (pp.role == kCols && !cols_map(&g.tm_in, in, p)) return TCU_DFT_ERR_CUDA;
   g.bimg = p->bimg[di];
   g.err = p->err;
@@ -270,7 +272,7 @@ int tcu_conv2_exec(tcu_dft2_plan_t p, const void *in, const void *spectrum, void
   if (rc != TCU_DFT_OK) return rc;
   GArgs g;
   memset(&g, 0, sizeof(g));
-  g.p[0] = dft2_pass(p, p->rows, 0, p->scratch, p->scratch, false, (const float2 *)spectrum);
+  g.p[0] = dft2_pass(p, p->rows, 0, p->scratch, p->scratch, false, (const float2 *)spectrum, 1);
   g.p[1].tw_stage = p->rows.tw_stage[1];
   g.bimg = p->cimg;
   g.err = p->err;

@@ -149,6 +149,9 @@ struct PRun {
   // sub-transforms: the pointwise product of a circular convolution)
   const float2 *spec;
   long long spec_mask;
+  // process the items last to first: set on a pass that reads what the
+  // previous pass wrote, whose latest output is still in L2
+  int reverse;
 };
 
 struct GArgs {
@@ -889,7 +892,7 @@ struct StaticNext {
   bool issued;  // a copy for `next` is in flight
   __device__ void issue(const WG &w) {
     issued = next < nitems;
-    if (issued) issue_input<G>(P, tm, next, w);
+    if (issued) issue_input<G>(P, tm, P.reverse ? nitems - 1 - next : next, w);
   }
   __device__ void publish() {}
 };
@@ -923,13 +926,15 @@ __global__ void __launch_bounds__(
   const long long istride = (long long)gridDim.x * G::NTEAM;
   long long item = (long long)blockIdx.x * G::NTEAM + team;
   StaticNext<G> nx{P, &a.tm_in, item, nitems, false};
-  if (w.team_lead && item < nitems) issue_input<G>(P, &a.tm_in, item, w);
+  // item: position in this CTA's sequence; phys: the item processed there
+  auto phys = [&](long long i) { return P.reverse ? nitems - 1 - i : i; };
+  if (w.team_lead && item < nitems) issue_input<G>(P, &a.tm_in, phys(item), w);
   while (item < nitems && !w.fail) {
     nx.next = item + istride;
     if constexpr (CONV)
-      process_item_conv<G, PREC>(P, tw, tw_inv, item, w, nx);
+      process_item_conv<G, PREC>(P, tw, tw_inv, phys(item), w, nx);
     else
-      process_item<G, PREC, false>(P, &a.tm_tw, tw, item, w, nx);
+      process_item<G, PREC, false>(P, &a.tm_tw, tw, phys(item), w, nx);
     item += istride;
   }
   if (w.fail && w.rho == 0) atomicCAS(a.err, 0, TCU_DFT_ERR_TIMEOUT);
