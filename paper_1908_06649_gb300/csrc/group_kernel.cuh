@@ -53,9 +53,16 @@ enum Role { kSingle = 0, kFirst = 1, kSecond = 2, kCols = 3 };
 __host__ __device__ constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 16 ? 4 : 5); }
 // Warpgroups per CTA: TMEM holds 512 columns, a warpgroup's slot 3 Q of
 // them; a radix-16 first (strided) pass also stages its inter-pass twiddles
-// in SMEM, which leaves room for four.
-__host__ __device__ constexpr int pass_nwg(int R, int ROLE) {
-  return R == 32 ? 2 : (ROLE == 1 && R == 16 ? 4 : 5);
+// in SMEM, which leaves room for four.  A radix-32 pass of two stages runs
+// four warpgroups whose slots hold A for half of K (the products of a stage
+// in two K halves); one-stage radix-32 passes (already near the copy rate),
+// the convolution row pass and the fused schedule keep whole-K slots, two
+// per CTA at radix 32 (whole_k_nwg).
+__host__ __device__ constexpr int pass_nwg(int R, int ROLE, int S = 2) {
+  return R == 32 ? (S >= 2 ? 4 : 2) : (ROLE == 1 && R == 16 ? 4 : 5);
+}
+__host__ __device__ constexpr int whole_k_nwg(int R, int ROLE) {
+  return R == 32 ? 2 : pass_nwg(R, ROLE);
 }
 
 // Compile-time geometry of one pass: S stages of radix R.  A transform of
@@ -79,7 +86,7 @@ __host__ __device__ constexpr int pass_nwg(int R, int ROLE) {
 // the team shares the item's SMEM staging and transpose buffers and
 // synchronises on one named barrier.  TW > 1 lets an item hold sub-transforms
 // longer than 128 rows, or more columns of a strided pass.
-template <int R, int S, int LO, int ROLE, int LP = 0, int NWG_ = pass_nwg(R, ROLE),
+template <int R, int S, int LO, int ROLE, int LP = 0, int NWG_ = pass_nwg(R, ROLE, S),
           int TW_ = 1>
 struct Geo {
   static constexpr int LOG2R = log2_radix(R);
@@ -121,8 +128,11 @@ struct Geo {
   static constexpr int TWB = (TW2L && TW_SMEM) ? L : 0;  // SMEM row of table B
   static constexpr int TMA_ROWS = L < 256 ? L : 256;  // tensor box height
   static constexpr int Q = (2 * R > 32) ? 2 * R : 32;
-  // TMEM slot: A_hi (Q) | A_lo (Q) | D (Q)
-  static constexpr int GCOLS = 3 * Q;
+  // half-K products (radix 32, four warpgroups): A regions of Q/2 columns
+  static constexpr bool KS = R == 32 && NWG == 4 && TW == 1;
+  static constexpr int QA = KS ? Q / 2 : Q;
+  // TMEM slot: A_hi (QA) | A_lo (QA) | D (Q)
+  static constexpr int GCOLS = 2 * QA + Q;
   static constexpr int IMG_BYTES = 16 * R * R;
   // entries of the stage twiddle tables: sum over t < S of R * R^(S-t)
   static constexpr int TW_ENTRIES = S == 1 ? 0 : (S == 2 ? R * R : R * R * R + R * R);
@@ -184,7 +194,8 @@ __host__ __device__ constexpr int tw_stage_offset(int t) {
 // transpose buffer, input staging and twiddle staging | mbarriers (3 per
 // warpgroup: products, input staging, twiddle staging) | TMEM slot |
 // scheduler mailboxes.
-template <int R, int NWG, int TW1, int TW2, bool TWS, int TWB = 0, int TEAM = 1>
+template <int R, int NWG, int TW1, int TW2, bool TWS, int TWB = 0, int TEAM = 1,
+          bool SHARE = false>
 struct SmemLayout {
   static constexpr int NTEAM = NWG / TEAM;
   static constexpr size_t IMG = 4 * 16 * R * R;
@@ -192,7 +203,8 @@ struct SmemLayout {
   static constexpr size_t OFF_TW2 = OFF_TW1 + (size_t)TW1 * 8;
   static constexpr size_t PTS = 128 * (size_t)TEAM * R;  // points per item
   static constexpr size_t OFF_BUF = (OFF_TW2 + (size_t)TW2 * 8 + 127) / 128 * 128;
-  static constexpr size_t OFF_STG = OFF_BUF + (size_t)NTEAM * PTS * 8;
+  // SHARE: staging and transpose in one buffer (the half-K radix-32 items)
+  static constexpr size_t OFF_STG = OFF_BUF + (SHARE ? 0 : (size_t)NTEAM * PTS * 8);
   static constexpr size_t OFF_TWS = OFF_STG + (size_t)NTEAM * PTS * 8;
   static constexpr size_t TWS_BYTES = TWS ? (size_t)NTEAM * PTS * 8 : 0;
   static constexpr size_t OFF_TWB = OFF_TWS + TWS_BYTES;  // [k] row of table B
@@ -341,29 +353,36 @@ __device__ __forceinline__ void split_store8(const float2 *x, uint32_t col_hi,
 // K-blocks read the same TMEM columns of A_hi twice; D has N = 2r columns.
 // Each product covers 32 bytes of K: 8 fp32 (kind::tf32) or 16 bf16
 // (kind::f16), i.e. 8 TMEM columns of A and two 16-byte core matrices of B.
-template <int R, int PREC>
+//
+// HALF >= 0: only the products of K half HALF, with A (QA columns per
+// operand) holding that half; half 1 accumulates onto half 0.
+template <int R, int PREC, int QA = ((2 * R > 32) ? 2 * R : 32), int HALF = -1>
 __device__ __forceinline__ void issue_stage_mma(uint32_t slot, uint32_t img_addr) {
-  constexpr int Q = (2 * R > 32) ? 2 * R : 32;
   constexpr bool BF = is_bf16(PREC);
   constexpr int IMG = img_bytes(R, PREC), LBO = 128, SBO = (BF ? 32 : 64) * R;
   constexpr int KSTEPS = 2 * R / (BF ? 16 : 8);
+  constexpr int K0 = HALF < 0 ? 0 : HALF * (KSTEPS / 2);
+  constexpr int K1 = HALF < 0 ? KSTEPS : K0 + KSTEPS / 2;
   constexpr uint32_t idesc = BF ? idesc_bf16(128, 2 * R) : idesc_tf32(128, 2 * R);
-  const uint32_t ahi = slot, alo = slot + Q, d = slot + 2 * Q;
+  const uint32_t ahi = slot, alo = slot + QA, d = slot + 2 * QA;
   const uint32_t ihi = img_addr, ilo = img_addr + IMG;
-  uint32_t acc = 0;
+  uint32_t acc = HALF > 0 ? 1 : 0;
   if (is_split(PREC)) {
 #pragma unroll
-    for (int kk = 0; kk < KSTEPS; ++kk) {
-      mma_ts<BF>(d, alo + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO), idesc, acc);
+    for (int kk = K0; kk < K1; ++kk) {
+      mma_ts<BF>(d, alo + 8 * (kk - K0), smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO), idesc,
+                 acc);
       acc = 1;
     }
 #pragma unroll
-    for (int kk = 0; kk < KSTEPS; ++kk)
-      mma_ts<BF>(d, ahi + 8 * kk, smem_desc_noswz(ilo + kk * 2 * LBO, LBO, SBO), idesc, 1);
+    for (int kk = K0; kk < K1; ++kk)
+      mma_ts<BF>(d, ahi + 8 * (kk - K0), smem_desc_noswz(ilo + kk * 2 * LBO, LBO, SBO), idesc,
+                 1);
   }
 #pragma unroll
-  for (int kk = 0; kk < KSTEPS; ++kk) {
-    mma_ts<BF>(d, ahi + 8 * kk, smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO), idesc, acc);
+  for (int kk = K0; kk < K1; ++kk) {
+    mma_ts<BF>(d, ahi + 8 * (kk - K0), smem_desc_noswz(ihi + kk * 2 * LBO, LBO, SBO), idesc,
+               acc);
     acc = 1;
   }
 }
@@ -372,7 +391,7 @@ __device__ __forceinline__ void issue_stage_mma(uint32_t slot, uint32_t img_addr
 template <class G, int PREC>
 __device__ __forceinline__ void load_d_row(const WG &w, float *d) {
   constexpr int R = 1 << G::LOG2R;
-  const uint32_t base = w.slot + 2 * G::Q + w.lane_off;
+  const uint32_t base = w.slot + 2 * G::QA + w.lane_off;
   if (R == 8) {
     tmem_ld16(base, d);
   } else if (R == 16) {
@@ -685,6 +704,136 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
   last_stage_store<G, PREC, OUT_L2>(P, item, w);
 }
 
+// ---- half-K items (radix 32, four warpgroups).  A warpgroup's TMEM slot
+// holds A for one half of K (A_hi, A_lo: QA columns each) and the whole D,
+// so four slots fit the 512 columns where whole-K slots fit two.  Each
+// stage runs its products in two K halves: the rows' first R/2 values go
+// into A, the products of that half are issued, and once they have read A
+// the second R/2 values replace them and the second half accumulates onto
+// D.  Staging and transpose share one buffer, so the next item's copy is
+// issued once the last transpose has been read.
+
+// Products of one K half (warp 0, converged; one elected lane).
+template <int R, int PREC, int QA>
+__device__ __forceinline__ void issue_stage_half(int h, uint32_t slot, uint32_t img_addr,
+                                                 uint32_t bar_mma) {
+  if (elect_one()) {
+    if (h == 0)
+      issue_stage_mma<R, PREC, QA, 0>(slot, img_addr);
+    else
+      issue_stage_mma<R, PREC, QA, 1>(slot, img_addr);
+    mma_commit(bar_mma);
+  }
+  __syncwarp();
+}
+
+// Values h R/2 .. (h+1) R/2 - 1 of this thread's stage-1 row.
+template <class G>
+__device__ __forceinline__ void staged_row_half(const WG &w, float2 *x, int h) {
+  constexpr int R = 1 << G::LOG2R, H = R / 2;
+  int ul, q;
+  row_of<G>(G::MODE_FIRST, w.rho, ul, q);
+  constexpr int JS = 1 << (G::LOG2L - G::LOG2R);  // a = j * R^(S-1) + q
+  const float2 zero = make_float2(0.f, 0.f);
+  const int i0 = G::MODE_FIRST == kUF ? q * G::GG + ul : (ul << G::LOG2L) + q;
+  constexpr int JST = G::MODE_FIRST == kUF ? JS * G::GG : JS;
+#pragma unroll
+  for (int j = 0; j < H; ++j) {
+    const int i = i0 + (h * H + j) * JST;
+    x[j] = in_range(w, i, G::GPTS) ? w.stg[i] : zero;
+  }
+}
+
+// Values h R/2 .. (h+1) R/2 - 1 of this thread's stage-T row, from the
+// transpose buffer into the half-K A region.
+template <class G, int PREC, int T>
+__device__ __forceinline__ void stage_rows_half(const PRun &P, const WG &w, int h) {
+  constexpr int R = 1 << G::LOG2R, H = R / 2;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  constexpr int SH = G::LOG2R * (S - T);
+  int ul, q;
+  row_of<G>(T == S ? G::MODE_LAST : G::MODE_MID, w.rho, ul, q);
+  const int hi = q >> SH, lo = q & ((1 << SH) - 1);
+  const int base = (ul << G::LOG2L) + (hi << (SH + G::LOG2R)) + lo;
+  const uint32_t tabv = (uint32_t)(P.swz_tab >> (4 * (ul & 15))) & 15u;
+#pragma unroll
+  for (int c = 0; c < H; c += 8) {
+    float2 row[8];
+#pragma unroll
+    for (int jj = 0; jj < 8; ++jj) {
+      const int bi = gswz<(G::LOG2L > 8)>(base + ((h * H + c + jj) << SH), tabv);
+      row[jj] = in_range(w, bi, G::GPTS) ? w.buf[bi] : make_float2(0.f, 0.f);
+    }
+    split_store8<PREC>(row, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
+                       w.slot + G::QA + w.lane_off + a_cols8(PREC) * c / 8);
+  }
+}
+
+template <class G, int PREC, class Mid>
+__device__ __forceinline__ void process_item_ks(const PRun &P, const float2 *tws,
+                                                long long item, WG &w, Mid &mid) {
+  constexpr int R = 1 << G::LOG2R, H = R / 2;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  static_assert(G::KS && S <= 2 && !G::TW_SMEM, "half-K items: radix 32, at most two stages");
+  if (!mbar_wait_bounded(w.bar_stg, w.ph_stg)) w.fail = true;
+  w.ph_stg ^= 1;
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    {
+      float2 x[H];
+      staged_row_half<G>(w, x, h);
+#pragma unroll
+      for (int c = 0; c < H; c += 8)
+        split_store8<PREC>(x + c, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
+                           w.slot + G::QA + w.lane_off + a_cols8(PREC) * c / 8);
+    }
+    tmem_wait_st();
+    fence_before_sync();
+    if (named_bar_or(w.bar_id, w.bar_count, w.fail)) {
+      w.fail = true;
+      return;
+    }
+    if (w.wg_lead) {
+      fence_after_sync();
+      issue_stage_half<R, PREC, G::QA>(h, w.slot, w.img_addr + (S == 1 ? P.last_img : 0),
+                                       w.bar_mma);
+    }
+    // one stage: the staging has been read and no transpose follows
+    if (S == 1 && h == 1 && w.team_lead) mid.issue(w);
+    if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
+    w.ph_mma ^= 1;
+    fence_after_sync();
+  }
+  if constexpr (S == 2) {
+    stage_epilogue<G, PREC, 1>(P, tws, w);
+    if (w.team_lead) mid.publish();
+    fence_before_sync();
+    named_bar_or(w.bar_id, w.bar_count, false);
+#pragma unroll
+    for (int h = 0; h < 2; ++h) {
+      stage_rows_half<G, PREC, 2>(P, w, h);
+      tmem_wait_st();
+      fence_before_sync();
+      if (named_bar_or(w.bar_id, w.bar_count, w.fail)) {
+        w.fail = true;
+        return;
+      }
+      if (w.wg_lead) {
+        fence_after_sync();
+        issue_stage_half<R, PREC, G::QA>(h, w.slot, w.img_addr + P.last_img, w.bar_mma);
+      }
+      // the transpose buffer (shared with the staging) has been read
+      if (h == 1 && w.team_lead) mid.issue(w);
+      if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
+      w.ph_mma ^= 1;
+      fence_after_sync();
+    }
+  } else {
+    if (w.team_lead) mid.publish();
+  }
+  last_stage_store<G, PREC, false>(P, item, w);
+}
+
 // Convolution row item (kSingle geometry): the forward transform of each
 // row, the product with the spectrum, and the inverse transform, all on chip.
 // The thread that holds forward outputs k = klow + j r^(S-1) of a row after
@@ -892,19 +1041,22 @@ struct StaticNext {
   bool issued;  // a copy for `next` is in flight
   __device__ void issue(const WG &w) {
     issued = next < nitems;
-    if (issued) issue_input<G>(P, tm, P.reverse ? nitems - 1 - next : next, w);
+    if (issued) issue_input<G>(P, tm, G::TW == 1 && P.reverse ? nitems - 1 - next : next, w);
   }
   __device__ void publish() {}
 };
 
 template <int R, int PREC, int S, int LO, int ROLE, int LP, bool CONV = false, int TW = 1>
 __global__ void __launch_bounds__(
-    Geo<R, S, LO, ROLE, LP, TW == 1 ? pass_nwg(R, ROLE) : 4, TW>::THREADS, 1)
-    dft_pass_kernel(const __grid_constant__ GArgs a) {
-  using G = Geo<R, S, LO, ROLE, LP, TW == 1 ? pass_nwg(R, ROLE) : 4, TW>;
+    Geo<R, S, LO, ROLE, LP,
+        TW == 1 ? (CONV ? whole_k_nwg(R, ROLE) : pass_nwg(R, ROLE, S)) : 4, TW>::THREADS,
+    1) dft_pass_kernel(const __grid_constant__ GArgs a) {
+  using G =
+      Geo<R, S, LO, ROLE, LP, TW == 1 ? (CONV ? whole_k_nwg(R, ROLE) : pass_nwg(R, ROLE, S)) : 4,
+          TW>;
   static_assert(!CONV || ROLE == kSingle, "convolution rows are whole transforms");
   using SM = SmemLayout<R, G::NWG, G::TW_ENTRIES, CONV ? G::TW_ENTRIES : 0, G::TW_SMEM, G::TWB,
-                        TW>;
+                        TW, G::KS>;
   extern __shared__ __align__(1024) unsigned char smem[];
   float2 *tw = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
   float2 *tw_inv = reinterpret_cast<float2 *>(smem + SM::OFF_TW2);
@@ -927,12 +1079,15 @@ __global__ void __launch_bounds__(
   long long item = (long long)blockIdx.x * G::NTEAM + team;
   StaticNext<G> nx{P, &a.tm_in, item, nitems, false};
   // item: position in this CTA's sequence; phys: the item processed there
-  auto phys = [&](long long i) { return P.reverse ? nitems - 1 - i : i; };
+  // (team passes always run forward: no reversal code in them)
+  auto phys = [&](long long i) { return TW == 1 && P.reverse ? nitems - 1 - i : i; };
   if (w.team_lead && item < nitems) issue_input<G>(P, &a.tm_in, phys(item), w);
   while (item < nitems && !w.fail) {
     nx.next = item + istride;
     if constexpr (CONV)
       process_item_conv<G, PREC>(P, tw, tw_inv, phys(item), w, nx);
+    else if constexpr (G::KS)
+      process_item_ks<G, PREC>(P, tw, phys(item), w, nx);
     else
       process_item<G, PREC, false>(P, &a.tm_tw, tw, phys(item), w, nx);
     item += istride;
@@ -1124,10 +1279,11 @@ struct FusedNext {
 };
 
 template <int R, int PREC, int S1, int S2>
-__global__ void __launch_bounds__(Geo<R, S1, log2_radix(R) * S2, kFirst>::THREADS, 1)
+__global__ void __launch_bounds__(
+    Geo<R, S1, log2_radix(R) * S2, kFirst, 0, whole_k_nwg(R, kFirst)>::THREADS, 1)
     dft_fused_kernel(const __grid_constant__ GArgs a) {
   static_assert(S1 >= 2 && S2 >= 2, "the fused schedule needs an SMEM barrier per item");
-  using G1 = Geo<R, S1, log2_radix(R) * S2, kFirst>;
+  using G1 = Geo<R, S1, log2_radix(R) * S2, kFirst, 0, whole_k_nwg(R, kFirst)>;
   using G2 = Geo<R, S2, log2_radix(R) * S1, kSecond, 0, G1::NWG>;
   using SM = SmemLayout<R, G1::NWG, G1::TW_ENTRIES, G2::TW_ENTRIES, G1::TW_SMEM, G1::TWB>;
   constexpr int NWG = G1::NWG;

@@ -8,7 +8,8 @@ namespace tcu {
 template <int R, int PREC, int S, int LO, int ROLE, int LP>
 cudaError_t launch_pass_t(const GArgs &a, int num_sms, cudaStream_t st) {
   using G = Geo<R, S, LO, ROLE, LP>;
-  const size_t sm = SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM, G::TWB>::BYTES;
+  const size_t sm =
+      SmemLayout<R, G::NWG, G::TW_ENTRIES, 0, G::TW_SMEM, G::TWB, 1, G::KS>::BYTES;
   cudaError_t e = cudaFuncSetAttribute(dft_pass_kernel<R, PREC, S, LO, ROLE, LP>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)sm);
@@ -48,7 +49,7 @@ cudaError_t launch_team_t(const GArgs &a, int num_sms, cudaStream_t st) {
 // The convolution row pass (forward rows, spectrum product, inverse rows).
 template <int R, int PREC, int S>
 cudaError_t launch_rowconv_t(const GArgs &a, int num_sms, cudaStream_t st) {
-  using G = Geo<R, S, 0, kSingle>;
+  using G = Geo<R, S, 0, kSingle, 0, whole_k_nwg(R, kSingle)>;
   const size_t sm = SmemLayout<R, G::NWG, G::TW_ENTRIES, G::TW_ENTRIES, false, 0>::BYTES;
   cudaError_t e = cudaFuncSetAttribute(dft_pass_kernel<R, PREC, S, 0, kSingle, 0, true>,
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -68,7 +69,7 @@ cudaError_t launch_rowconv_t(const GArgs &a, int num_sms, cudaStream_t st) {
 
 template <int R, int PREC, int S1, int S2>
 cudaError_t launch_fused_t(const GArgs &a, int num_sms, cudaStream_t st) {
-  using G1 = Geo<R, S1, log2_radix(R) * S2, kFirst>;
+  using G1 = Geo<R, S1, log2_radix(R) * S2, kFirst, 0, whole_k_nwg(R, kFirst)>;
   using G2 = Geo<R, S2, log2_radix(R) * S1, kSecond, 0, G1::NWG>;
   const size_t sm =
       SmemLayout<R, G1::NWG, G1::TW_ENTRIES, G2::TW_ENTRIES, G1::TW_SMEM, G1::TWB>::BYTES;
