@@ -24,6 +24,14 @@
 // small tables) applied on the way.  The inverse's 1/n is folded, exactly,
 // into a 2^-log2(n)-scaled copy of F_r used by the last stage.
 //
+// Radix-32 passes of two stages run half-K items: a slot holds A for half
+// of K, each stage's products run in two K halves, and staging and
+// transpose share one buffer (so the next item's copy is issued after the
+// last transpose read); four warpgroups then fit TMEM where whole-K slots
+// fit two.  Every second pass of a plan processes its items last to first,
+// starting on the part of its input the previous pass wrote last, which is
+// still in L2.
+//
 // The whole geometry of a pass (radix, stages, other-side size, role, prefix,
 // team) is a template parameter, so every stride is a compile-time constant.
 //
