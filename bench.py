@@ -429,7 +429,8 @@ def run_grid(args):
         Nt = 1
         while Nt < 3 * k or Nt * Nt < 128 * r:
             Nt *= r
-        tiles = (side // k) ** 2
+        B = Nt - 2 * k                     # output block side per tile
+        tiles = (-(-side // B)) ** 2
         points = tiles * Nt * Nt
         passes = 3
         # weights: place, 2-D DFT (2), power, inverse (2); kernel W': place,
@@ -439,11 +440,12 @@ def run_grid(args):
         metric = ("linear stencil grid-point updates/s (side^2 x steps), "
                   "%d^2 grid x %d steps, 1xGB300" % (side, k))
         config = {"workload": "linear 3x3 stencil (heat update) on a %dx%d fp32 "
-                              "grid for %d steps via Lemma 1 tiles (%d tiles of "
-                              "%dx%d) and Lemma 2 weights, %s" % (
-                                  side, side, k, tiles, Nt, Nt,
+                              "grid for %d steps via Lemma 1 windows (%d tiles of "
+                              "%dx%d, each giving a %dx%d output block) and Lemma 2 "
+                              "weights, %s" % (
+                                  side, side, k, tiles, Nt, Nt, B, B,
                                   "3xTF32" if args.precision == 3 else "TF32"),
-                  "side": side, "steps": k, "sqrt_m": r, "tile": Nt,
+                  "side": side, "steps": k, "sqrt_m": r, "tile": Nt, "block": B,
                   "l2": "grid %d MiB, but every step streams the %d MiB tile "
                         "batch through HBM three times, which evicts it; no "
                         "flush" % (side * side * 4 >> 20, points * 8 >> 20)}

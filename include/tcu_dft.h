@@ -239,14 +239,18 @@ int tcu_dft2_destroy(tcu_dft2_plan_t p);                /* NULL: no-op, OK */
  * tcu_stencil_weights: W ((2k+1)^2 fp32, device) as the coefficients of
  *   P(x,y)^k (Lemma 2): P on an Nw x Nw grid, 2-D DFT, pointwise k-th power,
  *   inverse 2-D DFT, Nw the smallest power of sqrt_m >= 2k + 1.
- * tcu_stencil_exec: Lemma 1 -- the (side/k)^2 tiles A'_{r,c} (3k x 3k,
- *   zero-padded to N x N, N the smallest power of sqrt_m >= 3k) convolved
- *   with the flipped, padded W as ONE batch, centres written to A_k (device,
- *   side^2 fp32; A_k == A allowed).
- * Needs side % k == 0 and N, Nw within one warpgroup pass (k <= 85 for
- * sqrt_m 16, 170 for 8, 341 for 32); else ERR_UNSUPPORTED.  The plan
- * allocates (side/k)^2 N^2 complex64 of tiles plus tables; the calls are
- * asynchronous on `stream` and allocate nothing.  w3x3 is a host array. */
+ * tcu_stencil_exec: Lemma 1 -- output blocks of B x B points, B = N - 2k,
+ *   N the smallest power of sqrt_m >= 3k: the (B + 2k) x (B + 2k) input
+ *   window of every block (Lemma 1's 3k x 3k tile A'_{r,c} when B = k),
+ *   zero-padded to N x N, convolved with the flipped, padded W as ONE batch,
+ *   the B x B centres written to A_k (device, side^2 fp32; A_k == A
+ *   allowed).  The result is the same for every B <= N - 2k; the largest
+ *   makes the fewest tiles.
+ * Needs N, Nw within one warpgroup pass (k <= 85 for sqrt_m 16, 170 for 8,
+ * 341 for 32); else ERR_UNSUPPORTED.  Any side >= 1 (the last blocks of a
+ * row or column are cut).  The plan allocates ceil(side/B)^2 N^2 complex64
+ * of tiles plus tables; the calls are asynchronous on `stream` and allocate
+ * nothing.  w3x3 is a host array. */
 typedef struct tcu_stencil_plan_s *tcu_stencil_plan_t;
 tcu_stencil_plan_t tcu_stencil_plan(int64_t side, int32_t steps, int32_t sqrt_m,
                                     int32_t precision);

@@ -75,36 +75,41 @@ __global__ void place_kernel_kernel(float2 *w, long long N, const float2 *g, lon
 }
 
 // Tile (r, c) of the side x side grid A as the N x N complex array whose
-// top-left 3k x 3k block is A'_{r,c} = A[(r-1)k .. (r+2)k)[(c-1)k .. (c+2)k)
-// (zero outside A) and whose other entries are 0.  One block per tile,
-// 32 x 8 threads: rows by threadIdx.y, columns by threadIdx.x, so reads of A
-// and writes of the tile are contiguous along the columns.
+// top-left (B + 2k) x (B + 2k) block is the window A[rB - k .. rB + B + k)
+// [cB - k .. cB + B + k) (zero outside A) and whose other entries are 0: the
+// input of output block (r, c) of B x B points.  B = k is Lemma 1's tile
+// A'_{r,c} (3k x 3k); the plan takes B = N - 2k, the largest block whose
+// window still fits N without wrapping.  One block per tile, 32 x 8
+// threads: rows by threadIdx.y, columns by threadIdx.x, so reads of A and
+// writes of the tile are contiguous along the columns.
 __global__ void gather_tiles_kernel(float2 *tiles, const float *A, long long side, int k,
-                                    int N, long long tpr) {
+                                    int N, int B, long long tpr) {
   const long long t = blockIdx.x;
-  const long long r0 = (t / tpr - 1) * k, c0 = (t % tpr - 1) * k;
+  const long long r0 = (t / tpr) * B - k, c0 = (t % tpr) * B - k;
+  const int win = B + 2 * k;
   float2 *dst = tiles + t * N * N;
   for (int i = threadIdx.y; i < N; i += blockDim.y) {
     const long long gi = r0 + i;
-    const bool row_in = i < 3 * k && gi >= 0 && gi < side;
+    const bool row_in = i < win && gi >= 0 && gi < side;
     for (int j = threadIdx.x; j < N; j += blockDim.x) {
       const long long gj = c0 + j;
       float v = 0.f;
-      if (row_in && j < 3 * k && gj >= 0 && gj < side) v = __ldg(A + gi * side + gj);
+      if (row_in && j < win && gj >= 0 && gj < side) v = __ldg(A + gi * side + gj);
       __stcs(dst + (long long)i * N + j, make_float2(v, 0.f));
     }
   }
 }
 
-// A_k[rk + i][ck + j] = Re tile_{r,c}[k + i][k + j] for i, j < k: one block
-// per tile, contiguous along the columns.
+// A_k[rB + i][cB + j] = Re tile_{r,c}[k + i][k + j] for i, j < B inside the
+// grid (the last blocks of a row or column may be cut): one block per tile,
+// contiguous along the columns.
 __global__ void extract_tiles_kernel(float *Ak, const float2 *tiles, long long side, int k,
-                                     int N, long long tpr) {
+                                     int N, int B, long long tpr) {
   const long long t = blockIdx.x;
-  const long long r0 = (t / tpr) * k, c0 = (t % tpr) * k;
+  const long long r0 = (t / tpr) * B, c0 = (t % tpr) * B;
   const float2 *src = tiles + t * N * N + (long long)k * N + k;
-  for (int i = threadIdx.y; i < k; i += blockDim.y)
-    for (int j = threadIdx.x; j < k; j += blockDim.x)
+  for (int i = threadIdx.y; i < B && r0 + i < side; i += blockDim.y)
+    for (int j = threadIdx.x; j < B && c0 + j < side; j += blockDim.x)
       Ak[(r0 + i) * side + c0 + j] = __ldcs(src + (long long)i * N + j).x;
 }
 
@@ -142,18 +147,18 @@ cudaError_t launch_place_kernel(float2 *w, long long N, const float2 *g, long lo
 }
 
 cudaError_t launch_gather_tiles(float2 *tiles, const float *A, long long side, int k,
-                                long long N, int num_sms, cudaStream_t st) {
-  const long long tpr = side / k;
+                                long long N, int B, int num_sms, cudaStream_t st) {
+  const long long tpr = (side + B - 1) / B;
   gather_tiles_kernel<<<(unsigned)(tpr * tpr), dim3(32, 8), 0, st>>>(tiles, A, side, k, (int)N,
-                                                                    tpr);
+                                                                    B, tpr);
   return cudaGetLastError();
 }
 
 cudaError_t launch_extract_tiles(float *Ak, const float2 *tiles, long long side, int k,
-                                 long long N, int num_sms, cudaStream_t st) {
-  const long long tpr = side / k;
+                                 long long N, int B, int num_sms, cudaStream_t st) {
+  const long long tpr = (side + B - 1) / B;
   extract_tiles_kernel<<<(unsigned)(tpr * tpr), dim3(32, 8), 0, st>>>(Ak, tiles, side, k,
-                                                                     (int)N, tpr);
+                                                                     (int)N, B, tpr);
   return cudaGetLastError();
 }
 

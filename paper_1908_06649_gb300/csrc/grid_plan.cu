@@ -39,6 +39,7 @@ struct tcu_dft2_plan_s {
 
 struct tcu_stencil_plan_s {
   long long side, N, Nw, tiles;
+  int B;  // output block side: N - 2k (Lemma 1's tiles are blocks of k)
   int k, r, precision, num_sms;
   tcu_dft2_plan_t conv;   // N x N, batch = tiles
   tcu_dft2_plan_t wconv;  // N x N, batch 1 (spectrum of the kernel)
@@ -315,11 +316,15 @@ tcu_stencil_plan_t tcu_stencil_plan(int64_t side, int32_t steps, int32_t sqrt_m,
   }
   const long long N = (sqrt_m == 8 || sqrt_m == 16 || sqrt_m == 32) ? grid_side(sqrt_m, 3ll * steps) : 0;
   const long long Nw = N ? grid_side(sqrt_m, 2ll * steps + 1) : 0;
-  if (!N || !Nw || side % steps != 0) {
+  if (!N || !Nw) {
     g_last_error = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
   }
-  const long long tpr = side / steps;
+  // output blocks of B = N - 2k >= k points a side: the (B + 2k)^2 input
+  // window of a block fits the N x N tile without wrapping (Lemma 1 is
+  // B = k); the last blocks of a row may be cut
+  const int B = (int)(N - 2ll * steps);
+  const long long tpr = (side + B - 1) / B;
   tcu_stencil_plan_s *p = new tcu_stencil_plan_s();
   memset(p, 0, sizeof(*p));
   p->side = side;
@@ -328,6 +333,7 @@ tcu_stencil_plan_t tcu_stencil_plan(int64_t side, int32_t steps, int32_t sqrt_m,
   p->precision = precision;
   p->N = N;
   p->Nw = Nw;
+  p->B = B;
   p->tiles = tpr * tpr;
   int rc = TCU_DFT_OK;
   p->conv = make_dft2(N, N, p->tiles, sqrt_m, precision, rc);
@@ -389,12 +395,14 @@ int tcu_stencil_exec(tcu_stencil_plan_t p, const float *w3x3, const float *A, fl
     return TCU_DFT_ERR_CUDA;
   rc = tcu_dft2_exec(p->wconv, p->wker, p->wker, TCU_DFT_FORWARD, st);
   if (rc != TCU_DFT_OK) return rc;
-  // Lemma 1: all tiles A'_{r,c} as one batch, circular convolution, centres
-  if (launch_gather_tiles(p->tile_buf, A, p->side, p->k, p->N, p->num_sms, st) != cudaSuccess)
+  // Lemma 1: every block's input window as one batch of tiles, circular
+  // convolution, the B x B centres
+  if (launch_gather_tiles(p->tile_buf, A, p->side, p->k, p->N, p->B, p->num_sms, st) !=
+      cudaSuccess)
     return TCU_DFT_ERR_CUDA;
   rc = tcu_conv2_exec(p->conv, p->tile_buf, p->wker, p->tile_buf, st);
   if (rc != TCU_DFT_OK) return rc;
-  if (launch_extract_tiles(Ak, p->tile_buf, p->side, p->k, p->N, p->num_sms, st) !=
+  if (launch_extract_tiles(Ak, p->tile_buf, p->side, p->k, p->N, p->B, p->num_sms, st) !=
       cudaSuccess)
     return TCU_DFT_ERR_CUDA;
   return debug_exec() ? tcu_stencil_check(p, stream) : TCU_DFT_OK;

@@ -48,9 +48,9 @@ cudaError_t launch_extract_weights(float *W, const float2 *g, long long Nw, int 
 cudaError_t launch_place_kernel(float2 *w, long long N, const float2 *g, long long Nw, int k,
                                 int num_sms, cudaStream_t st);
 cudaError_t launch_gather_tiles(float2 *tiles, const float *A, long long side, int k,
-                                long long N, int num_sms, cudaStream_t st);
+                                long long N, int B, int num_sms, cudaStream_t st);
 cudaError_t launch_extract_tiles(float *Ak, const float2 *tiles, long long side, int k,
-                                 long long N, int num_sms, cudaStream_t st);
+                                 long long N, int B, int num_sms, cudaStream_t st);
 
 // The q-point first pass of a mixed-radix transform (grid_kernels.cu).
 struct RootsQ {

@@ -119,7 +119,12 @@ def test_stencil_weights(pkg, r, k):
     plan.destroy()
 
 
-@pytest.mark.parametrize("r,side,k", [(8, 64, 4), (8, 96, 8), (16, 128, 16), (8, 120, 20)])
+# output blocks of N - 2k points: (8, 64, 4) one 56-block cut at 8, (8, 96, 8)
+# blocks of 48, (16, 128, 16) and (8, 120, 20) blocks of 224 and 24, and
+# sides that no block size divides: 100 with k = 6 (blocks of 52), 130 with
+# k = 16 (blocks of 224: one cut block), 37 with k = 5 (blocks of 54)
+@pytest.mark.parametrize("r,side,k", [(8, 64, 4), (8, 96, 8), (16, 128, 16), (8, 120, 20),
+                                      (8, 100, 6), (16, 130, 16), (8, 37, 5)])
 def test_stencil_apply(pkg, r, side, k):
     import torch
     rng = np.random.default_rng(side + k)
