@@ -327,7 +327,7 @@ GRID = {
     # uses, and the stencil itself (Sec. 4.6, Lemmas 1-2)
     "dft2": {"n1": 256, "n2": 256, "batch": 4096, "sqrt_m": 16, "seed": 5},
     "conv2": {"n1": 256, "n2": 256, "batch": 4096, "sqrt_m": 16, "seed": 6},
-    "stencil": {"side": 4096, "steps": 16, "sqrt_m": 8, "seed": 7},
+    "stencil": {"side": 4096, "steps": 16, "sqrt_m": 16, "seed": 7},
 }
 HEAT3 = [[0.0, 0.1, 0.0], [0.15, 0.5, 0.15], [0.0, 0.1, 0.0]]
 
@@ -426,11 +426,8 @@ def run_grid(args):
         out = torch.empty_like(A)
         plan = pkg.StencilPlan(side, k, r, args.precision)
         step = lambda: plan.apply(A, out, w3x3=HEAT3)
-        Nt = 1
-        while Nt < 3 * k or Nt * Nt < 128 * r:
-            Nt *= r
-        B = Nt - 2 * k                     # output block side per tile
-        tiles = (-(-side // B)) ** 2
+        # the plan's tiling: tiles of Nt x Nt, each giving a B x B output block
+        tiles, Nt, B = pkg.stencil_tiles(side, k, r)
         points = tiles * Nt * Nt
         passes = 3
         # weights: place, 2-D DFT (2), power, inverse (2); kernel W': place,

@@ -240,7 +240,8 @@ int tcu_dft2_destroy(tcu_dft2_plan_t p);                /* NULL: no-op, OK */
  *   P(x,y)^k (Lemma 2): P on an Nw x Nw grid, 2-D DFT, pointwise k-th power,
  *   inverse 2-D DFT, Nw the smallest power of sqrt_m >= 2k + 1.
  * tcu_stencil_exec: Lemma 1 -- output blocks of B x B points, B = N - 2k,
- *   N the smallest power of sqrt_m >= 3k: the (B + 2k) x (B + 2k) input
+ *   N the smallest power of sqrt_m >= 3k (tcu_stencil_tiles): the (B + 2k) x
+ *   (B + 2k) input
  *   window of every block (Lemma 1's 3k x 3k tile A'_{r,c} when B = k),
  *   zero-padded to N x N, convolved with the flipped, padded W as ONE batch,
  *   the B x B centres written to A_k (device, side^2 fp32; A_k == A
@@ -258,6 +259,13 @@ int tcu_stencil_weights(tcu_stencil_plan_t p, const float *w3x3, float *W, void 
 int tcu_stencil_exec(tcu_stencil_plan_t p, const float *w3x3, const float *A, float *Ak,
                      void *stream);
 int tcu_stencil_check(tcu_stencil_plan_t p, void *stream);
+/* The tiling tcu_stencil_plan would choose, without a plan or a GPU: the
+ * number of tiles ceil(side / B)^2 (0 if the arguments are unsupported), the
+ * tile side N (the smallest power of sqrt_m with N >= 3k and N^2 >=
+ * 128 sqrt_m, one warpgroup pass per axis) and the output block side
+ * B = N - 2k, written to *tile and *block (either may be NULL). */
+int64_t tcu_stencil_tiles(int64_t side, int32_t steps, int32_t sqrt_m, int64_t *tile,
+                          int64_t *block);
 int tcu_stencil_destroy(tcu_stencil_plan_t p);
 
 /* Failure-detection self-test (not a transform): runs a fused plan's

@@ -47,6 +47,7 @@ SYMBOLS = (
     "tcu_dft2_plan", "tcu_dft2_exec", "tcu_conv2_exec", "tcu_dft2_check",
     "tcu_dft2_destroy", "tcu_stencil_plan", "tcu_stencil_weights",
     "tcu_stencil_exec", "tcu_stencil_check", "tcu_stencil_destroy",
+    "tcu_stencil_tiles",
 )
 
 _lib = None
@@ -107,6 +108,9 @@ def lib():
     L.tcu_dft_num_passes.restype = ctypes.c_int
     L.tcu_dft_plan_passes.argtypes = [i64, i32, ctypes.POINTER(ctypes.c_int32)]
     L.tcu_dft_plan_passes.restype = ctypes.c_int
+    L.tcu_stencil_tiles.argtypes = [i64, i32, i32, ctypes.POINTER(ctypes.c_int64),
+                                    ctypes.POINTER(ctypes.c_int64)]
+    L.tcu_stencil_tiles.restype = ctypes.c_int64
     L.tcu_dft_pass_stages.argtypes = [vp, ctypes.c_int]
     L.tcu_dft_pass_stages.restype = ctypes.c_int
     L.tcu_dft_last_error.argtypes = []
@@ -142,6 +146,16 @@ def plan_passes(n: int, sqrt_m: int = 16):
     st = (ctypes.c_int32 * 3)()
     np_ = lib().tcu_dft_plan_passes(int(n), int(sqrt_m), st)
     return [int(st[i]) for i in range(np_)]
+
+
+def stencil_tiles(side: int, steps: int, sqrt_m: int = 16):
+    """(tiles, tile side N, output block side B) that tcu_stencil_plan would
+    choose; tiles = 0 if unsupported.  Host only: needs no GPU."""
+    N = ctypes.c_int64(0)
+    B = ctypes.c_int64(0)
+    t = lib().tcu_stencil_tiles(int(side), int(steps), int(sqrt_m), ctypes.byref(N),
+                                ctypes.byref(B))
+    return int(t), int(N.value), int(B.value)
 
 
 def strerror(status: int) -> str:

@@ -79,16 +79,20 @@ __global__ void place_kernel_kernel(float2 *w, long long N, const float2 *g, lon
 // [cB - k .. cB + B + k) (zero outside A) and whose other entries are 0: the
 // input of output block (r, c) of B x B points.  B = k is Lemma 1's tile
 // A'_{r,c} (3k x 3k); the plan takes B = N - 2k, the largest block whose
-// window still fits N without wrapping.  One block per tile, 32 x 8
-// threads: rows by threadIdx.y, columns by threadIdx.x, so reads of A and
-// writes of the tile are contiguous along the columns.
+// window still fits N without wrapping.  Blocks of 32 x 8 threads, one per
+// tile (blockIdx.x) and chunk of kRowChunk tile rows (blockIdx.y): rows by
+// threadIdx.y, columns by threadIdx.x, so reads of A and writes of the tile
+// are contiguous along the columns.
+constexpr int kRowChunk = 64;
+
 __global__ void gather_tiles_kernel(float2 *tiles, const float *A, long long side, int k,
                                     int N, int B, long long tpr) {
   const long long t = blockIdx.x;
   const long long r0 = (t / tpr) * B - k, c0 = (t % tpr) * B - k;
   const int win = B + 2 * k;
   float2 *dst = tiles + t * N * N;
-  for (int i = threadIdx.y; i < N; i += blockDim.y) {
+  const int i1 = min(N, (int)(blockIdx.y + 1) * kRowChunk);
+  for (int i = blockIdx.y * kRowChunk + threadIdx.y; i < i1; i += blockDim.y) {
     const long long gi = r0 + i;
     const bool row_in = i < win && gi >= 0 && gi < side;
     for (int j = threadIdx.x; j < N; j += blockDim.x) {
@@ -101,14 +105,15 @@ __global__ void gather_tiles_kernel(float2 *tiles, const float *A, long long sid
 }
 
 // A_k[rB + i][cB + j] = Re tile_{r,c}[k + i][k + j] for i, j < B inside the
-// grid (the last blocks of a row or column may be cut): one block per tile,
-// contiguous along the columns.
+// grid (the last blocks of a row or column may be cut): one thread block per
+// tile and chunk of kRowChunk block rows, contiguous along the columns.
 __global__ void extract_tiles_kernel(float *Ak, const float2 *tiles, long long side, int k,
                                      int N, int B, long long tpr) {
   const long long t = blockIdx.x;
   const long long r0 = (t / tpr) * B, c0 = (t % tpr) * B;
   const float2 *src = tiles + t * N * N + (long long)k * N + k;
-  for (int i = threadIdx.y; i < B && r0 + i < side; i += blockDim.y)
+  const int i1 = min(B, (int)(blockIdx.y + 1) * kRowChunk);
+  for (int i = blockIdx.y * kRowChunk + threadIdx.y; i < i1 && r0 + i < side; i += blockDim.y)
     for (int j = threadIdx.x; j < B && c0 + j < side; j += blockDim.x)
       Ak[(r0 + i) * side + c0 + j] = __ldcs(src + (long long)i * N + j).x;
 }
@@ -149,16 +154,16 @@ cudaError_t launch_place_kernel(float2 *w, long long N, const float2 *g, long lo
 cudaError_t launch_gather_tiles(float2 *tiles, const float *A, long long side, int k,
                                 long long N, int B, int num_sms, cudaStream_t st) {
   const long long tpr = (side + B - 1) / B;
-  gather_tiles_kernel<<<(unsigned)(tpr * tpr), dim3(32, 8), 0, st>>>(tiles, A, side, k, (int)N,
-                                                                    B, tpr);
+  const dim3 grid((unsigned)(tpr * tpr), (unsigned)((N + kRowChunk - 1) / kRowChunk));
+  gather_tiles_kernel<<<grid, dim3(32, 8), 0, st>>>(tiles, A, side, k, (int)N, B, tpr);
   return cudaGetLastError();
 }
 
 cudaError_t launch_extract_tiles(float *Ak, const float2 *tiles, long long side, int k,
                                  long long N, int B, int num_sms, cudaStream_t st) {
   const long long tpr = (side + B - 1) / B;
-  extract_tiles_kernel<<<(unsigned)(tpr * tpr), dim3(32, 8), 0, st>>>(Ak, tiles, side, k,
-                                                                     (int)N, B, tpr);
+  const dim3 grid((unsigned)(tpr * tpr), (unsigned)((B + kRowChunk - 1) / kRowChunk));
+  extract_tiles_kernel<<<grid, dim3(32, 8), 0, st>>>(Ak, tiles, side, k, (int)N, B, tpr);
   return cudaGetLastError();
 }
 

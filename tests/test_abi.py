@@ -167,6 +167,30 @@ def test_stencil_plan_rejects_before_cuda(lib, args, status):
     assert lib.tcu_dft_last_error() == status
 
 
+def test_stencil_tiling_choice(lib):
+    """tcu_stencil_tiles: the smallest tile side N = r^s with N >= 3k and
+    N^2 >= 128 r within one pass per axis, blocks of B = N - 2k, ceil(side /
+    B)^2 tiles -- checked against the rule evaluated here."""
+    import paper_1908_06649_gb300 as pkg
+    for side, k, r in [(4096, 16, 8), (4096, 16, 16), (4096, 16, 32), (64, 4, 8),
+                       (2000, 16, 8), (300, 16, 16), (120, 20, 8), (1, 1, 16),
+                       (5000, 85, 16), (777, 3, 32), (100, 30, 8)]:
+        smax = 3 if r == 8 else 2
+        Ns = [r ** s for s in range(1, smax + 1)
+              if r ** s >= 3 * k and r ** (2 * s) >= 128 * r]
+        got = pkg.stencil_tiles(side, k, r)
+        if not Ns:
+            assert got == (0, 0, 0)
+            continue
+        N = Ns[0]
+        B = N - 2 * k
+        assert got == ((-(-side // B)) ** 2, N, B), (side, k, r, got)
+    assert pkg.stencil_tiles(4096, 16, 8) == (16384, 64, 32)
+    assert pkg.stencil_tiles(4096, 16, 16) == (361, 256, 224)
+    assert pkg.stencil_tiles(64, 4, 12)[0] == 0
+    assert lib.tcu_stencil_tiles(0, 4, 8, None, None) == 0
+
+
 def test_grid_null_handling(lib):
     import paper_1908_06649_gb300 as pkg
     assert lib.tcu_dft2_destroy(None) == pkg.OK

@@ -123,8 +123,12 @@ def test_stencil_weights(pkg, r, k):
 # blocks of 48, (16, 128, 16) and (8, 120, 20) blocks of 224 and 24, and
 # sides that no block size divides: 100 with k = 6 (blocks of 52), 130 with
 # k = 16 (blocks of 224: one cut block), 37 with k = 5 (blocks of 54)
+# and more: (8, 2000, 16) 3969 tiles of 32^2 blocks, (16, 300, 16) four
+# tiles of 224^2 blocks (256^2 tiles), (8, 100, 30) one 512^2 tile (3k > 64:
+# three radix-8 stages per axis) whose 452^2 block is cut at 100
 @pytest.mark.parametrize("r,side,k", [(8, 64, 4), (8, 96, 8), (16, 128, 16), (8, 120, 20),
-                                      (8, 100, 6), (16, 130, 16), (8, 37, 5)])
+                                      (8, 100, 6), (16, 130, 16), (8, 37, 5),
+                                      (8, 2000, 16), (16, 300, 16), (8, 100, 30)])
 def test_stencil_apply(pkg, r, side, k):
     import torch
     rng = np.random.default_rng(side + k)
