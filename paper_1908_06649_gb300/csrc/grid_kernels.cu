@@ -81,25 +81,28 @@ __global__ void place_kernel_kernel(float2 *w, long long N, const float2 *g, lon
 // A'_{r,c} (3k x 3k); the plan takes B = N - 2k, the largest block whose
 // window still fits N without wrapping.  Blocks of 32 x 8 threads, one per
 // tile (blockIdx.x) and chunk of kRowChunk tile rows (blockIdx.y): rows by
-// threadIdx.y, columns by threadIdx.x, so reads of A and writes of the tile
-// are contiguous along the columns.
-constexpr int kRowChunk = 64;
+// threadIdx.y, column pairs by threadIdx.x (one 16-byte store of two complex
+// values: N is even, so every pair is 16-byte aligned), so reads of A and
+// writes of the tile are contiguous along the columns.
+constexpr int kRowChunk = 32;
 
 __global__ void gather_tiles_kernel(float2 *tiles, const float *A, long long side, int k,
                                     int N, int B, long long tpr) {
   const long long t = blockIdx.x;
   const long long r0 = (t / tpr) * B - k, c0 = (t % tpr) * B - k;
   const int win = B + 2 * k;
-  float2 *dst = tiles + t * N * N;
+  float4 *dst = reinterpret_cast<float4 *>(tiles + t * N * N);
   const int i1 = min(N, (int)(blockIdx.y + 1) * kRowChunk);
   for (int i = blockIdx.y * kRowChunk + threadIdx.y; i < i1; i += blockDim.y) {
     const long long gi = r0 + i;
     const bool row_in = i < win && gi >= 0 && gi < side;
-    for (int j = threadIdx.x; j < N; j += blockDim.x) {
+    for (int j = 2 * threadIdx.x; j < N; j += 2 * blockDim.x) {
       const long long gj = c0 + j;
-      float v = 0.f;
-      if (row_in && j < win && gj >= 0 && gj < side) v = __ldg(A + gi * side + gj);
-      __stcs(dst + (long long)i * N + j, make_float2(v, 0.f));
+      float v0 = 0.f, v1 = 0.f;
+      if (row_in && j < win && gj >= 0 && gj < side) v0 = __ldg(A + gi * side + gj);
+      if (row_in && j + 1 < win && gj + 1 >= 0 && gj + 1 < side)
+        v1 = __ldg(A + gi * side + gj + 1);
+      __stcs(dst + ((long long)i * N + j) / 2, make_float4(v0, 0.f, v1, 0.f));
     }
   }
 }
