@@ -53,6 +53,42 @@ def test_checked_variant_exports_the_same_symbols():
         assert name in exported, name
 
 
+C_PROGRAM = r"""
+#include <stdio.h>
+#include <string.h>
+#include "tcu_dft.h"
+int main(void) {
+  int32_t st[3] = {0, 0, 0};
+  int64_t N = 0, B = 0;
+  if (tcu_dft_plan_passes(65536, 16, st) != 2 || st[0] != 2 || st[1] != 2) return 1;
+  if (tcu_dft_plan_passes(48, 16, st) != 0) return 2;
+  if (tcu_stencil_tiles(4096, 16, 16, &N, &B) != 361 || N != 256 || B != 224) return 3;
+  if (strcmp(tcu_dft_strerror(TCU_DFT_OK), "ok") != 0) return 4;
+  if (tcu_dft_destroy(NULL) != TCU_DFT_OK) return 5;
+  if (tcu_dft_plan(0, 1, 16, TCU_DFT_3XTF32) != NULL) return 6;
+  if (tcu_dft_last_error() != TCU_DFT_ERR_INVALID) return 7;
+  puts("c abi ok");
+  return 0;
+}
+"""
+
+
+def test_plain_c_program_uses_the_boundary(tmp_path):
+    """The header is C99, and a plain C program links the library and calls
+    its host-side entry points (no Python, no torch, no GPU)."""
+    _build.build()
+    src = tmp_path / "abi.c"
+    src.write_text(C_PROGRAM)
+    exe = tmp_path / "abi"
+    libdir = os.path.dirname(_build.LIB_PATH)
+    subprocess.run(["gcc", "-std=c99", "-Wall", "-Werror", "-pedantic",
+                    "-I", os.path.join(ROOT, "include"), str(src), "-o", str(exe),
+                    "-L", libdir, "-ltcu_dft", "-Wl,-rpath," + libdir],
+                   check=True, capture_output=True, text=True)
+    out = subprocess.run([str(exe)], capture_output=True, text=True)
+    assert out.returncode == 0 and "c abi ok" in out.stdout, (out.returncode, out.stderr)
+
+
 def test_binding_lists_every_symbol():
     import paper_1908_06649_gb300 as pkg
     assert sorted(pkg.SYMBOLS) == declared_functions()
