@@ -1097,7 +1097,10 @@ __global__ void __launch_bounds__(
     else if constexpr (G::KS)
       process_item_ks<G, PREC>(P, tw, phys(item), w, nx);
     else
-      process_item<G, PREC, false>(P, &a.tm_tw, tw, phys(item), w, nx);
+      // a strided pass writes the next pass's input: L2-cached stores keep
+      // its latest part for the next pass (which starts there), streaming
+      // stores otherwise
+      process_item<G, PREC, ROLE == kFirst>(P, &a.tm_tw, tw, phys(item), w, nx);
     item += istride;
   }
   if (w.fail && w.rho == 0) atomicCAS(a.err, 0, TCU_DFT_ERR_TIMEOUT);
