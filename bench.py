@@ -528,6 +528,136 @@ def workload_config(wl, args):
             "parallelism": "replica/batch shard x%d" % args.gpus}
 
 
+def time_exec(torch, plan, x, y, steps, direction, stream, flush, l2buf):
+    """CUDA-event timing of `steps` executions of `plan` on `stream` (inputs
+    resident in HBM): per pass launch and per step.  With `flush`, an
+    untimed write of a buffer larger than L2 precedes every step and the
+    step time is the sum of the steps' own events."""
+    npass = len(plan.passes())
+    ev = [[torch.cuda.Event(enable_timing=True) for _ in range(npass + 1)]
+          for _ in range(steps)]
+    for row in ev:
+        for e in row:
+            e.record(stream)
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    t0.record(stream)
+    for i in range(steps):
+        if flush:
+            l2buf.fill_(float(i))
+        plan.exec_timed(x, y, ev[i], direction)
+    t1.record(stream)
+    torch.cuda.synchronize()
+    if flush:
+        total = sum(ev[i][0].elapsed_time(ev[i][npass]) for i in range(steps))
+    else:
+        total = t0.elapsed_time(t1)
+    passes = [sum(ev[i][p].elapsed_time(ev[i][p + 1]) for i in range(steps)) / steps
+              for p in range(npass)]
+    return total / steps, passes
+
+
+def sample_rows(batch, count=8):
+    """Transforms whose outputs the CPU-baseline leg checks: the first, the
+    last and evenly spaced ones in between."""
+    if batch <= count:
+        return list(range(batch))
+    return sorted(set(int(round(i * (batch - 1) / (count - 1))) for i in range(count)))
+
+
+def oracle_accuracy(x_rows, y_rows, tol, inverse=False):
+    """CPU-baseline leg: per-transform relative L2 of GPU outputs against the
+    fp64 oracle's outputs for the same inputs."""
+    import oracle
+    n = x_rows.shape[1]
+    sign, scale = (1, 1.0 / n) if inverse else (-1, 1.0)
+    ref = oracle.fft_radix2(x_rows, sign, scale, threads=oracle.default_threads())
+    err = oracle.rel_l2(y_rows, ref)
+    return {"max_rel_l2": float(err.max()), "median_rel_l2": float(np.median(err)),
+            "transforms": int(x_rows.shape[0]), "tolerance": tol,
+            "ok": bool(err.max() <= tol), "against": "fp64 oracle (radix-2 FFT)"}
+
+
+def per_workload(args, torch, pkg, dev, stream, hbm, p_tf32, skip):
+    """Every other workload the method is evaluated on (the configs besides
+    the headline's), each timed like the headline (warm-up, CUDA events on
+    the exec stream, L2 flushed where the buffers would stay cached), with
+    its step roofline, its dominant pass launch against the HBM peak and,
+    in the CPU-baseline leg, its accuracy against the oracle on sampled
+    transforms.  The two radix-sweep workloads add the inverse and the
+    round trip."""
+    out = {}
+    steps = max(5, min(args.steps, 30))
+    tol = 1e-5 if args.precision == 3 else 3e-3
+    for name in sorted(inputs.WORKLOADS):
+        if name == skip:
+            continue
+        wl = inputs.WORKLOADS[name]
+        n, batch, r = wl["n"], wl["batch"], wl["sqrt_m"]
+        t_gen = time.perf_counter()
+        x_host = inputs.make(wl["kind"], n, batch, wl["seed"])
+        t_gen = time.perf_counter() - t_gen
+        x = torch.from_numpy(x_host).to(dev)
+        y = torch.empty_like(x)
+        plan = pkg.Plan(n, batch, r, args.precision)
+        stages = plan.passes()
+        flush = needs_flush(wl)
+        l2buf = (torch.empty(L2_FLUSH_BYTES // 4, dtype=torch.float32, device=dev)
+                 if flush else None)
+        entry = {"n": n, "batch": batch, "sqrt_m": r, "kind": wl["kind"], "seed": wl["seed"],
+                 "passes": stages, "steps": steps,
+                 "l2": "flushed before every step" if flush else "inputs larger than L2"}
+        dirs = [("forward", pkg.FORWARD)]
+        if "inverse" in wl["dirs"]:
+            dirs.append(("inverse", pkg.INVERSE))
+        bytes_min = 16.0 * n * batch
+        k = sum(stages)
+        tensor_flops = 8.0 * r * n * batch * k * args.precision
+        t_roof = max(bytes_min / (hbm * 1e9), tensor_flops / (p_tf32 * 1e12))
+        ys = {}
+        for dname, d in dirs:
+            src = x if dname == "forward" else ys["forward"]
+            dst = torch.empty_like(x)
+            for _ in range(max(3, args.warmup)):
+                plan.exec(src, dst, d)
+            plan.check()
+            ms, pms = time_exec(torch, plan, src, dst, steps, d, stream, flush, l2buf)
+            plan.check()
+            dom = max(range(len(pms)), key=lambda i: pms[i])
+            ys[dname] = dst
+            entry[dname] = {
+                "ms_per_step": ms, "value": dft_flops(n, batch) / (ms * 1e-3) / 1e9,
+                "unit": UNIT,
+                "roofline_step": {"t_roof_ms": t_roof * 1e3, "frac": t_roof / (ms * 1e-3)},
+                "dominant_launch": {"pass": dom + 1, "stages": stages[dom], "ms": pms[dom],
+                                    "achieved_gbs": bytes_min / (pms[dom] * 1e-3) / 1e9,
+                                    "peak_gbs": hbm,
+                                    "frac": bytes_min / (pms[dom] * 1e-3) / 1e9 / hbm},
+                "launch_ms": pms}
+        rows = sample_rows(batch, 64 if n <= 4096 else 8)
+        if "inverse" in ys:
+            # round trip IDFT(DFT(x)) against x on every transform (no oracle)
+            num = torch.linalg.vector_norm((ys["inverse"] - x).reshape(batch, n), dim=1)
+            den = torch.linalg.vector_norm(x.reshape(batch, n), dim=1)
+            entry["round_trip_max_rel_l2"] = float((num / den).max())
+        if not args.no_cpu_baseline:
+            acc = {}
+            for dname in ys:
+                src_rows = (x_host[rows] if dname == "forward"
+                            else ys["forward"].reshape(batch, n)[rows].cpu().numpy())
+                got = ys[dname].reshape(batch, n)[rows].cpu().numpy()
+                acc[dname] = oracle_accuracy(src_rows, got, tol, inverse=dname == "inverse")
+            entry["accuracy"] = acc
+        entry["input_generation_s"] = t_gen
+        out[name] = entry
+        plan.destroy()
+        del x, y, ys, l2buf
+        torch.cuda.empty_cache()
+        log("per-workload %s: %.4f ms forward" % (name, entry["forward"]["ms_per_step"]))
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -546,6 +676,8 @@ def main():
                          "instead of two pass launches")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (profiling cases)")
+    ap.add_argument("--no-per-workload", action="store_true",
+                    help="skip the other workloads' extra fields")
     ap.add_argument("--grid", default=None, choices=sorted(GRID),
                     help="measure a 2-D workload (2-D DFT, circular 2-D "
                          "convolution or the stencil) instead of the 1-D one")
@@ -706,6 +838,11 @@ def main():
                                 y_gpu=y_head,
                                 tol=1e-5 if args.precision == 3 else 3e-3)
 
+    others = None
+    if (rank == 0 and world == 1 and not args.no_per_workload and args.batch == 0
+            and args.workload == "n65536_b1024"):
+        others = per_workload(args, torch, pkg, dev, stream, hbm, p_tf32, args.workload)
+
     if rank == 0:
         line = {
             "metric": metric_for(wl), "value": value, "unit": UNIT, "n_gpus": world,
@@ -730,6 +867,7 @@ def main():
             "gpu": torch.cuda.get_device_name(dev),
             "gpu_launches": K * launches,
             "clocks": clk,
+            "per_workload": others,
         }
         print(json.dumps(line), flush=True)
     if dist is not None:

@@ -92,7 +92,8 @@ enum {
  * intermediate (two for three passes); uses the current CUDA device.  This
  * is the only call that allocates.
  * Returns NULL on error and sets tcu_dft_last_error():
- *   ERR_INVALID (n < 1, batch < 1, precision not 1 or 3),
+ *   ERR_INVALID (n < 1, batch < 1, precision not one of TCU_DFT_TF32,
+ *   TCU_DFT_3XTF32, TCU_DFT_BF16, TCU_DFT_3XBF16),
  *   ERR_UNSUPPORTED (sqrt_m not in {8,16,32}, n not a power of sqrt_m, n
  *   beyond three passes, or batch*n > 2^40), ERR_CUDA (no sm_103 device),
  *   ERR_OOM. */
@@ -193,13 +194,20 @@ int tcu_dft_pass_stages(tcu_dft_plan_t p, int i);
  * with nothing launched; other argument errors ERR_INVALID / ERR_UNSUPPORTED
  * as tcu_dft_plan would.
  *
+ * Argument errors (including a misaligned or partially overlapping buffer)
+ * are found before any CUDA call.
+ *
  * The first call on a device resolves the device addresses of those arrays
  * (with that device current) and fills the tables; make that first call
  * before any stream capture.  A later call with another n or sqrt_m refills
- * the tables, stream-ordered on `stream`.  All calls share the arrays, which
- * keep the last call's contents: calls whose work overlaps on the GPU (other
- * streams, other host threads) race with each other.  Asynchronous like
- * tcu_dft_exec_dir; a device-side wait timeout is not reported here. */
+ * the tables from host memory, stream-ordered on `stream`: such a call must
+ * not be captured either, and returns ERR_INVALID with nothing enqueued if
+ * `stream` is capturing.  All calls share the arrays, which keep the last
+ * call's contents: calls whose work overlaps on the GPU (other streams, other
+ * host threads) race with each other.  Asynchronous like tcu_dft_exec_dir: a
+ * device-side wait timeout is not reported by default; with TCU_DFT_DEBUG=1
+ * in the environment the call synchronises `stream` and returns it
+ * (ERR_TIMEOUT), as tcu_dft_check does for plans. */
 int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t precision,
                          const void *in, void *out, int dir, void *stream);
 

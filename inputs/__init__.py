@@ -37,7 +37,7 @@ GOLDEN = np.uint64(0x9E3779B97F4A7C15)
 M1 = np.uint64(0xBF58476D1CE4E5B9)
 M2 = np.uint64(0x94D049BB133111EB)
 TONE_SALT = 0x70E5_5EED_0000_0005
-CHUNK = 1 << 22
+CHUNK = 1 << 18  # points per generator chunk (chunks run on threads)
 
 
 def splitmix64(seed: int, start: int, count: int) -> np.ndarray:
@@ -114,6 +114,26 @@ def tone_frequencies(seed: int, n: int, batch: int, count: int = 3,
     return out
 
 
+def _threads() -> int:
+    import os
+    return max(1, min(16, os.cpu_count() or 1))
+
+
+def _parallel(fn, starts):
+    """fn(s) for every chunk start s; chunks are independent (disjoint output
+    slices, counter-based draws), so they run on a thread pool (numpy
+    releases the GIL in the array arithmetic).  Same values as in order."""
+    starts = list(starts)
+    if len(starts) <= 1 or _threads() == 1:
+        for s in starts:
+            fn(s)
+        return
+    from concurrent.futures import ThreadPoolExecutor
+    with ThreadPoolExecutor(max_workers=_threads()) as ex:
+        for _ in ex.map(fn, starts):
+            pass
+
+
 def make(kind: str, n: int, batch: int, seed: int, first: int = 0,
          count: int | None = None, sigma: float = 0.01) -> np.ndarray:
     """Transforms first .. first+count-1 of a workload, shape (count, n), c64."""
@@ -123,9 +143,10 @@ def make(kind: str, n: int, batch: int, seed: int, first: int = 0,
     flat = out.reshape(-1)
     base = first * n
     if kind in ("uniform", "normal"):
-        for s in range(0, flat.shape[0], CHUNK):
+        def one(s):
             e = min(flat.shape[0], s + CHUNK)
             _fill(flat[s:e], seed, kind, base + s)
+        _parallel(one, range(0, flat.shape[0], CHUNK))
         return out
     if kind == "tones":
         freqs = tone_frequencies(seed, n, count, first=first)
@@ -134,16 +155,17 @@ def make(kind: str, n: int, batch: int, seed: int, first: int = 0,
         # values as evaluating it per element)
         roots = np.exp(2j * np.pi * np.arange(n, dtype=np.int64) / n)
         step = max(1, CHUNK // n)
-        noise = np.empty(step * n, dtype=np.complex64)
-        for b0 in range(0, count, step):
+
+        def one(b0):
             b1 = min(count, b0 + step)
-            nz = noise[:(b1 - b0) * n]
+            nz = np.empty((b1 - b0) * n, dtype=np.complex64)
             _fill(nz, seed, "normal", base + b0 * n)
             sig = np.zeros((b1 - b0, n), dtype=np.complex128)
             for t in range(freqs.shape[1]):
                 sig += roots[(freqs[b0:b1, t:t + 1] * j[None, :]) % n]
             sig += sigma * nz.reshape(b1 - b0, n).astype(np.complex128)
             out[b0:b1] = sig.astype(np.complex64)
+        _parallel(one, range(0, count, step))
         return out
     raise ValueError(kind)
 

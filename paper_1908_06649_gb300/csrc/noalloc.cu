@@ -60,6 +60,7 @@ int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t preci
       (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32 && !prec_bf16(precision)) ||
       !in || !out || (dir != TCU_DFT_FORWARD && dir != TCU_DFT_INVERSE))
     return TCU_DFT_ERR_INVALID;
+  if (((uintptr_t)in & 15) || ((uintptr_t)out & 15)) return TCU_DFT_ERR_INVALID;
   if (prec_bf16(precision)) return TCU_DFT_ERR_UNSUPPORTED;
   if (sqrt_m != 8 && sqrt_m != 16 && sqrt_m != 32) return TCU_DFT_ERR_UNSUPPORTED;
   const int r = sqrt_m, log2r = ilog2(r);
@@ -69,11 +70,15 @@ int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t preci
     m *= r;
     ++k;
   }
-  if (m != n) return TCU_DFT_ERR_UNSUPPORTED;
+  // n = r^k with k >= 1, as tcu_dft_plan requires
+  if (m != n || k < 1) return TCU_DFT_ERR_UNSUPPORTED;
   int st[kMaxPasses] = {0, 0, 0};
   const int npasses = plan_stages(r, k, st);
   if (npasses == 0 || npasses > 2 || n > kNaMaxN) return TCU_DFT_ERR_TOO_LARGE;
   if (npasses == 2 && batch * n > kNaMaxPoints) return TCU_DFT_ERR_TOO_LARGE;
+  // in == out is allowed; a partial overlap is not
+  if (in != out && overlaps(in, out, (size_t)batch * n * sizeof(float2)))
+    return TCU_DFT_ERR_INVALID;
   cudaStream_t stream_ = (cudaStream_t)stream;
 
   std::lock_guard<std::mutex> lock(g_na_mutex);
@@ -122,19 +127,30 @@ int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t preci
     for (int d = 0; d < 2; ++d)
       p.pass[pi].tw_stage[d] = D.tw_stage + ((size_t)d * 2 + pi) * kNaStageTw;
 
-  // ---- tables for this (n, r), refilled only when they change; table A of
-  // the strided pass at the start of the direction's twiddle array, B after it
-  DirTables t[2];
-  for (int d = 0; d < 2; ++d) {
-    dir_tables(&p, d, t[d]);
-    for (int pi = 0; pi < npasses; ++pi)
-      if (t[d].stage[pi].size() > (size_t)kNaStageTw) return TCU_DFT_ERR_TOO_LARGE;
-    if (npasses == 2) {
+  // ---- tables for this (n, r): table A of the strided pass at the start of
+  // the direction's twiddle array, B (more than 256 columns) after it
+  if (npasses == 2) {
+    const long long n2 = 1ll << p.pass[0].lo, VL = n2 > 256 ? 256 : n2;
+    for (int d = 0; d < 2; ++d) {
       p.pass[0].tw_a[d] = D.tw_out + (size_t)d * kNaMaxN;
-      if (!t[d].B[0].empty()) p.pass[0].tw_b[d] = p.pass[0].tw_a[d] + t[d].A[0].size();
+      if (n2 > VL) p.pass[0].tw_b[d] = p.pass[0].tw_a[d] + (1ll << p.pass[0].log2L) * VL;
     }
   }
+  // built and uploaded only when (n, r) changes: a call that changes them
+  // copies from host memory on `stream` and so must not be captured
   if (D.n != n || D.r != r) {
+    cudaStreamCaptureStatus cap = cudaStreamCaptureStatusNone;
+    if (cudaStreamIsCapturing(stream_, &cap) != cudaSuccess) {
+      cudaGetLastError();
+      return TCU_DFT_ERR_CUDA;
+    }
+    if (cap != cudaStreamCaptureStatusNone) return TCU_DFT_ERR_INVALID;
+    DirTables t[2];
+    for (int d = 0; d < 2; ++d) {
+      dir_tables(&p, d, t[d]);
+      for (int pi = 0; pi < npasses; ++pi)
+        if (t[d].stage[pi].size() > (size_t)kNaStageTw) return TCU_DFT_ERR_TOO_LARGE;
+    }
     D.n = 0;
     for (int d = 0; d < 2; ++d) {
       if (cudaMemcpyAsync(p.bimg[d], t[d].img.data(), t[d].img.size() * sizeof(float),
@@ -166,7 +182,15 @@ int tcu_dft_exec_noalloc(int64_t n, int64_t batch, int32_t sqrt_m, int32_t preci
 
   // the timeout word must start at zero; then the ordinary launch path
   if (cudaMemsetAsync(D.err, 0, sizeof(int), stream_) != cudaSuccess) return TCU_DFT_ERR_CUDA;
-  return exec_impl(&p, in, out, dir, stream, nullptr);
+  const int rc = exec_impl(&p, in, out, dir, stream, nullptr);
+  if (rc != TCU_DFT_OK || !debug_exec()) return rc;
+  // TCU_DFT_DEBUG=1: wait for the launches and report the error word (a
+  // device-side wait timeout) as tcu_dft_check does for plans
+  int flag = 0;
+  if (cudaStreamSynchronize(stream_) != cudaSuccess ||
+      cudaMemcpy(&flag, D.err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return TCU_DFT_ERR_CUDA;
+  return word_status(flag);
 }
 
 }  // extern "C"

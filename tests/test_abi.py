@@ -164,12 +164,25 @@ def test_python_plan_raises(lib):
     ((8 ** 7, 1, 8, 3, -1), 6),
     ((32 ** 4, 1, 32, 3, -1), 6),      # n beyond the fixed twiddle table
     ((65536, 65, 16, 3, -1), 6),       # batch*n beyond the fixed intermediate
+    ((1, 1, 16, 3, -1), 2),            # n = 1 = r^0: k >= 1 is required
 ])
 def test_noalloc_rejects_before_cuda(lib, args, status):
     import ctypes
     n, batch, r, prec, d = args
     fake = ctypes.c_void_p(1 << 20)  # never dereferenced: rejected first
     assert lib.tcu_dft_exec_noalloc(n, batch, r, prec, fake, fake, d, None) == status
+
+
+@pytest.mark.parametrize("a,b", [
+    ((1 << 20) + 8, 1 << 24),          # input not 16-byte aligned
+    (1 << 20, (1 << 24) + 4),          # output not 16-byte aligned
+    (1 << 20, (1 << 20) + 16),         # partial overlap of in and out
+])
+def test_noalloc_rejects_buffers_before_cuda(lib, a, b):
+    import ctypes
+    # never dereferenced: the pointers are rejected before any CUDA call
+    assert lib.tcu_dft_exec_noalloc(256, 4, 16, 3, ctypes.c_void_p(a), ctypes.c_void_p(b),
+                                    -1, None) == 1
 
 
 def test_noalloc_null_buffers(lib):

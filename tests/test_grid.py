@@ -115,7 +115,19 @@ def test_stencil_weights(pkg, r, k):
     ref = grid.stencil_weights(w3.astype(np.float64), k)
     got = W.cpu().numpy()
     assert got.shape == ref.shape
-    assert np.max(np.abs(got - ref)) <= 1e-5 * np.max(np.abs(ref)) * max(1, k / 10)
+    # Error bound, first order in the transforms' errors (P has unit sum and
+    # non-negative entries, so |P^(w)| <= 1 at every frequency w):
+    #  * forward 2-D DFT of P on the Nw x Nw grid: ||dP^||_2 <= 1e-5 ||P^||_2
+    #    = 1e-5 Nw ||P||_2 (the per-transform relative L2 bar, Parseval);
+    #  * k-th power: d(P^k) = k P^(k-1) dP^, and |P^|^(k-1) <= 1, so the
+    #    spectrum error is at most k ||dP^||_2; the inverse (1/Nw^2 times a
+    #    unitary-times-Nw map) turns it into k * 1e-5 ||P||_2 on W;
+    #  * the inverse DFT's own error: 1e-5 ||W||_2 (same bar);
+    #  * the pointwise power by repeated squaring in fp32: at most
+    #    2 log2(k) roundings of 2^-24 per frequency, 2 log2(k) 2^-24 ||W||_2.
+    pn, wn = np.linalg.norm(w3.astype(np.float64)), np.linalg.norm(ref)
+    bound = 1e-5 * (k * pn + wn) + 2 * max(1.0, np.log2(k)) * 2.0 ** -24 * wn
+    assert np.linalg.norm(got.astype(np.float64) - ref) <= bound
     plan.destroy()
 
 

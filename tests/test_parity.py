@@ -179,57 +179,77 @@ def test_tones_workload_peaks(pkg):
     check(y[:256], x[:256], 3)
 
 
-def test_full_size_headline_sampled(pkg):
-    # n = 65536, batch = 1024, N(0,1), seed 1 -- in the launch configuration
-    # the benchmark times.  Whole transforms checked on a sample; every
-    # transform checked through Parseval.
-    import torch
-    n, batch = 65536, 1024
-    x = inputs.make("normal", n, batch, seed=1)
-    plan = pkg.Plan(n, batch, 16, 3)
-    xd = torch.from_numpy(x).cuda()
-    y = plan.forward(xd)
-    plan.check()
-    yh = y.cpu().numpy()
-    plan.destroy()
-    sample = [0, 1, 511, 777, 1023]
-    check(yh[sample], x[sample], 3)
-    ex = np.sum(np.abs(x.astype(np.complex128)) ** 2, axis=1) * n
-    ey = np.sum(np.abs(yh.astype(np.complex128)) ** 2, axis=1)
-    assert np.max(np.abs(ey / ex - 1)) < 1e-5
-    rng = np.random.default_rng(0)
-    bs = rng.integers(0, batch, 8)
-    ks = rng.integers(0, n, 16)
-    ref = oracle.dft_entries(x[bs], ks)
-    got = yh[bs][:, ks]
-    scale = np.sqrt(n)
-    assert np.max(np.abs(got - ref)) / scale < 1e-4
-
-
-def _sampled_full_size(pkg, x, r, inverse=False, whole=(0,), nent=16):
-    # whole transforms on a sample against the oracle, Parseval on every
-    # transform, and single entries by direct summation
-    import torch
+def oracle_batch(x, inverse=False, chunk_points=1 << 23):
+    """The oracle's transform of every row of x (power-of-two n), chunk by
+    chunk through its recursive radix-2 FFT on every host core; yields
+    (first row, fp64 outputs) per chunk."""
     batch, n = x.shape
-    plan = pkg.Plan(n, batch, r, 3)
-    xd = torch.from_numpy(x).cuda()
-    y = plan.inverse(xd) if inverse else plan.forward(xd)
-    plan.check()
-    yh = y.cpu().numpy()
-    plan.destroy()
-    check(yh[list(whole)], x[list(whole)], 3, inverse=inverse)
-    scale = (1.0 / n) if inverse else float(n)
-    ex = np.sum(np.abs(x.astype(np.complex128)) ** 2, axis=1) * scale
-    ey = np.sum(np.abs(yh.astype(np.complex128)) ** 2, axis=1)
-    assert np.max(np.abs(ey / ex - 1)) < 1e-5
-    rng = np.random.default_rng(1)
-    bs = rng.integers(0, batch, 4)
-    ks = rng.integers(0, n, nent)
+    rows = max(1, chunk_points // n)
+    sign, scale = (1, 1.0 / n) if inverse else (-1, 1.0)
+    for a in range(0, batch, rows):
+        yield a, oracle.fft_radix2(x[a:a + rows], sign, scale,
+                                   threads=oracle.default_threads())
+
+
+def check_whole_batch(yh, x, prec, inverse=False):
+    """Per-transform relative L2 of EVERY transform of the batch against the
+    oracle (max over the batch <= the bar); returns the errors."""
+    err = np.empty(x.shape[0])
+    for a, ref in oracle_batch(x, inverse):
+        err[a:a + ref.shape[0]] = oracle.rel_l2(yh[a:a + ref.shape[0]], ref)
+    assert np.all(np.isfinite(err))
+    assert err.max() <= TOL[prec], "max rel L2 %.3e (transform %d)" % (err.max(),
+                                                                       int(err.argmax()))
+    return err
+
+
+def check_entries(yh, x, inverse=False, nb=8, nk=32, seed=0):
+    """Single entries of sampled transforms (the first and the last among
+    them) by the direct definition, each within 1e-5 of the RMS magnitude
+    of the sampled reference entries."""
+    batch, n = x.shape
+    rng = np.random.default_rng(seed)
+    bs = np.unique(np.concatenate([[0, batch - 1], rng.integers(0, batch, nb)]))
+    ks = np.unique(np.concatenate([[0, 1, n - 1], rng.integers(0, n, nk)]))
     ref = oracle.dft_entries(x[bs], ks, inverse=inverse)
     got = yh[bs][:, ks]
     mag = np.sqrt(np.mean(np.abs(ref) ** 2))
-    assert np.max(np.abs(got - ref)) / mag < 1e-4
-    return yh
+    assert np.max(np.abs(got - ref)) / mag <= 1e-5
+
+
+def _device_transform(pkg, x, r, prec=3, inverse=False):
+    import torch
+    batch, n = x.shape
+    plan = pkg.Plan(n, batch, r, prec)
+    xd = torch.from_numpy(x).cuda()
+    y = plan.inverse(xd) if inverse else plan.forward(xd)
+    plan.check()
+    passes = plan.passes()
+    yh = y.cpu().numpy()
+    del xd, y
+    plan.destroy()
+    return yh, passes
+
+
+def test_full_size_small_transforms(pkg):
+    # n = 4096 (16^3, one pass), batch 64, U[-1,1], seed 0: every transform
+    x = inputs.make("uniform", 4096, 64, seed=0)
+    yh, passes = _device_transform(pkg, x, 16)
+    assert passes == [3]
+    err = oracle.rel_l2(yh, oracle.dft(x, threads=oracle.default_threads()))
+    assert err.max() <= TOL[3]
+
+
+def test_full_size_headline(pkg):
+    # n = 65536, batch = 1024, N(0,1), seed 1 -- in the launch configuration
+    # the benchmark times: every transform whole against the oracle, and
+    # single entries by the definition
+    n, batch = 65536, 1024
+    x = inputs.make("normal", n, batch, seed=1)
+    yh, passes = _device_transform(pkg, x, 16)
+    assert passes == [2, 2]
+    check_whole_batch(yh, x, 3)
+    check_entries(yh, x)
 
 
 _CACHE = {}
@@ -242,21 +262,47 @@ def _sweep_input():
 
 
 @pytest.mark.parametrize("r", [8, 32])
-def test_full_size_radix_sweep_sampled(pkg, r):
+def test_full_size_radix_sweep(pkg, r):
     # n = 32768 (8^5 = 32^3), batch 4096, N(0,1), seed 2: forward and
-    # inverse, and the round trip, in the launch configuration of the plan
+    # inverse (of the forward outputs) of every transform, and the round trip
     x = _sweep_input()
-    y = _sampled_full_size(pkg, x, r, whole=(0, 4095))
-    back = _sampled_full_size(pkg, y, r, inverse=True, whole=(7,))
+    y, _ = _device_transform(pkg, x, r)
+    check_whole_batch(y, x, 3)
+    check_entries(y, x, seed=r)
+    back, _ = _device_transform(pkg, y, r, inverse=True)
+    check_whole_batch(back, y, 3, inverse=True)
     rt = np.linalg.norm(back - x, axis=1) / np.linalg.norm(x, axis=1)
     assert rt.max() <= 1e-5
 
 
 def test_full_size_long_transforms(pkg):
-    # n = 2^24 (16^6), batch 4, uniform, seed 3: three HBM passes
+    # n = 2^24 (16^6), batch 4, uniform, seed 3: three HBM passes, all four
+    # transforms whole
     n, batch = 1 << 24, 4
     x = inputs.make("uniform", n, batch, seed=3)
-    _sampled_full_size(pkg, x, 16, whole=(2,))
+    yh, passes = _device_transform(pkg, x, 16)
+    assert passes == [2, 2, 2]
+    check_whole_batch(yh, x, 3)
+    check_entries(yh, x, nb=4, nk=16)
+
+
+def test_full_size_many_short_transforms(pkg):
+    # n = 256 (16^2), batch 2^20, three tones + N(0, 0.01^2) noise, seed 4:
+    # every transform whole against the oracle, and on every transform the
+    # three largest outputs sit exactly at its seeded frequencies
+    n, batch = 256, 1 << 20
+    x = inputs.make("tones", n, batch, seed=4)
+    yh, passes = _device_transform(pkg, x, 16)
+    assert passes == [2]
+    check_whole_batch(yh, x, 3)
+    f = np.sort(inputs.tone_frequencies(4, n, batch), axis=1)
+    C = 1 << 16
+    for a in range(0, batch, C):
+        mag = np.abs(yh[a:a + C])
+        top = np.sort(np.argpartition(-mag, 3, axis=1)[:, :3], axis=1)
+        assert np.array_equal(top, f[a:a + C])
+        peaks = np.take_along_axis(mag, f[a:a + C], axis=1)
+        assert np.all(np.abs(peaks / n - 1) < 0.05)
 
 
 def test_maximum_size_radix8(pkg):
