@@ -674,6 +674,8 @@ def main():
     ap.add_argument("--fuse", action="store_true",
                     help="one fused launch with an L2-resident intermediate "
                          "instead of two pass launches")
+    ap.add_argument("--one-pass", action="store_true",
+                    help="both passes in one launch on cluster pairs (n = 16^4)")
     ap.add_argument("--batch", type=int, default=0,
                     help="override the workload's batch (profiling cases)")
     ap.add_argument("--no-per-workload", action="store_true",
@@ -716,7 +718,8 @@ def main():
     x = torch.from_numpy(x_host).to(dev)
     y = torch.empty_like(x)
     plan = pkg.Plan(n, batch, r, args.precision,
-                    pkg.PLAN_FUSE if args.fuse else pkg.PLAN_DEFAULT)
+                    pkg.PLAN_FUSE if args.fuse else
+                    (pkg.PLAN_ONE_PASS if args.one_pass else pkg.PLAN_DEFAULT))
     npass = len(plan.passes())
     stream = torch.cuda.current_stream()
 

@@ -109,7 +109,16 @@ enum {
   /* Run both passes in ONE fused launch whose intermediate is a small ring
    * of transforms kept in L2 (HBM then moves each point once in and once
    * out).  Only for two passes of >= 2 stages each; otherwise ignored. */
-  TCU_DFT_PLAN_FUSE = 2
+  TCU_DFT_PLAN_FUSE = 2,
+  /* Run both passes in ONE launch on clusters of two CTAs (one per SM):
+   * each cluster takes whole transforms, splits each one's pass-1 and
+   * pass-2 work between its two CTAs and keeps the transform's
+   * intermediate in one of two scratch slots of its own that stay in L2
+   * (2 * clusters * n complex64 of scratch instead of batch * n); the
+   * passes synchronise through mbarriers of the cluster.  HBM moves each
+   * point once in and once out.  For sqrt_m = 16, n = 16^4 in TF32 or
+   * 3xTF32; otherwise ignored.  Not with FUSE or NO_FUSE. */
+  TCU_DFT_PLAN_ONE_PASS = 4
 };
 
 /* tcu_dft_plan with scheduling flags (TCU_DFT_PLAN_*); unknown bits, or
@@ -118,7 +127,8 @@ enum {
 tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
                                int32_t precision, uint32_t flags);
 
-/* 1 if the plan runs its two passes as one fused launch, 0 if not, -1 for a
+/* 1 if the plan runs its two passes as one launch (TCU_DFT_PLAN_FUSE or
+ * TCU_DFT_PLAN_ONE_PASS), 0 if not, -1 for a
  * NULL plan. */
 int tcu_dft_is_fused(tcu_dft_plan_t p);
 

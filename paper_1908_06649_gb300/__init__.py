@@ -36,6 +36,7 @@ ERR_BOUNDS = 7
 PLAN_DEFAULT = 0
 PLAN_NO_FUSE = 1
 PLAN_FUSE = 2
+PLAN_ONE_PASS = 4
 
 SYMBOLS = (
     "tcu_dft_plan", "tcu_dft_plan_ex", "tcu_dft_is_fused", "tcu_dft_exec",

@@ -61,13 +61,15 @@ enum Role { kSingle = 0, kFirst = 1, kSecond = 2, kCols = 3 };
 __host__ __device__ constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 16 ? 4 : 5); }
 // Warpgroups per CTA: TMEM holds 512 columns, a warpgroup's slot 3 Q of
 // them; a radix-16 first (strided) pass also stages its inter-pass twiddles
-// in SMEM, which leaves room for four.  A radix-32 pass of two stages runs
+// in SMEM, which leaves room for four; a radix-16 last pass of several runs
+// four too (measured faster than five: 0.165 instead of 0.181 ms for the
+// second pass of n = 16^4 x 1024).  A radix-32 pass of two stages runs
 // four warpgroups whose slots hold A for half of K (the products of a stage
 // in two K halves); one-stage radix-32 passes (already near the copy rate),
 // the convolution row pass and the fused schedule keep whole-K slots, two
 // per CTA at radix 32 (whole_k_nwg).
 __host__ __device__ constexpr int pass_nwg(int R, int ROLE, int S = 2) {
-  return R == 32 ? (S >= 2 ? 4 : 2) : (ROLE == 1 && R == 16 ? 4 : 5);
+  return R == 32 ? (S >= 2 ? 4 : 2) : ((ROLE == 1 || ROLE == 2) && R == 16 ? 4 : 5);
 }
 __host__ __device__ constexpr int whole_k_nwg(int R, int ROLE) {
   return R == 32 ? 2 : pass_nwg(R, ROLE);
@@ -655,6 +657,7 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
   constexpr int S = G::LOG2L / G::LOG2R;
   if (!mbar_wait_bounded(w.bar_stg, w.ph_stg)) w.fail = true;
   w.ph_stg ^= 1;
+  mid.after_load(w);
   {
     float2 x[R];
     staged_row<G>(w, x);
@@ -709,6 +712,7 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
     fence_after_sync();
   }
   if (S == 1 && w.team_lead) mid.publish();
+  mid.before_store(w);
   last_stage_store<G, PREC, OUT_L2>(P, item, w);
 }
 
@@ -1052,6 +1056,8 @@ struct StaticNext {
     if (issued) issue_input<G>(P, tm, G::TW == 1 && P.reverse ? nitems - 1 - next : next, w);
   }
   __device__ void publish() {}
+  __device__ void after_load(const WG &) {}
+  __device__ void before_store(WG &) {}
 };
 
 template <int R, int PREC, int S, int LO, int ROLE, int LP, bool CONV = false, int TW = 1>
@@ -1276,6 +1282,9 @@ struct FusedNext {
     pos2 = claim();
   }
 
+  __device__ void after_load(const WG &) {}
+  __device__ void before_store(WG &) {}
+
   __device__ void publish() {
     publish_pending();
     if (lane0()) {
@@ -1378,6 +1387,254 @@ __global__ void __launch_bounds__(
   if (w.team_lead) nx.publish_pending();
   if (w.rho == 0 && w.fail) atomicCAS(a.err, 0, TCU_DFT_ERR_TIMEOUT);
   kernel_teardown(tbase, w, w.fail && stg_pending, w.fail && w.tws_inflight);
+}
+
+// ------------------------------------------ one HBM pass on cluster pairs
+// Both passes of a two-pass (four-step) transform in ONE launch, with the
+// intermediate of each transform kept in L2 and every synchronisation local
+// to a cluster of two CTAs.  Cluster c takes the transforms of pairs
+// c, c + NC, c + 2 NC, ... (NC clusters; pair p holds transforms 2p, 2p+1),
+// so its j-th transform is t_j = 2 (c + (j >> 1) NC) + (j & 1) and slot
+// j & 1 of its two-transform scratch holds t_j's intermediate: pass-1 items
+// write it with L2-cached stores, pass-2 items read it back by TMA.  HBM
+// then sees each point read once and written once.
+//
+// Each transform has 2H pass-1 items and 2H pass-2 items; CTA rank k of the
+// cluster takes items kH .. kH + H - 1 of both.  A CTA's sequence of items
+// is P1(0) [H items], then for j = 0, 1, ...: P1(j+1) [H], P2(j) [H]; its
+// warpgroups take positions round-robin.  Two mbarriers per slot in each
+// CTA count items of both CTAs (2H arrivals per phase):
+//   full[s]  -- pass-1 items of the slot's transform whose stores are
+//               visible (released at cluster scope after the warpgroup's
+//               barrier); a pass-2 item waits for it before copying;
+//   empty[s] -- pass-2 items of the slot's transform whose input copy has
+//               landed; a pass-1 item of transform j >= 2 waits for the
+//               phase of transform j - 2 before storing into the slot.
+// Every wait is for items at earlier positions of both CTAs' sequences, so
+// the schedule cannot deadlock; every wait is bounded (ERR_TIMEOUT).
+struct PairItem {
+  int type;  // 0: pass-1 item, 1: pass-2 item
+  int j;     // the CTA's transform (sequence index)
+  int m;     // item within this CTA's half of the transform
+  bool valid;
+};
+
+__device__ __forceinline__ PairItem pair_decode(long long pos, int H, int J) {
+  PairItem it;
+  it.valid = J > 0 && pos < 2ll * H * J;
+  it.type = 0;
+  it.j = 0;
+  it.m = 0;
+  if (!it.valid) return it;
+  if (pos < H) {
+    it.m = (int)pos;
+    return it;
+  }
+  const long long q = pos - H;
+  const int j = (int)(q / (2 * H)), r = (int)(q % (2 * H));
+  if (j < J - 1 && r < H) {
+    it.j = j + 1;
+    it.m = r;
+  } else {
+    it.type = 1;
+    it.j = j;
+    it.m = j < J - 1 ? r - H : r;
+  }
+  return it;
+}
+
+template <class G1, class G2>
+struct PairNext {
+  const GArgs &a;
+  const PRun &p1, &p2;
+  uint32_t full_bar, empty_bar;  // this CTA's full[0], empty[0] (slot s at + 8 s)
+  uint32_t peer;
+  long long cid, nc;
+  int crank, H, J;
+  PairItem cur, nxt;
+  bool issued;  // nxt's input copy is in flight
+
+  __device__ long long tf(int j) const { return 2 * (cid + (long long)(j >> 1) * nc) + (j & 1); }
+  __device__ long long gitem(const PairItem &it) const {
+    return tf(it.j) * (2ll * H) + (long long)crank * H + it.m;
+  }
+  // parity of the phase of full[s] / empty[s] that belongs to transform j
+  __device__ static uint32_t par(int j) { return (uint32_t)(j >> 1) & 1u; }
+
+  __device__ void copy(const PairItem &it, const WG &w) {
+    if (it.type == 0) {
+      issue_input<G1>(p1, &a.tm_in, gitem(it), w);
+    } else {
+      fence_proxy_async_global();  // after the acquire of full[]
+      issue_input<G2>(p2, nullptr, gitem(it), w);
+    }
+  }
+  // warp 0 of the warpgroup, converged: the next item's input, unless it is
+  // a pass-2 item whose transform's pass-1 items are not all stored yet
+  __device__ void issue(const WG &w) {
+    issued = false;
+    if (!nxt.valid) return;
+    if (nxt.type == 1) {
+      int ok = 0;
+      if ((threadIdx.x & 31) == 0)
+        ok = mbar_test_cluster(full_bar + 8 * (nxt.j & 1), par(nxt.j)) ? 1 : 0;
+      if (!__shfl_sync(0xffffffffu, ok, 0)) return;
+    }
+    copy(nxt, w);
+    issued = true;
+  }
+  // warp 0, converged: bounded wait for `it`'s dependency, then its copy
+  __device__ bool wait_and_copy(const PairItem &it, const WG &w) {
+    int ok = 1;
+    if (it.type == 1 && (threadIdx.x & 31) == 0)
+      ok = mbar_wait_cluster_bounded(full_bar + 8 * (it.j & 1), par(it.j)) ? 1 : 0;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (ok) copy(it, w);
+    return ok != 0;
+  }
+  __device__ void publish() {}
+  // a pass-2 item's input has landed in SMEM: its slot may be overwritten
+  __device__ void after_load(const WG &w) {
+    if (cur.type == 1 && w.team_lead) {
+      if (elect_one()) {
+        const uint32_t b = empty_bar + 8 * (cur.j & 1);
+        mbar_arrive_cluster_local(b);
+        mbar_arrive_cluster_remote(mapa_shared(b, peer));
+      }
+      __syncwarp();
+    }
+  }
+  // a pass-1 item of transform j >= 2 stores into the slot of j - 2 only
+  // once every pass-2 item of j - 2 has copied it out
+  __device__ void before_store(WG &w) {
+    if (cur.type == 0 && cur.j >= 2 &&
+        !mbar_wait_cluster_bounded(empty_bar + 8 * (cur.j & 1), par(cur.j - 2)))
+      w.fail = true;
+  }
+  // after the warpgroup's barrier that follows a pass-1 item's stores
+  __device__ void arrive_full(const WG &w) {
+    if (elect_one()) {
+      fence_acq_rel_cluster();
+      const uint32_t b = full_bar + 8 * (cur.j & 1);
+      mbar_arrive_cluster_local(b);
+      mbar_arrive_cluster_remote(mapa_shared(b, peer));
+    }
+    __syncwarp();
+  }
+};
+
+template <int R, int S1, int S2>
+struct PairLayout {
+  using G1 = Geo<R, S1, log2_radix(R) * S2, kFirst, 0, whole_k_nwg(R, kFirst)>;
+  using SM = SmemLayout<R, G1::NWG, G1::TW_ENTRIES, Geo<R, S2, log2_radix(R) * S1, kSecond, 0,
+                                                        G1::NWG>::TW_ENTRIES,
+                        G1::TW_SMEM, G1::TWB>;
+  static constexpr size_t OFF_PBAR = (SM::BYTES + 15) / 16 * 16;  // full[2], empty[2]
+  static constexpr size_t OFF_PRUN = OFF_PBAR + 32;               // per-CTA PRun copies
+  static constexpr size_t BYTES = OFF_PRUN + 2 * sizeof(PRun);
+  static_assert(BYTES <= 227 * 1024, "shared memory budget");
+};
+
+template <int R, int PREC, int S1, int S2>
+__global__ void __launch_bounds__(
+    Geo<R, S1, log2_radix(R) * S2, kFirst, 0, whole_k_nwg(R, kFirst)>::THREADS, 1)
+    dft_pair_kernel(const __grid_constant__ GArgs a) {
+  static_assert(S1 >= 2 && S2 >= 2, "the pair schedule needs an SMEM barrier per item");
+  using PL = PairLayout<R, S1, S2>;
+  using G1 = typename PL::G1;
+  using G2 = Geo<R, S2, log2_radix(R) * S1, kSecond, 0, G1::NWG>;
+  using SM = typename PL::SM;
+  constexpr int NWG = G1::NWG;
+  extern __shared__ __align__(1024) unsigned char smem[];
+  float2 *tw1 = reinterpret_cast<float2 *>(smem + SM::OFF_TW1);
+  float2 *tw2 = reinterpret_cast<float2 *>(smem + SM::OFF_TW2);
+  uint64_t *mbar = reinterpret_cast<uint64_t *>(smem + SM::OFF_BAR);
+  uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 3 * NWG);
+  uint64_t *pbar = reinterpret_cast<uint64_t *>(smem + PL::OFF_PBAR);
+  PRun *prun = reinterpret_cast<PRun *>(smem + PL::OFF_PRUN);
+  const int H = a.items1_per_tf / 2;
+  const long long cid = cluster_id_x(), nc = nclusters_x();
+  const int crank = (int)cluster_ctarank();
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < 4; ++i) mbar_init(smem_u32(pbar + i), 2 * H);
+    // this cluster's two slots: pass-1 output (slot t & 1), pass-2 input
+    const long long n = 1ll << G1::LOG2NT;
+    prun[0] = a.p[0];
+    prun[0].out = a.p[0].out + cid * 2 * n;
+    prun[1] = a.p[1];
+    prun[1].in = a.p[1].in + cid * 2 * n;
+  }
+  const uint32_t tbase = kernel_setup<NWG, G1::THREADS>(
+      a.bimg, (int)(SM::IMG / 4), reinterpret_cast<float *>(smem), a.p[0].tw_stage, tw1,
+      G1::TW_ENTRIES, a.p[1].tw_stage, tw2, G2::TW_ENTRIES, mbar, tmem_slot);
+  // the peer's barriers exist before any arrival on them
+  cluster_sync_all();
+  WG w;
+  init_wg<R, SM, G1::GCOLS>(w, tbase, smem);
+#ifdef TCU_DFT_CHECKED
+  w.err = a.err;
+#endif
+  // transforms of this cluster: t_j < batch for j < J
+  int J = 0;
+  {
+    const long long pairs = (a.batch + 1) / 2;
+    if (cid < pairs) {
+      const long long np = (pairs - 1 - cid) / nc + 1;  // pairs of this cluster
+      J = (int)(2 * np);
+      if (2 * (cid + (np - 1) * nc) + 1 >= a.batch) --J;  // a last pair of one
+    }
+  }
+  PairNext<G1, G2> nx{a,     prun[0], prun[1], smem_u32(pbar), smem_u32(pbar + 2),
+                      (uint32_t)(crank ^ 1), cid, nc, crank, H, J};
+  nx.issued = false;
+  const int wg = threadIdx.x >> 7;
+  long long pos = wg;
+  nx.cur = pair_decode(pos, H, J);
+  bool f = false;
+  if (w.team_lead && nx.cur.valid) f = !nx.wait_and_copy(nx.cur, w);
+  if (named_bar_or(w.bar_id, w.bar_count, f)) w.fail = true;
+  bool stg_pending = false;
+  while (nx.cur.valid && !w.fail) {
+    nx.nxt = pair_decode(pos + NWG, H, J);
+    if (nx.cur.type == 0) {
+      process_item<G1, PREC, true>(prun[0], &a.tm_tw, tw1, nx.gitem(nx.cur), w, nx);
+      // every thread's stores of the item, then its arrival on full[]
+      if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;
+      if (!w.fail && w.team_lead) nx.arrive_full(w);
+    } else {
+      process_item<G2, PREC, false>(prun[1], &a.tm_tw, tw2, nx.gitem(nx.cur), w, nx);
+      // a uniform failure state before the next item's barriers
+      if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;
+    }
+    stg_pending = nx.issued;
+    if (w.fail) break;
+    pos += NWG;
+    nx.cur = nx.nxt;
+    if (nx.cur.valid && !nx.issued) {
+      // the dependency was not met at prefetch time: wait, then copy
+      bool ff = false;
+      if (w.team_lead) ff = !nx.wait_and_copy(nx.cur, w);
+      if (named_bar_or(w.bar_id, w.bar_count, ff)) {
+        w.fail = true;
+        break;
+      }
+      stg_pending = true;
+    }
+  }
+  if (w.fail && w.rho == 0) atomicCAS(a.err, 0, TCU_DFT_ERR_TIMEOUT);
+  // leave: copies of this warpgroup still landing (on failure), then the
+  // cluster -- the peer may arrive on this CTA's barriers until it is done
+  if (w.rho == 0 && w.fail) {
+    if (stg_pending) mbar_wait_bounded(w.bar_stg, w.ph_stg);
+    if (w.tws_inflight) mbar_wait_bounded(w.bar_tws, w.ph_tws);
+  }
+  fence_before_sync();
+  __syncthreads();
+  cluster_sync_all();
+  if ((threadIdx.x >> 5) == 0) {
+    fence_after_sync();
+    tmem_dealloc(tbase, 512);
+  }
 }
 
 }  // namespace tcu

@@ -156,6 +156,9 @@ struct tcu_dft_plan_s {
   float2 *scratch[2];      // intermediates (or the fused ring in scratch[0])
   // fused two-pass schedule
   bool fused;
+  // one HBM pass on cluster pairs (scratch[0]: two slots per cluster)
+  bool pair;
+  int pair_clusters;
   int log2C, nchunks, lag, ring_chunks;
   int items1_per_tf, log2_items_per_chunk;
   int *counters;

@@ -38,6 +38,13 @@ cudaError_t launch_fused_r16(int prec, int s1, int s2, const GArgs &a, int num_s
   return cudaErrorInvalidValue;
 }
 
+cudaError_t launch_pair_r16(int prec, int s1, int s2, const GArgs &a, int clusters,
+                            cudaStream_t st) {
+  constexpr int R = 16;
+  TCU_PAIR_CASE(2, 2)
+  return cudaErrorInvalidValue;
+}
+
 cudaError_t launch_rowconv_r16(int prec, int s, const GArgs &a, int num_sms,
                                cudaStream_t st) {
   constexpr int R = 16;

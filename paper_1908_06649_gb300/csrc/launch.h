@@ -28,6 +28,10 @@ cudaError_t launch_team_r8(int prec, int s, int lo, int role, int lp, int tw, co
 // Radix-16 team passes (kernels_r16.cu).
 cudaError_t launch_team_r16(int prec, int s, int lo, int role, int lp, int tw, const GArgs &a,
                             int num_sms, cudaStream_t st);
+// Both passes of a two-pass transform in one launch on clusters of two CTAs,
+// each cluster's intermediate in two L2-resident slots (radix 16, 2 + 2).
+cudaError_t launch_pair_r16(int prec, int s1, int s2, const GArgs &a, int clusters,
+                            cudaStream_t st);
 // Both passes of a two-pass transform fused in one launch (s1, s2 >= 2).
 cudaError_t launch_fused_r8(int prec, int s1, int s2, const GArgs &a, int num_sms,
                             cudaStream_t st);

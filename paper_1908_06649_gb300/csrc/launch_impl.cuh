@@ -1,6 +1,8 @@
 // launch_impl.cuh -- launch wrappers for one radix; included once per radix
 // by kernels_r8.cu / kernels_r16.cu / kernels_r32.cu.
 #pragma once
+#include <string.h>
+
 #include "launch.h"
 
 namespace tcu {
@@ -80,6 +82,36 @@ cudaError_t launch_fused_t(const GArgs &a, int num_sms, cudaStream_t st) {
   dft_fused_kernel<R, PREC, S1, S2><<<(unsigned)num_sms, G1::THREADS, sm, st>>>(a);
   return cudaGetLastError();
 }
+
+// Both passes of a two-pass transform in one launch on clusters of two CTAs
+// (dft_pair_kernel): grid = 2 x clusters, one CTA per SM.
+template <int R, int PREC, int S1, int S2>
+cudaError_t launch_pair_t(const GArgs &a, int clusters, cudaStream_t st) {
+  using PL = PairLayout<R, S1, S2>;
+  const size_t sm = PL::BYTES;
+  cudaError_t e = cudaFuncSetAttribute(dft_pair_kernel<R, PREC, S1, S2>,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, (int)sm);
+  if (e != cudaSuccess) return e;
+  cudaLaunchConfig_t cfg;
+  memset(&cfg, 0, sizeof(cfg));
+  cfg.gridDim = dim3((unsigned)(2 * clusters), 1, 1);
+  cfg.blockDim = dim3(PL::G1::THREADS, 1, 1);
+  cfg.dynamicSmemBytes = sm;
+  cfg.stream = st;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeClusterDimension;
+  attr[0].val.clusterDim.x = 2;
+  attr[0].val.clusterDim.y = 1;
+  attr[0].val.clusterDim.z = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, dft_pair_kernel<R, PREC, S1, S2>, a);
+}
+
+#define TCU_PAIR_CASE(S1, S2)                                                       \
+  if (s1 == S1 && s2 == S2)                                                         \
+    return prec == 3 ? launch_pair_t<R, 3, S1, S2>(a, clusters, st)                 \
+                     : launch_pair_t<R, 1, S1, S2>(a, clusters, st);
 
 // Supported combinations of the warpgroup pass kernel for radix R, listed as
 // a compile-time table; the plan only asks for these.  The dispatcher gets

@@ -275,13 +275,36 @@ int exec_impl(tcu_dft_plan_t p, const void *in, void *out, int dir,
     return TCU_DFT_ERR_INVALID;
   if (((uintptr_t)in & 15) || ((uintptr_t)out & 15)) return TCU_DFT_ERR_INVALID;
   if (count < 0) count = p->batch;
-  if (b0 < 0 || b0 + count > p->batch || (p->fused && count != p->batch))
+  if (b0 < 0 || b0 + count > p->batch || ((p->fused || p->pair) && count != p->batch))
     return TCU_DFT_ERR_INVALID;
   const size_t bytes = (size_t)count * p->n * sizeof(float2);
   if (in != out && overlaps(in, out, bytes)) return TCU_DFT_ERR_INVALID;
   cudaStream_t st = (cudaStream_t)stream;
   const int di = dir_index(dir);
   const bool inverse = dir == TCU_DFT_INVERSE;
+  if (p->pair) {
+    // both passes in one launch; cluster c's intermediates in slots 2c, 2c+1
+    GArgs g;
+    memset(&g, 0, sizeof(g));
+    g.p[0] = group_pass(p, 0, di, (const float2 *)in, p->scratch[0], -1, 1, inverse, p->batch);
+    g.p[1] = group_pass(p, 1, di, p->scratch[0], (float2 *)out, 1, -1, inverse, p->batch);
+    if (!input_map(&g.tm_in, in, p, p->pass[0], p->batch)) return TCU_DFT_ERR_CUDA;
+    g.tm_tw = p->pass[0].tw_map[di];
+    g.bimg = p->bimg[di];
+    g.err = p->err;
+    g.batch = p->batch;
+    g.items1_per_tf = p->items1_per_tf;
+    if (events && cudaEventRecord((cudaEvent_t)events[0], st) != cudaSuccess)
+      return TCU_DFT_ERR_CUDA;
+    const NvtxRange range("tcu_dft one pass (cluster pairs)");
+    if (launch_pair_r16(p->precision, p->pass[0].s, p->pass[1].s, g, p->pair_clusters, st) !=
+        cudaSuccess)
+      return TCU_DFT_ERR_CUDA;
+    if (events && (cudaEventRecord((cudaEvent_t)events[1], st) != cudaSuccess ||
+                   cudaEventRecord((cudaEvent_t)events[2], st) != cudaSuccess))
+      return TCU_DFT_ERR_CUDA;
+    return TCU_DFT_OK;
+  }
   if (p->fused) {
     GArgs g;
     memset(&g, 0, sizeof(g));
@@ -393,8 +416,9 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
   arm_alloc_faults();
   if (n < 1 || batch < 1 ||
       (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32 && !prec_bf16(precision)) ||
-      (flags & ~(uint32_t)(TCU_DFT_PLAN_NO_FUSE | TCU_DFT_PLAN_FUSE)) ||
-      ((flags & TCU_DFT_PLAN_NO_FUSE) && (flags & TCU_DFT_PLAN_FUSE))) {
+      (flags & ~(uint32_t)(TCU_DFT_PLAN_NO_FUSE | TCU_DFT_PLAN_FUSE | TCU_DFT_PLAN_ONE_PASS)) ||
+      ((flags & TCU_DFT_PLAN_NO_FUSE) && (flags & (TCU_DFT_PLAN_FUSE | TCU_DFT_PLAN_ONE_PASS))) ||
+      ((flags & TCU_DFT_PLAN_FUSE) && (flags & TCU_DFT_PLAN_ONE_PASS))) {
     g_last_error = TCU_DFT_ERR_INVALID;
     return nullptr;
   }
@@ -474,7 +498,19 @@ tcu_dft_plan_t tcu_dft_plan_ex(int64_t n, int64_t batch, int32_t sqrt_m,
     // fused kernels are instantiated for 2 + 2 stages
     p->fused = !is_mixed && !prec_bf16(precision) && npasses == 2 && p1.s == 2 &&
                p2.s == 2 && (flags & TCU_DFT_PLAN_FUSE);
+    // one HBM pass on cluster pairs: radix 16, 2 + 2 stages (n = 16^4)
+    p->pair = !is_mixed && !prec_bf16(precision) && r == 16 && npasses == 2 && p1.s == 2 &&
+              p2.s == 2 && (flags & TCU_DFT_PLAN_ONE_PASS) && p->num_sms >= 2;
     long long scratch_tf = batch;
+    if (p->pair) {
+      const long long gg1 = (128ll * r) >> p1.log2L;
+      p->items1_per_tf = (int)((1ll << p2.log2L) / gg1);
+      // one cluster per two SMs, no more than there are pairs of transforms;
+      // two slots of scratch per cluster
+      const long long pairs = (batch + 1) / 2;
+      p->pair_clusters = (int)(pairs < p->num_sms / 2 ? pairs : p->num_sms / 2);
+      scratch_tf = 2ll * p->pair_clusters;
+    }
     if (p->fused) {
       // chunks of C transforms (a power of two dividing the batch, <= 8);
       // pass 2 trails pass 1 by `lag` chunks; the ring holds 8 chunks and
@@ -562,7 +598,7 @@ int tcu_dft_exec_host(tcu_dft_plan_t p, const void *h_in, void *h_out, void *d_w
   if ((uintptr_t)d_work & 15) return TCU_DFT_ERR_INVALID;
   const size_t bytes = (size_t)p->batch * p->n * sizeof(float2);
   cudaStream_t st = (cudaStream_t)stream;
-  if (p->fused || !p->has_copy_streams || p->batch < 2) {
+  if (p->fused || p->pair || !p->has_copy_streams || p->batch < 2) {
     if (cudaMemcpyAsync(d_work, h_in, bytes, cudaMemcpyHostToDevice, st) != cudaSuccess)
       return TCU_DFT_ERR_CUDA;
     const int rc = tcu_dft_exec_dir(p, d_work, d_work, dir, stream);
@@ -650,7 +686,7 @@ int tcu_dft_plan_passes(int64_t n, int32_t sqrt_m, int32_t *stages) {
 
 int tcu_dft_num_passes(tcu_dft_plan_t p) { return p ? p->npasses : -1; }
 
-int tcu_dft_is_fused(tcu_dft_plan_t p) { return p ? (p->fused ? 1 : 0) : -1; }
+int tcu_dft_is_fused(tcu_dft_plan_t p) { return p ? ((p->fused || p->pair) ? 1 : 0) : -1; }
 
 int tcu_dft_pass_stages(tcu_dft_plan_t p, int i) {
   if (!p || i < 0 || i >= p->npasses) return -1;

@@ -107,9 +107,13 @@ def test_strerror_and_null_handling(lib):
     assert lib.tcu_dft_exec_stalled(None, None, None, None) == pkg.ERR_INVALID
     assert lib.tcu_dft_num_passes(None) == -1
     assert lib.tcu_dft_is_fused(None) == -1
-    assert not lib.tcu_dft_plan_ex(256, 4, 16, 3, 4)   # unknown flag bit
+    assert not lib.tcu_dft_plan_ex(256, 4, 16, 3, 8)   # unknown flag bit
     assert lib.tcu_dft_last_error() == pkg.ERR_INVALID
     assert not lib.tcu_dft_plan_ex(256, 4, 16, 3, 3)   # FUSE with NO_FUSE
+    assert lib.tcu_dft_last_error() == pkg.ERR_INVALID
+    assert not lib.tcu_dft_plan_ex(256, 4, 16, 3, 6)   # FUSE with ONE_PASS
+    assert lib.tcu_dft_last_error() == pkg.ERR_INVALID
+    assert not lib.tcu_dft_plan_ex(256, 4, 16, 3, 5)   # NO_FUSE with ONE_PASS
     assert lib.tcu_dft_last_error() == pkg.ERR_INVALID
     assert lib.tcu_dft_pass_stages(None, 0) == -1
 

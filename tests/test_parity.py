@@ -113,6 +113,63 @@ def test_fused_schedule_is_used(pkg, r, k):
     plan.destroy()
 
 
+# ---- one HBM pass on cluster pairs (TCU_DFT_PLAN_ONE_PASS, n = 16^4): both
+# passes in one launch, each cluster's intermediates in two L2 slots.  Batches
+# below, at and above the number of cluster pairs, odd batches (a last pair
+# of one transform), forward and inverse, in place.
+@pytest.mark.parametrize("batch", [1, 2, 3, 7, 40, 151, 152, 153, 305])
+def test_one_pass_pairs(pkg, batch):
+    n = 16 ** 4
+    x = inputs.make("normal", n, batch, seed=300 + batch)
+    y, passes = run(pkg, x, 16, 3, flags=pkg.PLAN_ONE_PASS)
+    assert passes == [2, 2]
+    check(y, x, 3)
+
+
+@pytest.mark.parametrize("prec", [3, 1])
+def test_one_pass_pairs_inverse_in_place(pkg, prec):
+    import torch
+    n, batch = 16 ** 4, 77
+    x = inputs.make("uniform", n, batch, seed=31)
+    plan = pkg.Plan(n, batch, 16, prec, pkg.PLAN_ONE_PASS)
+    assert plan.fused
+    xd = torch.from_numpy(x).cuda()
+    y = plan.exec(xd, xd, pkg.INVERSE)  # in place
+    plan.check()
+    got = y.cpu().numpy()
+    err = oracle.rel_l2(got, oracle.dft(x, inverse=True, threads=8))
+    assert err.max() <= TOL[prec]
+    # and forward again, out of place, from the inverse's output
+    z = plan.forward(y)
+    plan.check()
+    back = z.cpu().numpy()
+    rt = np.linalg.norm(back - x, axis=1) / np.linalg.norm(x, axis=1)
+    assert rt.max() <= (1e-5 if prec == 3 else 3e-3)
+    plan.destroy()
+
+
+def test_one_pass_pairs_repeated_calls(pkg):
+    # the slots and barriers start afresh at every launch: several launches
+    # in a row on the same plan give the same bits
+    import torch
+    n, batch = 16 ** 4, 200
+    x = torch.from_numpy(inputs.make("normal", n, batch, seed=32)).cuda()
+    plan = pkg.Plan(n, batch, 16, 3, pkg.PLAN_ONE_PASS)
+    outs = [plan.forward(x) for _ in range(3)]
+    plan.check()
+    for o in outs[1:]:
+        assert torch.equal(o, outs[0])
+    ref = pkg.Plan(n, batch, 16, 3)
+    y2 = ref.forward(x)
+    ref.check()
+    err = oracle.rel_l2(outs[0][:4].cpu().numpy(), oracle.dft(x[:4].cpu().numpy(), threads=8))
+    assert err.max() <= TOL[3]
+    d = (outs[0] - y2).abs().max().item() / y2.abs().max().item()
+    assert d < 1e-5
+    plan.destroy()
+    ref.destroy()
+
+
 @pytest.mark.parametrize("r,k", [(16, 2), (16, 4), (8, 4)])
 def test_inverse_fused(pkg, r, k):
     n = r ** k
