@@ -1461,39 +1461,24 @@ struct PairNext {
   // parity of the phase of full[s] / empty[s] that belongs to transform j
   __device__ static uint32_t par(int j) { return (uint32_t)(j >> 1) & 1u; }
 
-  __device__ void copy(const PairItem &it, const WG &w) {
-    if (it.type == 0) {
-      issue_input<G1>(p1, &a.tm_in, gitem(it), w);
-    } else {
-      fence_proxy_async_global();  // after the acquire of full[]
-      issue_input<G2>(p2, nullptr, gitem(it), w);
-    }
-  }
-  // warp 0 of the warpgroup, converged: the next item's input, unless it is
-  // a pass-2 item whose transform's pass-1 items are not all stored yet
+  // every thread of the warpgroup (the same decision in all of them), once
+  // the staging buffer is free: warp 0 copies the next item's input if it
+  // is a pass-1 item (a pass-2 item reads its own input from the slot)
   __device__ void issue(const WG &w) {
-    issued = false;
-    if (!nxt.valid) return;
-    if (nxt.type == 1) {
-      int ok = 0;
-      if ((threadIdx.x & 31) == 0)
-        ok = mbar_test_cluster(full_bar + 8 * (nxt.j & 1), par(nxt.j)) ? 1 : 0;
-      if (!__shfl_sync(0xffffffffu, ok, 0)) return;
-    }
-    copy(nxt, w);
-    issued = true;
+    issued = nxt.valid && nxt.type == 0;
+    if (issued && w.team_lead) issue_input<G1>(p1, &a.tm_in, gitem(nxt), w);
   }
-  // warp 0, converged: bounded wait for `it`'s dependency, then its copy
-  __device__ bool wait_and_copy(const PairItem &it, const WG &w) {
+  // warp 0, converged: bounded wait until every pass-1 item of transform j
+  // (both CTAs) has stored its part of the slot
+  __device__ bool wait_full(int j) const {
     int ok = 1;
-    if (it.type == 1 && (threadIdx.x & 31) == 0)
-      ok = mbar_wait_cluster_bounded(full_bar + 8 * (it.j & 1), par(it.j)) ? 1 : 0;
-    ok = __shfl_sync(0xffffffffu, ok, 0);
-    if (ok) copy(it, w);
-    return ok != 0;
+    if ((threadIdx.x & 31) == 0)
+      ok = mbar_wait_cluster_bounded(full_bar + 8 * (j & 1), par(j)) ? 1 : 0;
+    return __shfl_sync(0xffffffffu, ok, 0) != 0;
   }
   __device__ void publish() {}
-  // a pass-2 item's input has landed in SMEM: its slot may be overwritten
+  // every row of a pass-2 item has been read from its slot (the warpgroup's
+  // barrier follows the reads): the slot may be overwritten
   __device__ void after_load(const WG &w) {
     if (cur.type == 1 && w.team_lead) {
       if (elect_one()) {
@@ -1523,12 +1508,164 @@ struct PairNext {
   }
 };
 
+// Stage-1 row of a pass-2 item of the pair schedule, straight from the
+// L2-resident slot: L1 is bypassed (ld.global.cg), since the slot is
+// rewritten by other CTAs between transforms.
+template <class G>
+__device__ __forceinline__ void slot_row(const PRun &P, long long item, const WG &w,
+                                         float2 *x) {
+  constexpr int R = 1 << G::LOG2R;
+  static_assert(G::MODE_FIRST == kQF, "contiguous sub-transforms");
+  int ul, q;
+  row_of<G>(G::MODE_FIRST, w.rho, ul, q);
+  const long long u = (item << G::LOG2GG) + ul;
+  const long long b = u >> G::LOG2UPER, v = u & ((1ll << G::LOG2UPER) - 1);
+  const long long off = ((b & P.in_bmask) << G::LOG2N) + (v << G::LOG2L) + q;
+  const long long in_elems = (P.in_bmask + 1) << G::LOG2N;
+  constexpr int JS = 1 << (G::LOG2L - G::LOG2R);  // a = j * R^(S-1) + q
+#pragma unroll
+  for (int j = 0; j < R; ++j)
+    x[j] = in_range(w, off + j * JS, in_elems) ? __ldcg(P.in + off + j * JS)
+                                               : make_float2(0.f, 0.f);
+}
+
+// The inter-pass twiddles w_M^{k v} of this thread's last-stage outputs
+// (k = klow + j r^(S-1), column v) from the L2-resident table A [k][vl];
+// loaded while the last stage's products run.
+template <class G>
+__device__ __forceinline__ void out_twiddles(const PRun &P, long long item, const WG &w,
+                                             float2 *tw) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  static_assert(G::TW_OUT && !G::TW2L, "one-level inter-pass table");
+  int ul, q;
+  row_of<G>(G::MODE_LAST, w.rho, ul, q);
+  int klow = 0, vq = q;
+#pragma unroll
+  for (int i = 0; i < S - 1; ++i) {
+    klow = (klow << G::LOG2R) | (vq & (R - 1));
+    vq >>= G::LOG2R;
+  }
+  const long long u = (item << G::LOG2GG) + ul;
+  const long long vl = u & ((1ll << G::LOG2VL) - 1);
+  const long long goff = ((long long)klow << G::LOG2VL) + vl;
+  constexpr long long TWG = 1ll << (G::LOG2VL + G::LOG2L - G::LOG2R);
+#pragma unroll
+  for (int j = 0; j < R; ++j)
+    tw[j] = in_range(w, goff + j * TWG, (long long)G::L << G::LOG2VL) ? __ldg(P.tw_out + goff + j * TWG)
+                                                                       : make_float2(1.f, 0.f);
+}
+
+// Last stage of a pass-1 item of the pair schedule: D -> registers, times
+// the prefetched inter-pass twiddles, L2-cached stores into the slot.
+template <class G, int PREC>
+__device__ __forceinline__ void pair_first_store(const PRun &P, long long item, const WG &w,
+                                                 const float2 *tw) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  int ul, q;
+  row_of<G>(G::MODE_LAST, w.rho, ul, q);
+  const long long u = (item << G::LOG2GG) + ul;
+  float d[2 * R];
+  load_d_row<G, PREC>(w, d);
+  if (u >= P.U) return;
+  int klow = 0, vq = q;
+#pragma unroll
+  for (int i = 0; i < S - 1; ++i) {
+    klow = (klow << G::LOG2R) | (vq & (R - 1));
+    vq >>= G::LOG2R;
+  }
+  const long long b = u >> G::LOG2UPER;
+  const long long v = u & ((1ll << G::LOG2UPER) - 1);
+  float2 *dst = P.out + ((b & P.out_bmask) << G::LOG2NT) + v + klow * G::OUT_STRIDE;
+  constexpr long long JS = G::OUT_STRIDE << (G::LOG2L - G::LOG2R);
+  const long long doff = dst - P.out;
+  const long long out_elems = (P.out_bmask + 1) << G::LOG2NT;
+#pragma unroll
+  for (int j = 0; j < R; ++j) {
+    const float2 y = cmul(make_float2(d[2 * j], d[2 * j + 1]), tw[j]);
+    if (in_range(w, doff + j * JS, out_elems)) __stcg(dst + j * JS, y);
+  }
+}
+
+// One item of the pair schedule (two stages): TYPE 0 a pass-1 item (input
+// staged by TMA from HBM, output into the slot), TYPE 1 a pass-2 item
+// (input read from the slot, output to HBM).  `mid` prefetches the next
+// pass-1 item's input into the staging buffer once it is free.
+template <class G, int PREC, int TYPE, class Mid>
+__device__ __forceinline__ void process_pair_item(const PRun &P, const float2 *tws,
+                                                  long long item, WG &w, Mid &mid) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  static_assert(S == 2, "two stages per pass");
+  {
+    float2 x[R];
+    if constexpr (TYPE == 0) {
+      if (!mbar_wait_bounded(w.bar_stg, w.ph_stg)) w.fail = true;
+      w.ph_stg ^= 1;
+      staged_row<G>(w, x);
+    } else {
+      slot_row<G>(P, item, w, x);
+    }
+#pragma unroll
+    for (int c = 0; c < R; c += 8)
+      split_store8<PREC>(x + c, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
+                         w.slot + G::Q + w.lane_off + a_cols8(PREC) * c / 8);
+  }
+  tmem_wait_st();
+  fence_before_sync();
+  if (named_bar_or(w.bar_id, w.bar_count, w.fail)) {
+    w.fail = true;
+    return;
+  }
+  // every row of the item has been read: a pass-2 item's slot may be reused
+  if (TYPE == 1) mid.after_load(w);
+  if (w.wg_lead) {
+    fence_after_sync();
+    issue_stage<R, PREC>(w.slot, w.img_addr, w.bar_mma);
+  }
+  mid.issue(w);
+  if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
+  w.ph_mma ^= 1;
+  fence_after_sync();
+  stage_epilogue<G, PREC, 1>(P, tws, w);
+  fence_before_sync();
+  named_bar_or(w.bar_id, w.bar_count, false);
+  stage_rows<G, PREC, 2>(P, w);
+  tmem_wait_st();
+  fence_before_sync();
+  if (named_bar_or(w.bar_id, w.bar_count, w.fail)) {
+    w.fail = true;
+    return;
+  }
+  if (w.wg_lead) {
+    fence_after_sync();
+    issue_stage<R, PREC>(w.slot, w.img_addr + P.last_img, w.bar_mma);
+  }
+  if constexpr (TYPE == 0) {
+    float2 tw[R];
+    out_twiddles<G>(P, item, w, tw);
+    if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
+    w.ph_mma ^= 1;
+    fence_after_sync();
+    mid.before_store(w);
+    pair_first_store<G, PREC>(P, item, w, tw);
+  } else {
+    if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
+    w.ph_mma ^= 1;
+    fence_after_sync();
+    last_stage_store<G, PREC, false>(P, item, w);
+  }
+}
+
 template <int R, int S1, int S2>
 struct PairLayout {
   using G1 = Geo<R, S1, log2_radix(R) * S2, kFirst, 0, whole_k_nwg(R, kFirst)>;
+  // no twiddle staging: pass-1 items read their inter-pass twiddles from
+  // the L2-resident table while their last products run
   using SM = SmemLayout<R, G1::NWG, G1::TW_ENTRIES, Geo<R, S2, log2_radix(R) * S1, kSecond, 0,
                                                         G1::NWG>::TW_ENTRIES,
-                        G1::TW_SMEM, G1::TWB>;
+                        false, 0>;
   static constexpr size_t OFF_PBAR = (SM::BYTES + 15) / 16 * 16;  // full[2], empty[2]
   static constexpr size_t OFF_PRUN = OFF_PBAR + 32;               // per-CTA PRun copies
   static constexpr size_t BYTES = OFF_PRUN + 2 * sizeof(PRun);
@@ -1590,36 +1727,35 @@ __global__ void __launch_bounds__(
   const int wg = threadIdx.x >> 7;
   long long pos = wg;
   nx.cur = pair_decode(pos, H, J);
-  bool f = false;
-  if (w.team_lead && nx.cur.valid) f = !nx.wait_and_copy(nx.cur, w);
-  if (named_bar_or(w.bar_id, w.bar_count, f)) w.fail = true;
-  bool stg_pending = false;
+  // the first items are pass-1 items: their copies need no wait.  Every
+  // later pass-1 item's copy is issued during the item before it.  All
+  // control flow below is the same in the four warps of a warpgroup (the
+  // warpgroup's named barriers must match).
+  nx.issued = nx.cur.valid && nx.cur.type == 0;
+  if (nx.issued && w.team_lead) issue_input<G1>(prun[0], &a.tm_in, nx.gitem(nx.cur), w);
+  bool stg_pending = nx.issued;
   while (nx.cur.valid && !w.fail) {
     nx.nxt = pair_decode(pos + NWG, H, J);
     if (nx.cur.type == 0) {
-      process_item<G1, PREC, true>(prun[0], &a.tm_tw, tw1, nx.gitem(nx.cur), w, nx);
+      process_pair_item<G1, PREC, 0>(prun[0], tw1, nx.gitem(nx.cur), w, nx);
       // every thread's stores of the item, then its arrival on full[]
       if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;
       if (!w.fail && w.team_lead) nx.arrive_full(w);
     } else {
-      process_item<G2, PREC, false>(prun[1], &a.tm_tw, tw2, nx.gitem(nx.cur), w, nx);
-      // a uniform failure state before the next item's barriers
+      // every pass-1 item of the transform (both CTAs) has stored its part
+      bool f = false;
+      if (w.team_lead) f = !nx.wait_full(nx.cur.j);
+      if (named_bar_or(w.bar_id, w.bar_count, f)) {
+        w.fail = true;
+        break;
+      }
+      process_pair_item<G2, PREC, 1>(prun[1], tw2, nx.gitem(nx.cur), w, nx);
       if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;
     }
     stg_pending = nx.issued;
     if (w.fail) break;
     pos += NWG;
     nx.cur = nx.nxt;
-    if (nx.cur.valid && !nx.issued) {
-      // the dependency was not met at prefetch time: wait, then copy
-      bool ff = false;
-      if (w.team_lead) ff = !nx.wait_and_copy(nx.cur, w);
-      if (named_bar_or(w.bar_id, w.bar_count, ff)) {
-        w.fail = true;
-        break;
-      }
-      stg_pending = true;
-    }
   }
   if (w.fail && w.rho == 0) atomicCAS(a.err, 0, TCU_DFT_ERR_TIMEOUT);
   // leave: copies of this warpgroup still landing (on failure), then the
