@@ -1461,24 +1461,50 @@ struct PairNext {
   // parity of the phase of full[s] / empty[s] that belongs to transform j
   __device__ static uint32_t par(int j) { return (uint32_t)(j >> 1) & 1u; }
 
-  // every thread of the warpgroup (the same decision in all of them), once
-  // the staging buffer is free: warp 0 copies the next item's input if it
-  // is a pass-1 item (a pass-2 item reads its own input from the slot)
+  int *mailbox;  // this warpgroup's word in SMEM: a pass-2 prefetch was issued
+
+  __device__ void copy(const PairItem &it, const WG &w) {
+    if (it.type == 0) {
+      issue_input<G1>(p1, &a.tm_in, gitem(it), w);
+    } else {
+      fence_proxy_async_global();  // after the acquire of full[]
+      issue_input<G2>(p2, nullptr, gitem(it), w);
+    }
+  }
+  // every thread of the warpgroup, once the staging buffer is free: warp 0
+  // copies the next item's input -- a pass-1 item's always, a pass-2 item's
+  // only if its transform's pass-1 items are all stored (a non-blocking
+  // test; the answer reaches the other warps through the mailbox, read by
+  // sync() after the warpgroup's next barrier)
   __device__ void issue(const WG &w) {
     issued = nxt.valid && nxt.type == 0;
-    if (issued && w.team_lead) issue_input<G1>(p1, &a.tm_in, gitem(nxt), w);
-  }
-  // warp 0, converged: bounded wait until every pass-1 item of transform j
-  // (both CTAs) has stored its part of the slot
-  __device__ bool wait_full(int j) const {
+    if (!nxt.valid || !w.team_lead) return;
     int ok = 1;
-    if ((threadIdx.x & 31) == 0)
-      ok = mbar_wait_cluster_bounded(full_bar + 8 * (j & 1), par(j)) ? 1 : 0;
-    return __shfl_sync(0xffffffffu, ok, 0) != 0;
+    if (nxt.type == 1) {
+      if ((threadIdx.x & 31) == 0)
+        ok = mbar_test_cluster(full_bar + 8 * (nxt.j & 1), par(nxt.j)) ? 1 : 0;
+      ok = __shfl_sync(0xffffffffu, ok, 0);
+      if ((threadIdx.x & 31) == 0) *mailbox = ok;
+    }
+    if (ok) copy(nxt, w);
   }
+  // every thread, after the warpgroup barrier that follows issue()
+  __device__ void sync() {
+    if (nxt.valid && nxt.type == 1) issued = *(volatile int *)mailbox != 0;
+  }
+  // warp 0, converged: bounded wait for a pass-2 item's dependency, then its
+  // copy (the prefetch found the dependency unmet)
+  __device__ bool wait_and_copy(const PairItem &it, const WG &w) {
+    int ok = 1;
+    if (it.type == 1 && (threadIdx.x & 31) == 0)
+      ok = mbar_wait_cluster_bounded(full_bar + 8 * (it.j & 1), par(it.j)) ? 1 : 0;
+    ok = __shfl_sync(0xffffffffu, ok, 0);
+    if (ok) copy(it, w);
+    return ok != 0;
+  }
+
   __device__ void publish() {}
-  // every row of a pass-2 item has been read from its slot (the warpgroup's
-  // barrier follows the reads): the slot may be overwritten
+  // a pass-2 item's input has landed in SMEM: its slot may be overwritten
   __device__ void after_load(const WG &w) {
     if (cur.type == 1 && w.team_lead) {
       if (elect_one()) {
@@ -1507,27 +1533,6 @@ struct PairNext {
     __syncwarp();
   }
 };
-
-// Stage-1 row of a pass-2 item of the pair schedule, straight from the
-// L2-resident slot: L1 is bypassed (ld.global.cg), since the slot is
-// rewritten by other CTAs between transforms.
-template <class G>
-__device__ __forceinline__ void slot_row(const PRun &P, long long item, const WG &w,
-                                         float2 *x) {
-  constexpr int R = 1 << G::LOG2R;
-  static_assert(G::MODE_FIRST == kQF, "contiguous sub-transforms");
-  int ul, q;
-  row_of<G>(G::MODE_FIRST, w.rho, ul, q);
-  const long long u = (item << G::LOG2GG) + ul;
-  const long long b = u >> G::LOG2UPER, v = u & ((1ll << G::LOG2UPER) - 1);
-  const long long off = ((b & P.in_bmask) << G::LOG2N) + (v << G::LOG2L) + q;
-  const long long in_elems = (P.in_bmask + 1) << G::LOG2N;
-  constexpr int JS = 1 << (G::LOG2L - G::LOG2R);  // a = j * R^(S-1) + q
-#pragma unroll
-  for (int j = 0; j < R; ++j)
-    x[j] = in_range(w, off + j * JS, in_elems) ? __ldcg(P.in + off + j * JS)
-                                               : make_float2(0.f, 0.f);
-}
 
 // The inter-pass twiddles w_M^{k v} of this thread's last-stage outputs
 // (k = klow + j r^(S-1), column v) from the L2-resident table A [k][vl];
@@ -1590,23 +1595,21 @@ __device__ __forceinline__ void pair_first_store(const PRun &P, long long item, 
 
 // One item of the pair schedule (two stages): TYPE 0 a pass-1 item (input
 // staged by TMA from HBM, output into the slot), TYPE 1 a pass-2 item
-// (input read from the slot, output to HBM).  `mid` prefetches the next
-// pass-1 item's input into the staging buffer once it is free.
+// (input staged by TMA from the slot, output to HBM).  `mid` prefetches the
+// next item's input into the staging buffer once it is free.
 template <class G, int PREC, int TYPE, class Mid>
 __device__ __forceinline__ void process_pair_item(const PRun &P, const float2 *tws,
                                                   long long item, WG &w, Mid &mid) {
   constexpr int R = 1 << G::LOG2R;
   constexpr int S = G::LOG2L / G::LOG2R;
   static_assert(S == 2, "two stages per pass");
+  if (!mbar_wait_bounded(w.bar_stg, w.ph_stg)) w.fail = true;
+  w.ph_stg ^= 1;
+  // a pass-2 item's input has landed: its slot may be overwritten
+  if (TYPE == 1) mid.after_load(w);
   {
     float2 x[R];
-    if constexpr (TYPE == 0) {
-      if (!mbar_wait_bounded(w.bar_stg, w.ph_stg)) w.fail = true;
-      w.ph_stg ^= 1;
-      staged_row<G>(w, x);
-    } else {
-      slot_row<G>(P, item, w, x);
-    }
+    staged_row<G>(w, x);
 #pragma unroll
     for (int c = 0; c < R; c += 8)
       split_store8<PREC>(x + c, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
@@ -1618,12 +1621,11 @@ __device__ __forceinline__ void process_pair_item(const PRun &P, const float2 *t
     w.fail = true;
     return;
   }
-  // every row of the item has been read: a pass-2 item's slot may be reused
-  if (TYPE == 1) mid.after_load(w);
   if (w.wg_lead) {
     fence_after_sync();
     issue_stage<R, PREC>(w.slot, w.img_addr, w.bar_mma);
   }
+  // the staging buffer is free: the next item's copy
   mid.issue(w);
   if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
   w.ph_mma ^= 1;
@@ -1631,6 +1633,7 @@ __device__ __forceinline__ void process_pair_item(const PRun &P, const float2 *t
   stage_epilogue<G, PREC, 1>(P, tws, w);
   fence_before_sync();
   named_bar_or(w.bar_id, w.bar_count, false);
+  mid.sync();
   stage_rows<G, PREC, 2>(P, w);
   tmem_wait_st();
   fence_before_sync();
@@ -1667,7 +1670,8 @@ struct PairLayout {
                                                         G1::NWG>::TW_ENTRIES,
                         false, 0>;
   static constexpr size_t OFF_PBAR = (SM::BYTES + 15) / 16 * 16;  // full[2], empty[2]
-  static constexpr size_t OFF_PRUN = OFF_PBAR + 32;               // per-CTA PRun copies
+  static constexpr size_t OFF_MBOX = OFF_PBAR + 32;               // a word per warpgroup
+  static constexpr size_t OFF_PRUN = OFF_MBOX + 16 * 4;           // per-CTA PRun copies
   static constexpr size_t BYTES = OFF_PRUN + 2 * sizeof(PRun);
   static_assert(BYTES <= 227 * 1024, "shared memory budget");
 };
@@ -1725,6 +1729,7 @@ __global__ void __launch_bounds__(
                       (uint32_t)(crank ^ 1), cid, nc, crank, H, J};
   nx.issued = false;
   const int wg = threadIdx.x >> 7;
+  nx.mailbox = reinterpret_cast<int *>(smem + PL::OFF_MBOX) + wg;
   long long pos = wg;
   nx.cur = pair_decode(pos, H, J);
   // the first items are pass-1 items: their copies need no wait.  Every
@@ -1742,13 +1747,6 @@ __global__ void __launch_bounds__(
       if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;
       if (!w.fail && w.team_lead) nx.arrive_full(w);
     } else {
-      // every pass-1 item of the transform (both CTAs) has stored its part
-      bool f = false;
-      if (w.team_lead) f = !nx.wait_full(nx.cur.j);
-      if (named_bar_or(w.bar_id, w.bar_count, f)) {
-        w.fail = true;
-        break;
-      }
       process_pair_item<G2, PREC, 1>(prun[1], tw2, nx.gitem(nx.cur), w, nx);
       if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;
     }
@@ -1756,6 +1754,17 @@ __global__ void __launch_bounds__(
     if (w.fail) break;
     pos += NWG;
     nx.cur = nx.nxt;
+    if (nx.cur.valid && !nx.issued) {
+      // a pass-2 item whose dependency was unmet at prefetch time: wait
+      // (bounded), then copy; the same branch in every warp
+      bool f = false;
+      if (w.team_lead) f = !nx.wait_and_copy(nx.cur, w);
+      if (named_bar_or(w.bar_id, w.bar_count, f)) {
+        w.fail = true;
+        break;
+      }
+      stg_pending = true;
+    }
   }
   if (w.fail && w.rho == 0) atomicCAS(a.err, 0, TCU_DFT_ERR_TIMEOUT);
   // leave: copies of this warpgroup still landing (on failure), then the
