@@ -413,9 +413,9 @@ __device__ __forceinline__ void load_d_row(const WG &w, float *d) {
 
 // ---- TMA issue (warp 0 of the warpgroup, converged; one elected lane
 // issues): the input block of `item` into staging
-template <class G>
+template <class G, bool HINT = false>
 __device__ __forceinline__ void issue_input(const PRun &P, const CUtensorMap *tm,
-                                            long long item, const WG &w) {
+                                            long long item, const WG &w, uint64_t pol = 0) {
   const long long u0 = item << G::LOG2GG;
   const uint32_t dst = smem_u32(w.stg);
   if (G::MODE_FIRST == kUF) {
@@ -425,8 +425,12 @@ __device__ __forceinline__ void issue_input(const PRun &P, const CUtensorMap *tm
     if (elect_one()) {
       mbar_expect_tx(w.bar_stg, G::GPTS * 8);
 #pragma unroll
-      for (int a0 = 0; a0 < G::L; a0 += G::TMA_ROWS)
-        tma_load_3d(dst + a0 * G::GG * 8, tm, 2 * v0, a0, (int)b, w.bar_stg);
+      for (int a0 = 0; a0 < G::L; a0 += G::TMA_ROWS) {
+        if (HINT)
+          tma_load_3d_hint(dst + a0 * G::GG * 8, tm, 2 * v0, a0, (int)b, w.bar_stg, pol);
+        else
+          tma_load_3d(dst + a0 * G::GG * 8, tm, 2 * v0, a0, (int)b, w.bar_stg);
+      }
     }
   } else {
     // contiguous block of GG sub-transforms (the last item may be short)
@@ -443,7 +447,12 @@ __device__ __forceinline__ void issue_input(const PRun &P, const CUtensorMap *tm
     if (elect_one()) {
       // a skipped copy still completes the phase (no bytes expected)
       mbar_expect_tx(w.bar_stg, ok ? bytes : 0u);
-      if (ok) tma_load_1d(dst, src, bytes, w.bar_stg);
+      if (ok) {
+        if (HINT)
+          tma_load_1d_hint(dst, src, bytes, w.bar_stg, pol);
+        else
+          tma_load_1d(dst, src, bytes, w.bar_stg);
+      }
     }
   }
   __syncwarp();
@@ -1463,12 +1472,16 @@ struct PairNext {
 
   int *mailbox;  // this warpgroup's word in SMEM: a pass-2 prefetch was issued
 
+  uint64_t pol_first, pol_last;  // L2 policies: streaming data, the slots
+
+  // the input x streams through L2 (first out); a slot is read back
+  // without lowering its priority, since pass 1 rewrites it
   __device__ void copy(const PairItem &it, const WG &w) {
     if (it.type == 0) {
-      issue_input<G1>(p1, &a.tm_in, gitem(it), w);
+      issue_input<G1, true>(p1, &a.tm_in, gitem(it), w, pol_first);
     } else {
       fence_proxy_async_global();  // after the acquire of full[]
-      issue_input<G2>(p2, nullptr, gitem(it), w);
+      issue_input<G2, true>(p2, nullptr, gitem(it), w, pol_last);
     }
   }
   // every thread of the warpgroup, once the staging buffer is free: warp 0
@@ -1522,13 +1535,15 @@ struct PairNext {
         !mbar_wait_cluster_bounded(empty_bar + 8 * (cur.j & 1), par(cur.j - 2)))
       w.fail = true;
   }
-  // after the warpgroup's barrier that follows a pass-1 item's stores
-  __device__ void arrive_full(const WG &w) {
+  // after the warpgroup's barrier that follows the last of this
+  // warpgroup's `count` pass-1 items of a transform: their stores, then
+  // `count` arrivals on full[] of both CTAs
+  __device__ void arrive_full(const WG &w, uint32_t count) {
     if (elect_one()) {
       fence_acq_rel_cluster();
       const uint32_t b = full_bar + 8 * (cur.j & 1);
-      mbar_arrive_cluster_local(b);
-      mbar_arrive_cluster_remote(mapa_shared(b, peer));
+      mbar_arrive_cluster_local_n(b, count);
+      mbar_arrive_cluster_remote_n(mapa_shared(b, peer), count);
     }
     __syncwarp();
   }
@@ -1562,10 +1577,10 @@ __device__ __forceinline__ void out_twiddles(const PRun &P, long long item, cons
 }
 
 // Last stage of a pass-1 item of the pair schedule: D -> registers, times
-// the prefetched inter-pass twiddles, L2-cached stores into the slot.
+// the prefetched inter-pass twiddles, stores into the slot (last out of L2).
 template <class G, int PREC>
 __device__ __forceinline__ void pair_first_store(const PRun &P, long long item, const WG &w,
-                                                 const float2 *tw) {
+                                                 const float2 *tw, uint64_t pol) {
   constexpr int R = 1 << G::LOG2R;
   constexpr int S = G::LOG2L / G::LOG2R;
   int ul, q;
@@ -1589,8 +1604,41 @@ __device__ __forceinline__ void pair_first_store(const PRun &P, long long item, 
 #pragma unroll
   for (int j = 0; j < R; ++j) {
     const float2 y = cmul(make_float2(d[2 * j], d[2 * j + 1]), tw[j]);
-    if (in_range(w, doff + j * JS, out_elems)) __stcg(dst + j * JS, y);
+    if (in_range(w, doff + j * JS, out_elems)) st_global_hint(dst + j * JS, y, pol);
   }
+}
+
+// Last stage of a pass-2 item of the pair schedule: D -> registers ->
+// natural-order output (first out of L2).
+template <class G, int PREC>
+__device__ __forceinline__ void pair_second_store(const PRun &P, long long item, const WG &w,
+                                                  uint64_t pol) {
+  constexpr int R = 1 << G::LOG2R;
+  constexpr int S = G::LOG2L / G::LOG2R;
+  static_assert(G::MODE_LAST == kUF && !G::TW_OUT, "last pass of several");
+  int ul, q;
+  row_of<G>(G::MODE_LAST, w.rho, ul, q);
+  const long long u = (item << G::LOG2GG) + ul;
+  float d[2 * R];
+  load_d_row<G, PREC>(w, d);
+  if (u >= P.U) return;
+  int klow = 0, vq = q;
+#pragma unroll
+  for (int i = 0; i < S - 1; ++i) {
+    klow = (klow << G::LOG2R) | (vq & (R - 1));
+    vq >>= G::LOG2R;
+  }
+  const long long b = u >> G::LOG2UPER;
+  const long long v = u & ((1ll << G::LOG2UPER) - 1);
+  float2 *dst = P.out + ((b & P.out_bmask) << G::LOG2NT) + v + klow * G::OUT_STRIDE;
+  constexpr long long JS = G::OUT_STRIDE << (G::LOG2L - G::LOG2R);
+  const long long doff = dst - P.out;
+  const long long out_elems =
+      P.out_bmask == -1 ? (P.U << G::LOG2L) : ((P.out_bmask + 1) << G::LOG2NT);
+#pragma unroll
+  for (int j = 0; j < R; ++j)
+    if (in_range(w, doff + j * JS, out_elems))
+      st_global_hint(dst + j * JS, make_float2(d[2 * j], d[2 * j + 1]), pol);
 }
 
 // One item of the pair schedule (two stages): TYPE 0 a pass-1 item (input
@@ -1652,12 +1700,12 @@ __device__ __forceinline__ void process_pair_item(const PRun &P, const float2 *t
     w.ph_mma ^= 1;
     fence_after_sync();
     mid.before_store(w);
-    pair_first_store<G, PREC>(P, item, w, tw);
+    pair_first_store<G, PREC>(P, item, w, tw, mid.pol_last);
   } else {
     if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
     w.ph_mma ^= 1;
     fence_after_sync();
-    last_stage_store<G, PREC, false>(P, item, w);
+    pair_second_store<G, PREC>(P, item, w, mid.pol_first);
   }
 }
 
@@ -1693,6 +1741,8 @@ __global__ void __launch_bounds__(
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 3 * NWG);
   uint64_t *pbar = reinterpret_cast<uint64_t *>(smem + PL::OFF_PBAR);
   PRun *prun = reinterpret_cast<PRun *>(smem + PL::OFF_PRUN);
+  // H items per CTA and pass of a transform, a multiple of the warpgroups
+  // (every warpgroup takes the same number of a transform's pass-1 items)
   const int H = a.items1_per_tf / 2;
   const long long cid = cluster_id_x(), nc = nclusters_x();
   const int crank = (int)cluster_ctarank();
@@ -1736,16 +1786,22 @@ __global__ void __launch_bounds__(
   // later pass-1 item's copy is issued during the item before it.  All
   // control flow below is the same in the four warps of a warpgroup (the
   // warpgroup's named barriers must match).
+  nx.pol_first = l2_policy_evict_first();
+  nx.pol_last = l2_policy_evict_last();
   nx.issued = nx.cur.valid && nx.cur.type == 0;
-  if (nx.issued && w.team_lead) issue_input<G1>(prun[0], &a.tm_in, nx.gitem(nx.cur), w);
+  if (nx.issued && w.team_lead) nx.copy(nx.cur, w);
   bool stg_pending = nx.issued;
   while (nx.cur.valid && !w.fail) {
     nx.nxt = pair_decode(pos + NWG, H, J);
     if (nx.cur.type == 0) {
       process_pair_item<G1, PREC, 0>(prun[0], tw1, nx.gitem(nx.cur), w, nx);
-      // every thread's stores of the item, then its arrival on full[]
+      // every thread's stores of the item; after this warpgroup's last
+      // pass-1 item of the transform (items m, m - NWG, ... of the H
+      // consecutive positions of its pass-1 items) the arrivals of all of
+      // them on full[]
       if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;
-      if (!w.fail && w.team_lead) nx.arrive_full(w);
+      if (!w.fail && w.team_lead && nx.cur.m + NWG >= H)
+        nx.arrive_full(w, (uint32_t)(nx.cur.m / NWG + 1));
     } else {
       process_pair_item<G2, PREC, 1>(prun[1], tw2, nx.gitem(nx.cur), w, nx);
       if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;

@@ -347,6 +347,19 @@ __device__ __forceinline__ void mbar_arrive_cluster_remote(uint32_t cluster_addr
                    cluster_addr)
                : "memory");
 }
+// `count` arrivals at once
+__device__ __forceinline__ void mbar_arrive_cluster_local_n(uint32_t addr, uint32_t count) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cta.b64 _, [%0], %1;" ::"r"(addr),
+               "r"(count)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_cluster_remote_n(uint32_t cluster_addr,
+                                                             uint32_t count) {
+  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0], %1;" ::"r"(
+                   cluster_addr),
+               "r"(count)
+               : "memory");
+}
 // Non-blocking test / bounded wait for completion of the phase of parity
 // `parity`, acquiring at cluster scope what the arrivals released.
 __device__ __forceinline__ bool mbar_test_cluster(uint32_t addr, uint32_t parity) {
@@ -360,17 +373,63 @@ __device__ __forceinline__ bool mbar_test_cluster(uint32_t addr, uint32_t parity
       : "memory");
   return ok != 0;
 }
+__device__ __forceinline__ bool mbar_try_cluster(uint32_t addr, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
+      "selp.b32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(addr), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
 __device__ __forceinline__ bool mbar_wait_cluster_bounded(uint32_t addr, uint32_t parity) {
-  if (mbar_test_cluster(addr, parity)) return true;
+  if (mbar_try_cluster(addr, parity)) return true;
   const unsigned long long t0 = global_ns();
   while (true) {
-    if (mbar_test_cluster(addr, parity)) return true;
+    if (mbar_try_cluster(addr, parity)) return true;
     if (global_ns() - t0 > kWaitNs) return false;
-    __nanosleep(32);
   }
 }
 __device__ __forceinline__ void fence_acq_rel_cluster() {
   asm volatile("fence.acq_rel.cluster;" ::: "memory");
+}
+
+// --------------------------------------------------- L2 eviction priority
+// Cache policies for the L2 (all of a thread's accesses with the policy):
+// streaming data first out, data that is read back soon last out.
+__device__ __forceinline__ uint64_t l2_policy_evict_first() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_first.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ uint64_t l2_policy_evict_last() {
+  uint64_t p;
+  asm volatile("createpolicy.fractional.L2::evict_last.b64 %0, 1.0;" : "=l"(p));
+  return p;
+}
+__device__ __forceinline__ void st_global_hint(float2 *p, float2 v, uint64_t pol) {
+  asm volatile("st.global.L1::no_allocate.L2::cache_hint.v2.f32 [%0], {%1, %2}, %3;" ::"l"(p),
+               "f"(v.x), "f"(v.y), "l"(pol)
+               : "memory");
+}
+// tma_load_1d / tma_load_3d with an L2 cache policy
+__device__ __forceinline__ void tma_load_1d_hint(uint32_t smem_dst, const void *gsrc,
+                                                 uint32_t bytes, uint32_t mbar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes.L2::cache_hint "
+      "[%0], [%1], %2, [%3], %4;" ::"r"(smem_dst),
+      "l"(gsrc), "r"(bytes), "r"(mbar), "l"(pol)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_3d_hint(uint32_t smem_dst, const void *tmap, int c0,
+                                                 int c1, int c2, uint32_t mbar, uint64_t pol) {
+  asm volatile(
+      "cp.async.bulk.tensor.3d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".L2::cache_hint [%0], [%1, {%2, %3, %4}], [%5], %6;" ::"r"(smem_dst),
+      "l"(tmap), "r"(c0), "r"(c1), "r"(c2), "r"(mbar), "l"(pol)
+      : "memory");
 }
 
 // Order this thread's earlier generic-proxy accesses (e.g. an acquire of a
