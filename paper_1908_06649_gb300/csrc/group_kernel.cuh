@@ -1517,13 +1517,15 @@ struct PairNext {
   }
 
   __device__ void publish() {}
-  // a pass-2 item's input has landed in SMEM: its slot may be overwritten
+  // a pass-2 item's input has landed in SMEM: its slot may be overwritten.
+  // The arrival orders nothing but that copy, which has completed, so it is
+  // relaxed (a release would wait for this warp's stores still in flight).
   __device__ void after_load(const WG &w) {
     if (cur.type == 1 && w.team_lead) {
       if (elect_one()) {
         const uint32_t b = empty_bar + 8 * (cur.j & 1);
-        mbar_arrive_cluster_local(b);
-        mbar_arrive_cluster_remote(mapa_shared(b, peer));
+        mbar_arrive_relaxed_local(b);
+        mbar_arrive_relaxed_remote(mapa_shared(b, peer));
       }
       __syncwarp();
     }
@@ -1535,17 +1537,22 @@ struct PairNext {
         !mbar_wait_cluster_bounded(empty_bar + 8 * (cur.j & 1), par(cur.j - 2)))
       w.fail = true;
   }
-  // after the warpgroup's barrier that follows the last of this
-  // warpgroup's `count` pass-1 items of a transform: their stores, then
-  // `count` arrivals on full[] of both CTAs
-  __device__ void arrive_full(const WG &w, uint32_t count) {
+  // pending publication of this warpgroup's pass-1 items of one transform
+  int pend_j;
+  uint32_t pend_count;  // 0: none
+  // warp 0, converged, some time after the warpgroup's barrier that follows
+  // the last of its `pend_count` pass-1 items of transform pend_j (their
+  // stores have drained by then, so the fence is cheap): a release at
+  // cluster scope, then pend_count arrivals on full[] of both CTAs
+  __device__ void publish_full() {
     if (elect_one()) {
       fence_acq_rel_cluster();
-      const uint32_t b = full_bar + 8 * (cur.j & 1);
-      mbar_arrive_cluster_local_n(b, count);
-      mbar_arrive_cluster_remote_n(mapa_shared(b, peer), count);
+      const uint32_t b = full_bar + 8 * (pend_j & 1);
+      mbar_arrive_cluster_local_n(b, pend_count);
+      mbar_arrive_cluster_remote_n(mapa_shared(b, peer), pend_count);
     }
     __syncwarp();
+    pend_count = 0;
   }
 };
 
@@ -1672,12 +1679,14 @@ __device__ __forceinline__ void process_pair_item(const PRun &P, const float2 *t
   if (w.wg_lead) {
     fence_after_sync();
     issue_stage<R, PREC>(w.slot, w.img_addr, w.bar_mma);
+    // the previous pass-1 items' stores have had an item's time to drain
+    if (mid.pend_count) mid.publish_full();
   }
-  // the staging buffer is free: the next item's copy
-  mid.issue(w);
   if (!mbar_wait_bounded(w.bar_mma, w.ph_mma)) w.fail = true;
   w.ph_mma ^= 1;
   fence_after_sync();
+  // the staging buffer is free: the next item's copy
+  mid.issue(w);
   stage_epilogue<G, PREC, 1>(P, tws, w);
   fence_before_sync();
   named_bar_or(w.bar_id, w.bar_count, false);
@@ -1786,6 +1795,7 @@ __global__ void __launch_bounds__(
   // later pass-1 item's copy is issued during the item before it.  All
   // control flow below is the same in the four warps of a warpgroup (the
   // warpgroup's named barriers must match).
+  nx.pend_count = 0;
   nx.pol_first = l2_policy_evict_first();
   nx.pol_last = l2_policy_evict_last();
   nx.issued = nx.cur.valid && nx.cur.type == 0;
@@ -1800,8 +1810,10 @@ __global__ void __launch_bounds__(
       // consecutive positions of its pass-1 items) the arrivals of all of
       // them on full[]
       if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;
-      if (!w.fail && w.team_lead && nx.cur.m + NWG >= H)
-        nx.arrive_full(w, (uint32_t)(nx.cur.m / NWG + 1));
+      if (nx.cur.m + NWG >= H) {
+        nx.pend_j = nx.cur.j;
+        nx.pend_count = (uint32_t)(nx.cur.m / NWG + 1);
+      }
     } else {
       process_pair_item<G2, PREC, 1>(prun[1], tw2, nx.gitem(nx.cur), w, nx);
       if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;
@@ -1811,9 +1823,11 @@ __global__ void __launch_bounds__(
     pos += NWG;
     nx.cur = nx.nxt;
     if (nx.cur.valid && !nx.issued) {
-      // a pass-2 item whose dependency was unmet at prefetch time: wait
-      // (bounded), then copy; the same branch in every warp
+      // a pass-2 item whose dependency was unmet at prefetch time: publish
+      // this warpgroup's own pending pass-1 items (it may be waiting for
+      // them), wait (bounded), then copy; the same branch in every warp
       bool f = false;
+      if (w.team_lead && nx.pend_count) nx.publish_full();
       if (w.team_lead) f = !nx.wait_and_copy(nx.cur, w);
       if (named_bar_or(w.bar_id, w.bar_count, f)) {
         w.fail = true;
@@ -1822,6 +1836,9 @@ __global__ void __launch_bounds__(
       stg_pending = true;
     }
   }
+  // a last publication (after the last item nobody waits for it, but the
+  // arrivals keep the barriers' counts whole)
+  if (!w.fail && w.team_lead && nx.pend_count) nx.publish_full();
   if (w.fail && w.rho == 0) atomicCAS(a.err, 0, TCU_DFT_ERR_TIMEOUT);
   // leave: copies of this warpgroup still landing (on failure), then the
   // cluster -- the peer may arrive on this CTA's barriers until it is done

@@ -347,6 +347,17 @@ __device__ __forceinline__ void mbar_arrive_cluster_remote(uint32_t cluster_addr
                    cluster_addr)
                : "memory");
 }
+// Relaxed arrivals: no ordering of this thread's earlier accesses (for a
+// signal that orders nothing but loads that have already completed).
+__device__ __forceinline__ void mbar_arrive_relaxed_local(uint32_t addr) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cta.b64 _, [%0];" ::"r"(addr)
+               : "memory");
+}
+__device__ __forceinline__ void mbar_arrive_relaxed_remote(uint32_t cluster_addr) {
+  asm volatile("mbarrier.arrive.relaxed.cluster.shared::cluster.b64 _, [%0];" ::"r"(
+                   cluster_addr)
+               : "memory");
+}
 // `count` arrivals at once
 __device__ __forceinline__ void mbar_arrive_cluster_local_n(uint32_t addr, uint32_t count) {
   asm volatile("mbarrier.arrive.release.cluster.shared::cta.b64 _, [%0], %1;" ::"r"(addr),
