@@ -173,8 +173,8 @@ cudaError_t launch_extract_tiles(float *Ak, const float2 *tiles, long long side,
 }  // namespace tcu
 
 // ---------------------------------------------------------- mixed radix
-// The q-point pass of a mixed-radix transform n = q R^k (q < R, a power of
-// two): the four-step split n = q x n2 with the q-point DFTs over the
+// The q-point pass of a mixed-radix transform n = q R^k (q = 2 .. 16, any
+// integer): the four-step split n = q x n2 with the q-point DFTs over the
 // stride-n2 columns done on the CUDA cores -- for q <= 16 a tensor-core
 // product would be mostly padding -- straight from the definition
 // y_k = sum_a x_a w_q^{a k}, then the inter-pass twiddle w_n^{k v} from the
@@ -221,8 +221,19 @@ cudaError_t launch_radix_q(int q, const float2 *x, float2 *out, long long batch,
   const unsigned grid = grid_for(batch << log2n2, num_sms);
   switch (q) {
     case 2: radix_q_kernel<2><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 3: radix_q_kernel<3><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
     case 4: radix_q_kernel<4><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 5: radix_q_kernel<5><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 6: radix_q_kernel<6><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 7: radix_q_kernel<7><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
     case 8: radix_q_kernel<8><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 9: radix_q_kernel<9><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 10: radix_q_kernel<10><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 11: radix_q_kernel<11><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 12: radix_q_kernel<12><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 13: radix_q_kernel<13><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 14: radix_q_kernel<14><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
+    case 15: radix_q_kernel<15><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
     case 16: radix_q_kernel<16><<<grid, kBlock, 0, st>>>(x, out, batch, log2n2, twA, twB, roots); break;
     default: return cudaErrorInvalidValue;
   }

@@ -185,7 +185,7 @@ tcu_dft2_plan_s *make_dft2(int64_t n1, int64_t n2, int64_t batch, int32_t r,
   for (int d = 0; d < 2 && rc == TCU_DFT_OK; ++d) {
     const int sign = d == 0 ? -1 : 1;
     std::vector<float> img;
-    build_images(r, sign, ilog2(n1 * n2), precision, img);
+    build_images(r, sign, n1 * n2, precision, img);
     rc = upload(&p->bimg[d], img);
     // hi and lo of this direction (the first two images)
     conv_img.insert(conv_img.end(), img.begin(), img.begin() + img.size() / 2);

@@ -56,7 +56,10 @@
 namespace tcu {
 
 enum RowMode { kQF = 0, kUF = 1, kRQF = 2 };
-enum Role { kSingle = 0, kFirst = 1, kSecond = 2, kCols = 3 };
+// kSecondQ: the last pass of a mixed-radix transform n = q R^S whose factor
+// q (2 .. 16, any integer) is a runtime value: the q-point first pass's
+// output T[b n + v L + a], v < q, -> y[b n + v + k q]
+enum Role { kSingle = 0, kFirst = 1, kSecond = 2, kCols = 3, kSecondQ = 4 };
 
 __host__ __device__ constexpr int log2_radix(int R) { return R == 8 ? 3 : (R == 16 ? 4 : 5); }
 // Warpgroups per CTA: TMEM holds 512 columns, a warpgroup's slot 3 Q of
@@ -122,6 +125,8 @@ struct Geo {
       ROLE == kSingle ? 1 : (1ll << (LOG2O + LOG2PRE));
   static constexpr long long OUT_VSTRIDE = ROLE == kSingle ? 0 : 1;
   static constexpr bool STRIDED = ROLE == kFirst || ROLE == kCols;
+  // the sub-transforms' prefix count q is a runtime value (PRun::q)
+  static constexpr bool RTQ = ROLE == kSecondQ;
   static constexpr int MODE_FIRST = STRIDED ? kUF : kQF;
   static constexpr int MODE_MID = kUF;
   static constexpr int MODE_LAST = ROLE == kSingle ? kRQF : kUF;
@@ -172,6 +177,8 @@ struct PRun {
   // process the items last to first: set on a pass that reads what the
   // previous pass wrote, whose latest output is still in L2
   int reverse;
+  // kSecondQ: the factor q of n = q R^S (sub-transforms per transform)
+  int q;
 };
 
 struct GArgs {
@@ -439,10 +446,12 @@ __device__ __forceinline__ void issue_input(const PRun &P, const CUtensorMap *tm
     const uint32_t bytes = (uint32_t)(rem << G::LOG2L) * 8u;
     const long long b = u0 >> G::LOG2UPER;
     const long long v = u0 & ((1ll << G::LOG2UPER) - 1);
-    const long long off = ((b & P.in_bmask) << G::LOG2N) + (v << G::LOG2L);
+    // with a runtime q the sub-transforms are simply consecutive
+    const long long off =
+        G::RTQ ? (u0 << G::LOG2L) : ((b & P.in_bmask) << G::LOG2N) + (v << G::LOG2L);
     const float2 *src = P.in + off;
     const long long in_elems =
-        P.in_bmask == -1 ? (P.U << G::LOG2L) : ((P.in_bmask + 1) << G::LOG2N);
+        (P.in_bmask == -1 || G::RTQ) ? (P.U << G::LOG2L) : ((P.in_bmask + 1) << G::LOG2N);
     const bool ok = in_range(w, off + (rem << G::LOG2L) - 1, in_elems);
     if (elect_one()) {
       // a skipped copy still completes the phase (no bytes expected)
@@ -591,14 +600,22 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, 
     klow = (klow << G::LOG2R) | (vq & (R - 1));
     vq >>= G::LOG2R;
   }
-  const long long b = u >> G::LOG2UPER;
-  const long long v = u & ((1ll << G::LOG2UPER) - 1);
+  long long b = u >> G::LOG2UPER;
+  long long v = u & ((1ll << G::LOG2UPER) - 1);
   // kFirst after a prefix: sequence b = (transform, p) -> transform-major,
   // k above p
   const long long bt = b >> G::LOG2PRE, bp = b & ((1ll << G::LOG2PRE) - 1);
   float2 *dst = P.out + ((bt & P.out_bmask) << G::LOG2NT) + (bp << G::LOG2UPER) +
                 v * G::OUT_VSTRIDE + klow * G::OUT_STRIDE;
-  constexpr long long JS = G::OUT_STRIDE << (G::LOG2L - G::LOG2R);
+  long long JS = G::OUT_STRIDE << (G::LOG2L - G::LOG2R);
+  if constexpr (G::RTQ) {
+    // transform b = u / q, row v = u mod q: y[b q L + v + k q]
+    const long long q = P.q;
+    b = u / q;
+    v = u - b * q;
+    dst = P.out + b * (q << G::LOG2L) + v + klow * q;
+    JS = q << (G::LOG2L - G::LOG2R);
+  }
   // twiddle of output k = klow + j r^(S-1): table A staged as [k][ul] in SMEM,
   // or read from global [k][vl]; two-level: times B[vh][k]
   const float2 *tws = w.tws + klow * G::GG + ul;

@@ -43,6 +43,7 @@ struct PassPlan {
   int q;
   RootsQ roots[2];
   bool mixed;
+  int qrt;          // kSecondQ: the factor q of n = q r^s (runtime prefix count)
   int tw;           // warpgroups per item (teams for the 3-stage radix-8 passes)
 };
 
@@ -75,7 +76,7 @@ bool prec_bf16(int precision);
 // are 8 rows x 16 bytes: 4 fp32 (TF32 modes) or 8 bf16 (BF16 modes) of K;
 // the four images sit at multiples of their size (16 r^2 or 8 r^2 bytes) in
 // a buffer of 64 r^2 bytes.
-void build_images(int r, int sign, int log2n, int precision, std::vector<float> &out);
+void build_images(int r, int sign, long long n, int precision, std::vector<float> &out);
 // Stage twiddles of a warpgroup pass: for t = 1 .. s-1 a block [j][lo],
 // j < r, lo < r^(s-t), holding w_L^{j * lo * r^(t-1)}.
 std::vector<float2> stage_twiddles(int r, int s, int sign);
@@ -182,12 +183,13 @@ namespace host {
 // passes have shorter sub-transforms, more adjacent columns per item and
 // wider TMA rows.  Returns the number of passes, 0 if n is too long.
 int plan_stages(int r, int k, int st[kMaxPasses]);
-// Mixed radix n = q r^k (q < r a power of two; the base case of the
-// recursion is a DFT of size q < sqrt(m)): a CUDA-core q-point first pass,
-// then the r^k-point transforms of its q rows in one or two tensor-core
-// passes (stage split as plan_stages).  Instantiated: k = 2..4 for r = 8
-// and 16, k = 2..3 for r = 32.  Returns the number of passes (0: not such
-// an n) and fills the passes.
+// Mixed radix n = q r^k (the base case of the recursion is a DFT of size
+// q): a CUDA-core q-point first pass, then the r^k-point transforms of its q
+// rows in tensor-core passes.  q < r a power of two: one or two passes
+// (stage split as plan_stages; k = 2..4 for r = 8 and 16, k = 2..3 for
+// r = 32).  Any other q = 2 .. 16 (odd factors): one pass with a runtime
+// q, k = 1..3 for r = 8, k = 1..2 for r = 16 and 32.  Returns the number of
+// passes (0: not such an n) and fills the passes.
 int plan_mixed(int r, long long n, long long batch, PassPlan pass[kMaxPasses]);
 // Warpgroups per item of pass pp: 4 for the 3-stage radix-8 passes of
 // two-pass transforms (an item of 512 rows holds 8 sub-transforms of 512

@@ -132,12 +132,15 @@ bool prec_bf16(int precision) { return precision == TCU_DFT_BF16 || precision ==
 // are 8 rows x 16 bytes: 4 fp32 (TF32 modes) or 8 bf16 (BF16 modes) of K;
 // the four images sit at multiples of their size (16 r^2 or 8 r^2 bytes) in
 // a buffer of 64 r^2 bytes.
-void build_images(int r, int sign, int log2n, int precision, std::vector<float> &out) {
+void build_images(int r, int sign, long long n, int precision, std::vector<float> &out) {
   const int K = 2 * r, N = 2 * r;
   const bool bf = prec_bf16(precision);
   const size_t lbo = 128, sbo = (bf ? 32 : 64) * (size_t)r, esz = bf ? 2 : 4;
   const size_t img_bytes = (bf ? 8 : 16) * (size_t)r * r;
-  const float sc = ldexpf(1.0f, -log2n);
+  // n a power of two: the scaled copies are hi, lo times 2^-log2 n (exact);
+  // otherwise hi and lo of the fp64 value F / n, rounded separately
+  const bool pow2 = (n & (n - 1)) == 0;
+  const float sc = pow2 ? ldexpf(1.0f, -ilog2(n)) : 0.f;
   out.assign((size_t)16 * r * r, 0.f);  // 64 r^2 bytes
   unsigned char *bytes = reinterpret_cast<unsigned char *>(out.data());
   for (int kr = 0; kr < K; ++kr) {
@@ -163,7 +166,10 @@ void build_images(int r, int sign, int log2n, int precision, std::vector<float> 
       } else {
         const float hi = host_tf32_rna((float)v);
         const float lo = host_tf32_rna((float)(v - (double)hi));
-        const float vals[4] = {hi, lo, hi * sc, lo * sc};
+        const double vs = v / (double)n;
+        const float his = pow2 ? hi * sc : host_tf32_rna((float)vs);
+        const float los = pow2 ? lo * sc : host_tf32_rna((float)(vs - (double)his));
+        const float vals[4] = {hi, lo, his, los};
         for (int i = 0; i < 4; ++i) memcpy(bytes + i * img_bytes + off, &vals[i], 4);
       }
     }

@@ -25,6 +25,9 @@ cudaError_t launch_pass_mixed_r16(int prec, int s, int lo, int role, int lp,
   TCU_PASS_CASE_L(2, 7, kSecond, 0)
   TCU_PASS_CASE_L(2, 8, kFirst, 3)
   TCU_PASS_CASE_L(2, 11, kSecond, 0)
+  // n = q 16^s with any q = 2 .. 16 (runtime q; one tensor-core pass)
+  TCU_PASS_CASE_L(1, 0, kSecondQ, 0)
+  TCU_PASS_CASE_L(2, 0, kSecondQ, 0)
   return cudaErrorInvalidValue;
 }
 

@@ -22,6 +22,9 @@ cudaError_t launch_pass_mixed_r32(int prec, int s, int lo, int role, int lp,
   TCU_PASS_CASE_L(2, 4, kSecond, 0)
   TCU_PASS_CASE_L(1, 10, kFirst, 4)
   TCU_PASS_CASE_L(2, 9, kSecond, 0)
+  // n = q 32^s with any q = 2 .. 16 (runtime q; one tensor-core pass)
+  TCU_PASS_CASE_L(1, 0, kSecondQ, 0)
+  TCU_PASS_CASE_L(2, 0, kSecondQ, 0)
   return cudaErrorInvalidValue;
 }
 

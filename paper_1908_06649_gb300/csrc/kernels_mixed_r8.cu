@@ -18,6 +18,10 @@ cudaError_t launch_pass_mixed_r8(int prec, int s, int lo, int role, int lp,
   TCU_PASS_CASE_L(3, 2, kSecond, 0)
   TCU_PASS_CASE_L(2, 6, kFirst, 2)
   TCU_PASS_CASE_L(2, 8, kSecond, 0)
+  // n = q 8^s with any q = 2 .. 16 (runtime q; one tensor-core pass)
+  TCU_PASS_CASE_L(1, 0, kSecondQ, 0)
+  TCU_PASS_CASE_L(2, 0, kSecondQ, 0)
+  TCU_PASS_CASE_L(3, 0, kSecondQ, 0)
   return cudaErrorInvalidValue;
 }
 

@@ -91,9 +91,54 @@ int plan_stages(int r, int k, int st[kMaxPasses]) {
 // passes (stage split as plan_stages).  Instantiated: k = 2..4 for r = 8
 // and 16, k = 2..3 for r = 32.  Returns the number of passes (0: not such
 // an n) and fills the passes.
+// n = q r^k with q = 2 .. 16 not a power of two: the q-point pass, then one
+// tensor-core pass over the q rows (role kSecondQ, q at run time).
+int plan_mixed_q(int r, long long n, long long batch, PassPlan pass[kMaxPasses]) {
+  const int log2r = ilog2(r);
+  const int kmax = r == 8 ? 3 : 2;
+  int k = 0;
+  long long rest = n;
+  while (rest % r == 0 && k < kmax) {
+    rest /= r;
+    ++k;
+  }
+  // the factor left must be a q the CUDA-core pass has, and r^k must hold
+  // all of n's powers of r that fit one pass
+  if (k < 1 || rest < 2 || rest > 16 || (rest & (rest - 1)) == 0) return 0;
+  if (rest % r == 0) return 0;
+  const int q = (int)rest;
+  PassPlan &p0 = pass[0];
+  p0.q = q;
+  p0.s = 1;
+  p0.role = kFirst;
+  p0.log2L = 0;  // not a power of two: the q-pass uses q itself
+  p0.lo = k * log2r;
+  p0.lp = 0;
+  p0.U = batch * (n / q);
+  for (int d = 0; d < 2; ++d)
+    for (int m = 0; m < 16; ++m) p0.roots[d].w[m] = root(m % q, q, d == 0 ? -1 : 1);
+  PassPlan &pp = pass[1];
+  pp.mixed = true;
+  pp.s = k;
+  pp.log2L = log2r * k;
+  pp.last = true;
+  pp.role = kSecondQ;
+  pp.lo = 0;
+  pp.lp = 0;
+  pp.qrt = q;
+  pp.U = batch * q;
+  pp.modes[0] = kQF;
+  pp.modes[1] = kUF;
+  pp.modes[2] = kUF;
+  pp.tw = 1;
+  pp.swz_tab = choose_swizzle(r, pp.s, pp.modes, 1);
+  return 2;
+}
+
 int plan_mixed(int r, long long n, long long batch, PassPlan pass[kMaxPasses]) {
   const int log2r = ilog2(r);
-  if (n < 1 || (n & (n - 1))) return 0;
+  if (n < 1) return 0;
+  if (n & (n - 1)) return plan_mixed_q(r, n, batch, pass);
   const int log2n = ilog2(n), k = log2n / log2r, lq = log2n - k * log2r;
   const int kmax = r == 32 ? 3 : 4;
   if (lq == 0 || k < 2 || k > kmax) return 0;
@@ -253,6 +298,7 @@ PRun group_pass(const tcu_dft_plan_s *p, int pi, int di, const float2 *in, float
   // pass before wrote last, still in L2 (measured 0.5-2.5 % per pass; not on
   // team passes, where it measured 1.5 % slower)
   g.reverse = (pi & 1) && pp.tw == 1;
+  g.q = pp.qrt;
   // the inverse's last stage uses the F images scaled by 1/n
   g.last_img = (pp.last && inverse) ? 2 * (prec_bf16(p->precision) ? 8 : 16) * p->r * p->r : 0;
   return g;
@@ -260,11 +306,13 @@ PRun group_pass(const tcu_dft_plan_s *p, int pi, int di, const float2 *in, float
 
 void dir_tables(const tcu_dft_plan_s *p, int d, DirTables &t) {
   const int sign = d == 0 ? -1 : 1;
-  build_images(p->r, sign, ilog2(p->n), p->precision, t.img);
+  build_images(p->r, sign, p->n, p->precision, t.img);
   for (int pi = 0; pi < p->npasses; ++pi) {
     const PassPlan &pp = p->pass[pi];
     t.stage[pi] = stage_twiddles(p->r, pp.q ? 1 : pp.s, sign);
-    if (pp.role == kFirst) pass_twiddles(1ll << pp.log2L, 1ll << pp.lo, sign, t.A[pi], t.B[pi]);
+    // the q-point pass has L = q rows (any q); a tensor-core pass L = r^s
+    if (pp.role == kFirst)
+      pass_twiddles(pp.q ? pp.q : (1ll << pp.log2L), 1ll << pp.lo, sign, t.A[pi], t.B[pi]);
   }
 }
 

@@ -61,7 +61,8 @@ int main(void) {
   int32_t st[3] = {0, 0, 0};
   int64_t N = 0, B = 0;
   if (tcu_dft_plan_passes(65536, 16, st) != 2 || st[0] != 2 || st[1] != 2) return 1;
-  if (tcu_dft_plan_passes(48, 16, st) != 0) return 2;
+  if (tcu_dft_plan_passes(272, 16, st) != 0) return 2;             /* 17 * 16 */
+  if (tcu_dft_plan_passes(48, 16, st) != 2 || st[0] != 1 || st[1] != 1) return 8;  /* 3 * 16 */
   if (tcu_stencil_tiles(4096, 16, 16, &N, &B) != 361 || N != 256 || B != 224) return 3;
   if (strcmp(tcu_dft_strerror(TCU_DFT_OK), "ok") != 0) return 4;
   if (tcu_dft_destroy(NULL) != TCU_DFT_OK) return 5;
@@ -127,11 +128,14 @@ def test_strerror_and_null_handling(lib):
     (512, 1, 16, 5, 2),      # BF16 modes: no mixed radix
     (16, 1, 4, 3, 2),        # radix not in {8, 16, 32}
     (16, 1, 64, 3, 2),
-    (48, 1, 16, 3, 2),       # not a power of the radix
+    (17 * 16, 1, 16, 3, 2),  # a factor beyond 16
     (128, 1, 16, 3, 2),      # power of two but not of 16
     (2 * 16, 1, 16, 3, 2),   # mixed radix with one radix-16 stage (k < 2)
     (2 * 16 ** 5, 1, 16, 3, 2),  # mixed radix beyond k = 4
-    (3 * 256, 1, 16, 3, 2),  # a factor that is not a power of two
+    (3 * 16 ** 3, 1, 16, 3, 2),  # an odd factor with more than one tensor pass
+    (5 * 32 ** 3, 1, 32, 3, 2),
+    (3 * 8 ** 4, 1, 8, 3, 2),
+    (48, 1, 16, 4, 2),       # BF16 modes: no mixed radix (3 x 16)
     (16 ** 7, 1, 16, 3, 2),  # beyond three passes
     (32 ** 7, 1, 32, 3, 2),
     (8 ** 10, 1, 8, 3, 2),
@@ -150,10 +154,24 @@ def test_plan_without_gpu_reports_cuda_error(lib):
     assert lib.tcu_dft_last_error() == 3
 
 
+@pytest.mark.parametrize("r,kmax", [(8, 3), (16, 2), (32, 2)])
+def test_pass_grouping_odd_factors(lib, r, kmax):
+    """n = q r^k with q = 2 .. 16 not a power of two: the q-point pass, then
+    one tensor-core pass of k stages (k up to one warpgroup pass)."""
+    import ctypes
+    st = (ctypes.c_int32 * 3)()
+    for q in (3, 5, 6, 7, 9, 10, 11, 12, 13, 14, 15):
+        for k in range(1, kmax + 1):
+            assert lib.tcu_dft_plan_passes(q * r ** k, r, st) == 2, (q, k)
+            assert list(st)[:2] == [1, k]
+        assert lib.tcu_dft_plan_passes(q * r ** (kmax + 1), r, st) == 0
+    assert lib.tcu_dft_plan_passes(17 * r, r, st) == 0
+
+
 def test_python_plan_raises(lib):
     import paper_1908_06649_gb300 as pkg
     with pytest.raises(pkg.TcuDftError) as e:
-        pkg.Plan(48, 1, 16)
+        pkg.Plan(17 * 16, 1, 16)
     assert e.value.status == pkg.ERR_UNSUPPORTED
 
 
@@ -265,7 +283,8 @@ def test_grid_null_handling(lib):
     (2 * 256, 16, [1, 2]), (8 * 4096, 16, [1, 1, 2]), (4 * 65536, 16, [1, 2, 2]),
     (2 * 64, 8, [1, 2]), (4 * 512, 8, [1, 3]), (2 * 4096, 8, [1, 2, 2]),
     (16 * 1024, 32, [1, 2]), (2 * 32 ** 3, 32, [1, 1, 2]),
-    (2 * 16, 16, []), (3 * 256, 16, []), (2 * 16 ** 5, 16, []), (0, 16, [])])
+    (2 * 16, 16, []), (3 * 256, 16, [1, 2]), (3 * 16 ** 3, 16, []), (2 * 16 ** 5, 16, []),
+    (0, 16, [])])
 def test_plan_grouping(n, r, stages):
     # the documented grouping, computed on the host without a GPU
     import paper_1908_06649_gb300 as pkg

@@ -462,6 +462,47 @@ def test_mixed_radix(pkg, r, q, k, prec):
     check(yi, x, prec, inverse=True)
 
 
+# ---- mixed radix with any factor q = 2 .. 16 (odd factors included): the
+# q-point pass on CUDA cores, then one tensor-core pass whose output stride
+# is q; forward and inverse (1/n with n not a power of two) against the
+# oracle's direct definition
+@pytest.mark.parametrize("r,q,k", [(8, 3, 3), (8, 5, 2), (8, 6, 3), (8, 12, 2), (8, 7, 1),
+                                   (16, 3, 2), (16, 5, 2), (16, 6, 2), (16, 12, 2),
+                                   (16, 15, 1), (16, 9, 2),
+                                   (32, 3, 2), (32, 5, 1), (32, 6, 2), (32, 12, 2)])
+@pytest.mark.parametrize("inverse", [False, True])
+def test_mixed_radix_odd_factors(pkg, r, q, k, inverse):
+    n = q * r ** k
+    batch = 5  # ragged: not a multiple of an item's sub-transforms
+    x = inputs.make("normal", n, batch, seed=1000 + n)
+    y, passes = run(pkg, x, r, 3, inverse=inverse)
+    assert passes == [1, k]
+    check(y, x, 3, inverse=inverse)
+
+
+@pytest.mark.parametrize("r,q,k", [(16, 3, 2), (8, 10, 3), (32, 7, 2)])
+def test_mixed_radix_odd_factors_tf32_and_tones(pkg, r, q, k):
+    n = q * r ** k
+    x = inputs.make("uniform", n, 3, seed=77)
+    y, _ = run(pkg, x, r, 1)
+    check(y, x, 1)
+    # a pure tone at frequency f -> n at f, zero elsewhere (3xTF32)
+    f = (n // 3) + 1
+    j = np.arange(n)
+    tone = np.exp(2j * np.pi * ((f * j) % n) / n).astype(np.complex64)[None, :]
+    yt, _ = run(pkg, np.repeat(tone, 2, axis=0), r, 3)
+    ef = np.zeros(n)
+    ef[f] = n
+    assert np.max(np.abs(yt - ef)) < 1e-5 * n
+
+
+def test_mixed_radix_odd_factor_in_place(pkg):
+    n, batch = 5 * 16 ** 2, 9
+    x = inputs.make("normal", n, batch, seed=5)
+    y, _ = run(pkg, x, 16, 3, inplace=True)
+    check(y, x, 3)
+
+
 def test_mixed_radix_in_place(pkg):
     n = 8 * 16 ** 4
     x = inputs.make("uniform", n, 3, seed=8)
