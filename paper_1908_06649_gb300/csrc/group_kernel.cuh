@@ -228,7 +228,8 @@ struct SmemLayout {
   static constexpr size_t TWB_PER_WG = TWB;               // per team
   static constexpr size_t TWB_BYTES = (size_t)NTEAM * TWB * 8;
   static constexpr size_t OFF_BAR = OFF_TWB + TWB_BYTES;
-  static constexpr size_t OFF_SCHED = OFF_BAR + 8 * 3 * NWG + 8;
+  // 3 mbarriers per warpgroup, the TMEM slot word, the tables' mbarrier
+  static constexpr size_t OFF_SCHED = OFF_BAR + 8 * 3 * NWG + 16;
   static constexpr size_t BYTES = OFF_SCHED + 32 * NWG;
   static_assert(BYTES <= 227 * 1024, "shared memory budget");
 };
@@ -1000,7 +1001,12 @@ __device__ __forceinline__ void process_item_conv(const PRun &P, const float2 *t
   last_stage_store<G, PREC, false, false>(P, item, w);
 }
 
-// Common set-up: F images and stage twiddles into SMEM, mbarriers, TMEM.
+// Common set-up: mbarriers, TMEM, and the F images and stage twiddles into
+// SMEM by asynchronous bulk copies (issued by one thread, completing on the
+// tables' mbarrier, the word after the TMEM slot) so that they overlap the
+// first item's input copy; wait_tables() before the first use.  Every size
+// is a multiple of 16 bytes (the images 64 r^2 bytes, the twiddle tables an
+// even number of complex values).
 template <int NWG, int THREADS>
 __device__ __forceinline__ uint32_t kernel_setup(const float *bimg, int img_floats,
                                                  float *img, const float2 *tw_src0,
@@ -1009,23 +1015,28 @@ __device__ __forceinline__ uint32_t kernel_setup(const float *bimg, int img_floa
                                                  int tw_n1, uint64_t *mbar,
                                                  uint32_t *tmem_slot) {
   const int tid = threadIdx.x;
-  {
-    const float4 *src = reinterpret_cast<const float4 *>(bimg);
-    float4 *dst = reinterpret_cast<float4 *>(img);
-    for (int i = tid; i < img_floats / 4; i += THREADS) dst[i] = __ldg(src + i);
-    for (int i = tid; i < tw_n0; i += THREADS) tw_dst0[i] = __ldg(tw_src0 + i);
-    for (int i = tid; i < tw_n1; i += THREADS) tw_dst1[i] = __ldg(tw_src1 + i);
-  }
+  uint64_t *tbar = mbar + 3 * NWG + 1;
   if (tid == 0) {
     for (int w = 0; w < 3 * NWG; ++w) mbar_init(smem_u32(mbar + w), 1);
+    mbar_init(smem_u32(tbar), 1);
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    const uint32_t bytes0 = (uint32_t)img_floats * 4u, bytes1 = (uint32_t)tw_n0 * 8u,
+                   bytes2 = (uint32_t)tw_n1 * 8u;
+    mbar_expect_tx(smem_u32(tbar), bytes0 + bytes1 + bytes2);
+    tma_load_1d(smem_u32(img), bimg, bytes0, smem_u32(tbar));
+    if (bytes1) tma_load_1d(smem_u32(tw_dst0), tw_src0, bytes1, smem_u32(tbar));
+    if (bytes2) tma_load_1d(smem_u32(tw_dst1), tw_src1, bytes2, smem_u32(tbar));
   }
-  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
   if ((tid >> 5) == 0) tmem_alloc(smem_u32(tmem_slot), 512);
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
   return *tmem_slot;
+}
+
+// Every thread, before the first use of the F images or stage twiddles.
+__device__ __forceinline__ bool wait_tables(uint64_t *mbar, int nwg) {
+  return mbar_wait_bounded(smem_u32(mbar + 3 * nwg + 1), 0);
 }
 
 // Leave: wait (bounded) for any copy still landing in this warpgroup's
@@ -1116,12 +1127,15 @@ __global__ void __launch_bounds__(
   const int team = (threadIdx.x >> 7) / TW;
   const long long nitems = (P.U + G::GG - 1) >> G::LOG2GG;
   const long long istride = (long long)gridDim.x * G::NTEAM;
-  long long item = (long long)blockIdx.x * G::NTEAM + team;
+  // team-major: with fewer items than SMs each CTA holds one item
+  long long item = (long long)team * gridDim.x + blockIdx.x;
   StaticNext<G> nx{P, &a.tm_in, item, nitems, false};
   // item: position in this CTA's sequence; phys: the item processed there
   // (team passes always run forward: no reversal code in them)
   auto phys = [&](long long i) { return TW == 1 && P.reverse ? nitems - 1 - i : i; };
   if (w.team_lead && item < nitems) issue_input<G>(P, &a.tm_in, phys(item), w);
+  // the tables have landed (the same answer in every thread of the team)
+  if (named_bar_or(w.bar_id, w.bar_count, !wait_tables(mbar, G::NWG))) w.fail = true;
   while (item < nitems && !w.fail) {
     nx.next = item + istride;
     if constexpr (CONV)
@@ -1372,6 +1386,7 @@ __global__ void __launch_bounds__(
     nx.n1 = nx.decode(__shfl_sync(0xffffffffu, nx.claim(), 0));
     nx.read_dep(nx.n1);
   }
+  if (!wait_tables(mbar, NWG)) f = true;
   if (named_bar_or(w.bar_id, w.bar_count, f)) w.fail = true;
 
   bool stg_pending = false;
@@ -1817,6 +1832,9 @@ __global__ void __launch_bounds__(
   nx.pol_last = l2_policy_evict_last();
   nx.issued = nx.cur.valid && nx.cur.type == 0;
   if (nx.issued && w.team_lead) nx.copy(nx.cur, w);
+  if (!wait_tables(mbar, NWG)) w.fail = true;
+  // a uniform failure state before the first barrier
+  if (named_bar_or(w.bar_id, w.bar_count, w.fail)) w.fail = true;
   bool stg_pending = nx.issued;
   while (nx.cur.valid && !w.fail) {
     nx.nxt = pair_decode(pos + NWG, H, J);

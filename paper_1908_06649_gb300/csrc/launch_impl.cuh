@@ -16,9 +16,10 @@ cudaError_t launch_pass_t(const GArgs &a, int num_sms, cudaStream_t st) {
                                        cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        (int)sm);
   if (e != cudaSuccess) return e;
+  // one CTA per SM, each item on its own SM while there are fewer items
+  // than SMs (latency), several per SM otherwise
   const long long nitems = (a.p[0].U + G::GG - 1) >> G::LOG2GG;
-  long long grid = (nitems + G::NWG - 1) / G::NWG;
-  if (grid > num_sms) grid = num_sms;
+  long long grid = nitems < num_sms ? nitems : num_sms;
   dft_pass_kernel<R, PREC, S, LO, ROLE, LP><<<(unsigned)grid, G::THREADS, sm, st>>>(a);
   return cudaGetLastError();
 }
@@ -33,8 +34,7 @@ cudaError_t launch_team_t(const GArgs &a, int num_sms, cudaStream_t st) {
                                        (int)sm);
   if (e != cudaSuccess) return e;
   const long long nitems = (a.p[0].U + G::GG - 1) >> G::LOG2GG;
-  long long grid = (nitems + G::NTEAM - 1) / G::NTEAM;
-  if (grid > num_sms) grid = num_sms;
+  long long grid = nitems < num_sms ? nitems : num_sms;
   dft_pass_kernel<R, PREC, S, LO, ROLE, LP, false, TW>
       <<<(unsigned)grid, G::THREADS, sm, st>>>(a);
   return cudaGetLastError();
@@ -58,8 +58,7 @@ cudaError_t launch_rowconv_t(const GArgs &a, int num_sms, cudaStream_t st) {
                                        (int)sm);
   if (e != cudaSuccess) return e;
   const long long nitems = (a.p[0].U + G::GG - 1) >> G::LOG2GG;
-  long long grid = (nitems + G::NWG - 1) / G::NWG;
-  if (grid > num_sms) grid = num_sms;
+  long long grid = nitems < num_sms ? nitems : num_sms;
   dft_pass_kernel<R, PREC, S, 0, kSingle, 0, true><<<(unsigned)grid, G::THREADS, sm, st>>>(a);
   return cudaGetLastError();
 }
