@@ -121,6 +121,45 @@ __global__ void extract_tiles_kernel(float *Ak, const float2 *tiles, long long s
       Ak[(r0 + i) * side + c0 + j] = __ldcs(src + (long long)i * N + j).x;
 }
 
+// out[b][j][i] = in[b][i][j] for n1 x n2 arrays: 32 x 32 tiles through
+// shared memory (a column of 33 for conflict-free reads of the transposed
+// tile), blocks of 32 x 8 threads; both the read of `in` and the write of
+// `out` run along contiguous rows of 32 complex values.  The grid walks
+// every (array, tile) pair.
+constexpr int kTile = 32;
+
+__global__ void transpose_kernel(float2 *out, const float2 *in, long long batch, long long n1,
+                                 long long n2) {
+  __shared__ float2 t[kTile][kTile + 1];
+  const long long ti = (n1 + kTile - 1) / kTile, tj = (n2 + kTile - 1) / kTile;
+  const long long total = batch * ti * tj;
+  for (long long tile = blockIdx.x; tile < total; tile += gridDim.x) {
+    const long long b = tile / (ti * tj), rem = tile % (ti * tj);
+    const long long i0 = (rem / tj) * kTile, j0 = (rem % tj) * kTile;
+    const float2 *src = in + b * n1 * n2;
+    float2 *dst = out + b * n1 * n2;
+    for (int y = threadIdx.y; y < kTile; y += blockDim.y) {
+      const long long i = i0 + y, j = j0 + threadIdx.x;
+      if (i < n1 && j < n2) t[y][threadIdx.x] = __ldcs(src + i * n2 + j);
+    }
+    __syncthreads();
+    for (int y = threadIdx.y; y < kTile; y += blockDim.y) {
+      const long long j = j0 + y, i = i0 + threadIdx.x;
+      if (i < n1 && j < n2) __stcs(dst + j * n1 + i, t[threadIdx.x][y]);
+    }
+    __syncthreads();
+  }
+}
+
+// x[b][e] *= spec[e] for every array b of n complex values.
+__global__ void spectrum_product_kernel(float2 *x, const float2 *spec, long long batch,
+                                        long long n) {
+  const long long count = batch * n;
+  for (long long e = blockIdx.x * (long long)blockDim.x + threadIdx.x; e < count;
+       e += (long long)gridDim.x * blockDim.x)
+    x[e] = cmul(x[e], __ldg(spec + e % n));
+}
+
 unsigned grid_for(long long count, int num_sms) {
   long long blocks = (count + kBlock - 1) / kBlock;
   const long long cap = (long long)num_sms * 8;  // 8 resident 256-thread blocks per SM
@@ -151,6 +190,21 @@ cudaError_t launch_extract_weights(float *W, const float2 *g, long long Nw, int 
 cudaError_t launch_place_kernel(float2 *w, long long N, const float2 *g, long long Nw, int k,
                                 int num_sms, cudaStream_t st) {
   place_kernel_kernel<<<grid_for(N * N, num_sms), kBlock, 0, st>>>(w, N, g, Nw, k);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_transpose(float2 *out, const float2 *in, long long batch, long long n1,
+                             long long n2, int num_sms, cudaStream_t st) {
+  const long long tiles = batch * ((n1 + kTile - 1) / kTile) * ((n2 + kTile - 1) / kTile);
+  const long long cap = (long long)num_sms * 8;
+  const unsigned grid = (unsigned)(tiles < cap ? tiles : cap);
+  transpose_kernel<<<grid, dim3(kTile, 8), 0, st>>>(out, in, batch, n1, n2);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_spectrum_product(float2 *x, const float2 *spec, long long batch,
+                                    long long n, int num_sms, cudaStream_t st) {
+  spectrum_product_kernel<<<grid_for(batch * n, num_sms), kBlock, 0, st>>>(x, spec, batch, n);
   return cudaGetLastError();
 }
 

@@ -27,6 +27,13 @@ using namespace tcu::host;
 // inverse columns (1/(n1 n2) folded into the last stage's F images).
 
 
+// Axes beyond one warpgroup pass (or the BF16 modes): the general path.
+// The rows of every array are one batched 1-D plan of length n2 (several
+// passes where needed); the arrays are transposed so that the columns are
+// contiguous, transformed by a 1-D plan of length n1 and transposed back.
+// A convolution multiplies by the spectrum on the transposed layout (the
+// spectrum transposed once per call into a plan buffer) between the forward
+// and the inverse column plans.
 struct tcu_dft2_plan_s {
   long long n1, n2, batch;
   int r, precision, num_sms;
@@ -35,6 +42,9 @@ struct tcu_dft2_plan_s {
   float *cimg;        // convolution rows: forward hi, lo | inverse hi, lo
   float2 *scratch;    // batch * n1 * n2
   int *err;
+  bool general;
+  tcu_dft_plan_t rows1d, cols1d;  // general path: length n2 / n1 plans
+  float2 *spec_t;                 // general path: the spectrum transposed
 };
 
 struct tcu_stencil_plan_s {
@@ -67,6 +77,9 @@ int single_pass_stages(int r) { return r == 8 ? 3 : 2; }
 
 void free_dft2(tcu_dft2_plan_s *p) {
   if (!p) return;
+  tcu_dft_destroy(p->rows1d);
+  tcu_dft_destroy(p->cols1d);
+  cudaFree(p->spec_t);
   for (int d = 0; d < 2; ++d) {
     cudaFree(p->bimg[d]);
     cudaFree(p->cols.tw_stage[d]);
@@ -122,6 +135,67 @@ int check_buffers(const void *in, const void *out, size_t bytes) {
   return TCU_DFT_OK;
 }
 
+// The general path: 1-D plans for the rows (n2, batch n1 of them) and the
+// columns (n1, batch n2 of them), a scratch array and the transposed
+// spectrum of a convolution.  UNSUPPORTED if either length has no 1-D plan.
+tcu_dft2_plan_s *make_dft2_general(int64_t n1, int64_t n2, int64_t batch, int32_t r,
+                                   int32_t precision, int &rc) {
+  // both lengths must have a 1-D plan (a host-side question: no CUDA call)
+  int32_t st[kMaxPasses];
+  if (tcu_dft_plan_passes(n1, r, st) == 0 || tcu_dft_plan_passes(n2, r, st) == 0) {
+    rc = TCU_DFT_ERR_UNSUPPORTED;
+    return nullptr;
+  }
+  tcu_dft2_plan_s *p = new tcu_dft2_plan_s();
+  memset(p, 0, sizeof(*p));
+  p->n1 = n1;
+  p->n2 = n2;
+  p->batch = batch;
+  p->r = r;
+  p->precision = precision;
+  p->general = true;
+  p->rows1d = tcu_dft_plan(n2, batch * n1, r, precision);
+  rc = p->rows1d ? TCU_DFT_OK : tcu_dft_last_error();
+  if (rc == TCU_DFT_OK) {
+    p->cols1d = tcu_dft_plan(n1, batch * n2, r, precision);
+    rc = p->cols1d ? TCU_DFT_OK : tcu_dft_last_error();
+  }
+  if (rc == TCU_DFT_OK) {
+    p->num_sms = p->rows1d->num_sms;
+    if (dev_malloc((void **)&p->scratch, (size_t)(batch * n1 * n2) * sizeof(float2)) !=
+            cudaSuccess ||
+        dev_malloc((void **)&p->spec_t, (size_t)(n1 * n2) * sizeof(float2)) != cudaSuccess ||
+        dev_malloc((void **)&p->err, sizeof(int)) != cudaSuccess ||
+        cudaMemset(p->err, 0, sizeof(int)) != cudaSuccess) {
+      cudaGetLastError();
+      rc = TCU_DFT_ERR_OOM;
+    }
+  }
+  if (rc != TCU_DFT_OK) {
+    free_dft2(p);
+    return nullptr;
+  }
+  return p;
+}
+
+// General path: the 2-D transform of `in` into `out` (rows, transpose,
+// columns, transpose back), or -- with keep_t -- left transposed in the
+// plan's scratch after the columns (the convolution continues there).
+int general_dft2(const tcu_dft2_plan_s *p, const void *in, void *out, int dir, bool keep_t,
+                 cudaStream_t st) {
+  int rc = tcu_dft_exec_dir(p->rows1d, in, out, dir, st);
+  if (rc != TCU_DFT_OK) return rc;
+  if (launch_transpose(p->scratch, (const float2 *)out, p->batch, p->n1, p->n2, p->num_sms,
+                       st) != cudaSuccess)
+    return TCU_DFT_ERR_CUDA;
+  rc = tcu_dft_exec_dir(p->cols1d, p->scratch, p->scratch, dir, st);
+  if (rc != TCU_DFT_OK || keep_t) return rc;
+  return launch_transpose((float2 *)out, p->scratch, p->batch, p->n2, p->n1, p->num_sms, st) ==
+                 cudaSuccess
+             ? TCU_DFT_OK
+             : TCU_DFT_ERR_CUDA;
+}
+
 tcu_dft2_plan_s *make_dft2(int64_t n1, int64_t n2, int64_t batch, int32_t r,
                            int32_t precision, int &rc) {
   rc = TCU_DFT_OK;
@@ -130,18 +204,17 @@ tcu_dft2_plan_s *make_dft2(int64_t n1, int64_t n2, int64_t batch, int32_t r,
     rc = TCU_DFT_ERR_INVALID;
     return nullptr;
   }
-  if (prec_bf16(precision)) {  // the 2-D passes are instantiated for the TF32 modes
-    rc = TCU_DFT_ERR_UNSUPPORTED;
-    return nullptr;
-  }
   int k1 = 0, k2 = 0;
   if ((r != 8 && r != 16 && r != 32) || !is_power_of(n1, r, k1) || !is_power_of(n2, r, k2) ||
-      k1 > single_pass_stages(r) || k2 > single_pass_stages(r) ||
-      n1 * n2 < 128ll * r || batch * n1 * n2 > (1ll << 40)) {
-    // each axis one warpgroup pass; a column item spans 128 r / n1 columns
+      batch * n1 * n2 > (1ll << 40)) {
     rc = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
   }
+  // each axis one warpgroup pass (a column item spans 128 r / n1 columns),
+  // TF32 modes: the two-pass path; otherwise the general path
+  if (prec_bf16(precision) || k1 > single_pass_stages(r) || k2 > single_pass_stages(r) ||
+      n1 * n2 < 128ll * r)
+    return make_dft2_general(n1, n2, batch, r, precision, rc);
   int dev = 0;
   cudaDeviceProp prop;
   if (cudaGetDevice(&dev) != cudaSuccess || cudaGetDeviceProperties(&prop, dev) != cudaSuccess ||
@@ -220,10 +293,10 @@ void free_stencil(tcu_stencil_plan_s *p) {
 }
 
 // Smallest power of r, at least `need`, whose square holds a column item
-// (128 r points) and that one warpgroup pass transforms; 0 if none.
+// (128 r points): one warpgroup pass per axis where that suffices, else the
+// general path up to 2^26 points per grid (8192^2); 0 if none.
 long long grid_side(int r, long long need) {
-  long long N = r;
-  for (int s = 1; s <= single_pass_stages(r); ++s, N *= r)
+  for (long long N = r; N * N <= (1ll << 26); N *= r)
     if (N >= need && N * N >= 128ll * r) return N;
   return 0;
 }
@@ -269,6 +342,11 @@ int tcu_dft2_exec(tcu_dft2_plan_t p, const void *in, void *out, int dir, void *s
   if (rc != TCU_DFT_OK) return rc;
   cudaStream_t st = (cudaStream_t)stream;
   const int di = dir_index(dir);
+  if (p->general) {
+    const NvtxRange range("tcu_dft2 (general)");
+    rc = general_dft2(p, in, out, dir, false, st);
+    return rc == TCU_DFT_OK && debug_exec() ? tcu_dft2_check(p, stream) : rc;
+  }
   {
     const NvtxRange range("tcu_dft2");
     rc = run_dft2_pass(p, p->cols, di, (const float2 *)in, p->scratch, false, nullptr, st);
@@ -287,6 +365,24 @@ int tcu_conv2_exec(tcu_dft2_plan_t p, const void *in, const void *spectrum, void
   if (rc != TCU_DFT_OK) return rc;
   cudaStream_t st = (cudaStream_t)stream;
   const NvtxRange range("tcu_conv2");
+  if (p->general) {
+    // forward rows and columns (left transposed in the scratch), times the
+    // spectrum transposed, inverse columns, transpose back, inverse rows
+    rc = general_dft2(p, in, out, TCU_DFT_FORWARD, true, st);
+    if (rc != TCU_DFT_OK) return rc;
+    if (launch_transpose(p->spec_t, (const float2 *)spectrum, 1, p->n1, p->n2, p->num_sms,
+                         st) != cudaSuccess ||
+        launch_spectrum_product(p->scratch, p->spec_t, p->batch, p->n1 * p->n2, p->num_sms,
+                                st) != cudaSuccess)
+      return TCU_DFT_ERR_CUDA;
+    rc = tcu_dft_exec_dir(p->cols1d, p->scratch, p->scratch, TCU_DFT_INVERSE, st);
+    if (rc != TCU_DFT_OK) return rc;
+    if (launch_transpose((float2 *)out, p->scratch, p->batch, p->n2, p->n1, p->num_sms, st) !=
+        cudaSuccess)
+      return TCU_DFT_ERR_CUDA;
+    rc = tcu_dft_exec_dir(p->rows1d, out, out, TCU_DFT_INVERSE, st);
+    return rc == TCU_DFT_OK && debug_exec() ? tcu_dft2_check(p, stream) : rc;
+  }
   // columns: in -> scratch; rows forward, times the spectrum and inverse on
   // chip: scratch -> scratch (an item reads its rows before writing them);
   // inverse columns with 1/(n1 n2): scratch -> out
@@ -309,6 +405,11 @@ int tcu_conv2_exec(tcu_dft2_plan_t p, const void *in, const void *spectrum, void
 
 int tcu_dft2_check(tcu_dft2_plan_t p, void *stream) {
   if (!p) return TCU_DFT_ERR_INVALID;
+  if (p->general) {
+    int rc = tcu_dft_check(p->rows1d, stream);
+    if (rc == TCU_DFT_OK) rc = tcu_dft_check(p->cols1d, stream);
+    if (rc != TCU_DFT_OK) return rc;
+  }
   if (cudaStreamSynchronize((cudaStream_t)stream) != cudaSuccess) return TCU_DFT_ERR_CUDA;
   int flag = 0;
   if (cudaMemcpy(&flag, p->err, sizeof(int), cudaMemcpyDeviceToHost) != cudaSuccess)
@@ -329,10 +430,6 @@ tcu_stencil_plan_t tcu_stencil_plan(int64_t side, int32_t steps, int32_t sqrt_m,
   if (side < 1 || steps < 1 ||
       (precision != TCU_DFT_TF32 && precision != TCU_DFT_3XTF32 && !prec_bf16(precision))) {
     g_last_error = TCU_DFT_ERR_INVALID;
-    return nullptr;
-  }
-  if (prec_bf16(precision)) {
-    g_last_error = TCU_DFT_ERR_UNSUPPORTED;
     return nullptr;
   }
   const long long N =

@@ -56,6 +56,14 @@ cudaError_t launch_gather_tiles(float2 *tiles, const float *A, long long side, i
 cudaError_t launch_extract_tiles(float *Ak, const float2 *tiles, long long side, int k,
                                  long long N, int B, int num_sms, cudaStream_t st);
 
+// 2-D transforms whose axes need several passes (grid_kernels.cu): the
+// transpose of every n1 x n2 array of a batch (out[b][j][i] = in[b][i][j]),
+// and the pointwise product of every array with one spectrum.
+cudaError_t launch_transpose(float2 *out, const float2 *in, long long batch, long long n1,
+                             long long n2, int num_sms, cudaStream_t st);
+cudaError_t launch_spectrum_product(float2 *x, const float2 *spec, long long batch,
+                                    long long n, int num_sms, cudaStream_t st);
+
 // The q-point first pass of a mixed-radix transform (grid_kernels.cu).
 struct RootsQ {
   float2 w[16];  // w_q^m, m < q, of the direction

@@ -216,8 +216,7 @@ def test_noalloc_null_buffers(lib):
     ((0, 256, 1, 16, 3), 1),        # n1 < 1
     ((16, 256, 0, 16, 3), 1),       # batch < 1
     ((16, 256, 1, 16, 2), 1),       # precision
-    ((16, 16, 1, 16, 3), 2),        # n1 n2 below one column item (128 r)
-    ((4096, 16, 1, 16, 3), 2),      # an axis beyond one warpgroup pass
+    ((16 ** 7, 16, 1, 16, 3), 2),   # an axis beyond the 1-D plans (three passes)
     ((48, 256, 1, 16, 3), 2),       # not a power of the radix
     ((16, 256, 1, 12, 3), 2),       # radix
 ])
@@ -229,8 +228,7 @@ def test_dft2_plan_rejects_before_cuda(lib, args, status):
 @pytest.mark.parametrize("args,status", [
     ((0, 4, 8, 3), 1),              # side
     ((64, 0, 8, 3), 1),             # steps
-    ((64, 4, 8, 4), 2),             # BF16 modes: no 2-D plans
-    ((1024, 200, 8, 3), 2),         # 3k beyond one pass (8^3)
+    ((1024, 3000, 8, 3), 2),        # 3k beyond the largest tile (8192^2 points)
     ((64, 4, 12, 3), 2),            # radix
 ])
 def test_stencil_plan_rejects_before_cuda(lib, args, status):
@@ -240,15 +238,16 @@ def test_stencil_plan_rejects_before_cuda(lib, args, status):
 
 def test_stencil_tiling_choice(lib):
     """tcu_stencil_tiles: the smallest tile side N = r^s with N >= 3k and
-    N^2 >= 128 r within one pass per axis, blocks of B = N - 2k, ceil(side /
+    N^2 >= 128 r, at most 2^26 points a tile (one pass per axis where that
+    holds them, the general 2-D path above), blocks of B = N - 2k, ceil(side /
     B)^2 tiles -- checked against the rule evaluated here."""
     import paper_1908_06649_gb300 as pkg
     for side, k, r in [(4096, 16, 8), (4096, 16, 16), (4096, 16, 32), (64, 4, 8),
                        (2000, 16, 8), (300, 16, 16), (120, 20, 8), (1, 1, 16),
-                       (5000, 85, 16), (777, 3, 32), (100, 30, 8)]:
-        smax = 3 if r == 8 else 2
-        Ns = [r ** s for s in range(1, smax + 1)
-              if r ** s >= 3 * k and r ** (2 * s) >= 128 * r]
+                       (5000, 85, 16), (777, 3, 32), (100, 30, 8), (300, 128, 16),
+                       (5000, 200, 8), (2000, 400, 32), (100, 3000, 16)]:
+        Ns = [r ** s for s in range(1, 9)
+              if r ** s >= 3 * k and r ** (2 * s) >= 128 * r and r ** (2 * s) <= 1 << 26]
         got = pkg.stencil_tiles(side, k, r)
         if not Ns:
             assert got == (0, 0, 0)

@@ -54,6 +54,71 @@ def test_dft2(pkg, r, n1, n2, batch, prec):
     plan.destroy()
 
 
+# ---- the general 2-D path: axes beyond one warpgroup pass (1-D plans for
+# the rows and, after a transpose, the columns), arrays below one column item,
+# and the BF16 modes
+@pytest.mark.parametrize("r,n1,n2,batch", [
+    (16, 4096, 4096, 1), (16, 65536, 16, 2), (16, 16, 65536, 2), (16, 16, 16, 3),
+    (8, 4096, 512, 1), (8, 8, 8, 5), (32, 32768, 32, 1), (32, 32, 32768, 1)])
+def test_dft2_general(pkg, r, n1, n2, batch):
+    import torch
+    x = inputs.make("normal", n1 * n2, batch, seed=n1 + 3 * n2).reshape(batch, n1, n2)
+    plan = pkg.Plan2(n1, n2, batch, r, 3)
+    xd = torch.from_numpy(x).cuda().reshape(-1)
+    y = plan.forward(xd)
+    plan.check()
+    yh = y.cpu().numpy().reshape(batch, n1, n2)
+    assert _rel(yh, grid.dft2(x, threads=8)).max() <= TOL[3]
+    back = plan.inverse(y)
+    plan.check()
+    bh = back.cpu().numpy().reshape(batch, n1, n2)
+    assert _rel(bh, x).max() <= 2 * TOL[3]
+    # in place
+    plan.forward(xd, xd)
+    plan.check()
+    assert np.array_equal(xd.cpu().numpy().reshape(batch, n1, n2), yh)
+    plan.destroy()
+
+
+BF16_TOL = {4: 2e-2, 5: 1e-4}
+
+
+@pytest.mark.parametrize("r,n1,n2", [(16, 256, 256), (8, 64, 512), (32, 1024, 32)])
+@pytest.mark.parametrize("prec", [5, 4])
+def test_dft2_bf16(pkg, r, n1, n2, prec):
+    import torch
+    batch = 2
+    x = inputs.make("normal", n1 * n2, batch, seed=11).reshape(batch, n1, n2)
+    plan = pkg.Plan2(n1, n2, batch, r, prec)
+    y = plan.forward(torch.from_numpy(x).cuda().reshape(-1))
+    plan.check()
+    yh = y.cpu().numpy().reshape(batch, n1, n2)
+    assert _rel(yh, grid.dft2(x, threads=8)).max() <= BF16_TOL[prec]
+    plan.destroy()
+
+
+@pytest.mark.parametrize("r,n1,n2,batch", [(16, 4096, 256, 2), (8, 512, 4096, 1),
+                                           (16, 16, 16, 4)])
+def test_conv2_general(pkg, r, n1, n2, batch):
+    # against the convolution theorem on the oracle's 2-D DFT (pinned)
+    import torch
+    x = inputs.make("uniform", n1 * n2, batch, seed=8).reshape(batch, n1, n2)
+    w = inputs.make("normal", n1 * n2, 1, seed=9).reshape(n1, n2)
+    one = pkg.Plan2(n1, n2, 1, r, 3)
+    spec = one.forward(torch.from_numpy(w).cuda().reshape(-1))
+    plan = pkg.Plan2(n1, n2, batch, r, 3)
+    xd = torch.from_numpy(x).cuda().reshape(-1)
+    y = plan.conv(xd, spec)
+    plan.check()
+    one.check()
+    yh = y.cpu().numpy().reshape(batch, n1, n2)
+    ref = grid.dft2(grid.dft2(x, threads=8) * grid.dft2(w, threads=8)[None], inverse=True,
+                    threads=8)
+    assert _rel(yh, ref).max() <= 1e-5
+    plan.destroy()
+    one.destroy()
+
+
 def test_dft2_in_place_and_closed_form(pkg):
     import torch
     n1, n2 = 64, 64
@@ -102,7 +167,8 @@ def test_conv2_matches_the_definition(pkg, r, n1, n2, batch):
 HEAT = [[0.0, 0.1, 0.0], [0.15, 0.5, 0.15], [0.0, 0.1, 0.0]]
 
 
-@pytest.mark.parametrize("r,k", [(8, 1), (8, 5), (16, 20), (8, 40), (32, 100)])
+@pytest.mark.parametrize("r,k", [(8, 1), (8, 5), (16, 20), (8, 40), (32, 100), (16, 128),
+                                 (8, 200)])
 def test_stencil_weights(pkg, r, k):
     # a positive stencil of unit sum (like the heat update): coefficients of
     # P^k stay within fp32 range for any k
@@ -140,7 +206,8 @@ def test_stencil_weights(pkg, r, k):
 # three radix-8 stages per axis) whose 452^2 block is cut at 100
 @pytest.mark.parametrize("r,side,k", [(8, 64, 4), (8, 96, 8), (16, 128, 16), (8, 120, 20),
                                       (8, 100, 6), (16, 130, 16), (8, 37, 5),
-                                      (8, 2000, 16), (16, 300, 16), (8, 100, 30)])
+                                      (8, 2000, 16), (16, 300, 16), (8, 100, 30),
+                                      (16, 300, 128), (8, 300, 200)])
 def test_stencil_apply(pkg, r, side, k):
     import torch
     rng = np.random.default_rng(side + k)
