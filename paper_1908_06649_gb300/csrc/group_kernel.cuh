@@ -219,7 +219,8 @@ struct SmemLayout {
   static constexpr size_t OFF_TW1 = IMG;
   static constexpr size_t OFF_TW2 = OFF_TW1 + (size_t)TW1 * 8;
   static constexpr size_t PTS = 128 * (size_t)TEAM * R;  // points per item
-  static constexpr size_t OFF_BUF = (OFF_TW2 + (size_t)TW2 * 8 + 127) / 128 * 128;
+  // transpose buffers aligned to 1024 bytes (swz_addr XORs address bits)
+  static constexpr size_t OFF_BUF = (OFF_TW2 + (size_t)TW2 * 8 + 1023) / 1024 * 1024;
   // SHARE: staging and transpose in one buffer (the half-K radix-32 items)
   static constexpr size_t OFF_STG = OFF_BUF + (SHARE ? 0 : (size_t)NTEAM * PTS * 8);
   static constexpr size_t OFF_TWS = OFF_STG + (size_t)NTEAM * PTS * 8;
@@ -307,6 +308,26 @@ __device__ __forceinline__ int gswz(int p, uint32_t tabv) {
   uint32_t h = tabv ^ (uint32_t)(p >> 4);
   if (WIDE) h ^= (uint32_t)(p >> 8);
   return p ^ (int)(h & 15u);
+}
+
+// The swizzle with a zero table value, at compile time.
+template <bool WIDE>
+__host__ __device__ constexpr int gswz0(int p) {
+  return p ^ (((p >> 4) ^ (WIDE ? (p >> 8) : 0)) & 15);
+}
+
+// Shared address of entry gswz(base | (j << SH)) of a transpose buffer,
+// for a row whose base index has no bit in [SH, SH + log2 R): the swizzle
+// is linear over XOR, so the entry is gswz(base) ^ gswz0(j << SH).  `a` is
+// the address of gswz(base) in a buffer aligned to 1024 bytes, so that an
+// XOR below bit 10 of the byte offset is an XOR of the address; the part
+// of j << SH above the first 16 entries (SH >= 4) is disjoint from the
+// other bits and is added instead (an immediate offset of the access).
+template <bool WIDE, int SH>
+__device__ __forceinline__ uint32_t swz_addr(uint32_t a, int j) {
+  const int c = gswz0<WIDE>(j << SH);
+  const int hi = SH >= 4 ? (j << SH) : 0;
+  return (a ^ (uint32_t)(8 * (c ^ hi))) + (uint32_t)(8 * hi);
 }
 
 // Precision modes: 1 TF32, 3 3xTF32 (kind::tf32, K = 8 fp32 per product);
@@ -543,13 +564,20 @@ __device__ __forceinline__ void stage_epilogue(const PRun &P, const float2 *tws,
   const float2 *twrow = tws + TWOFF + lo;  // [j][lo], row length R^(S-T)
   float d[2 * R];
   load_d_row<G, PREC>(w, d);
+#ifndef TCU_DFT_CHECKED
+  const uint32_t a = smem_u32(w.buf) + 8u * (uint32_t)gswz<(G::LOG2L > 8)>(base, tabv);
+#endif
 #pragma unroll
   for (int j = 0; j < R; ++j) {
     const float2 t = in_range(w, TWOFF + lo + (j << SH), G::TW_ENTRIES) ? twrow[j << SH]
                                                                          : make_float2(1.f, 0.f);
     const float2 y = cmul(make_float2(d[2 * j], d[2 * j + 1]), t);
+#ifdef TCU_DFT_CHECKED
     const int bi = gswz<(G::LOG2L > 8)>(base + (j << SH), tabv);
     if (in_range(w, bi, G::GPTS)) w.buf[bi] = y;
+#else
+    st_shared_f2(swz_addr<(G::LOG2L > 8), SH>(a, j), y);
+#endif
   }
 }
 
@@ -564,13 +592,20 @@ __device__ __forceinline__ void stage_rows(const PRun &P, const WG &w) {
   const int hi = q >> SH, lo = q & ((1 << SH) - 1);
   const int base = (ul << G::LOG2L) + (hi << (SH + G::LOG2R)) + lo;
   const uint32_t tabv = (uint32_t)(P.swz_tab >> (4 * (ul & 15))) & 15u;
+#ifndef TCU_DFT_CHECKED
+  const uint32_t a = smem_u32(w.buf) + 8u * (uint32_t)gswz<(G::LOG2L > 8)>(base, tabv);
+#endif
 #pragma unroll
   for (int c = 0; c < R; c += 8) {
     float2 row[8];
 #pragma unroll
     for (int jj = 0; jj < 8; ++jj) {
+#ifdef TCU_DFT_CHECKED
       const int bi = gswz<(G::LOG2L > 8)>(base + ((c + jj) << SH), tabv);
       row[jj] = in_range(w, bi, G::GPTS) ? w.buf[bi] : make_float2(0.f, 0.f);
+#else
+      row[jj] = ld_shared_f2(swz_addr<(G::LOG2L > 8), SH>(a, c + jj));
+#endif
     }
     split_store8<PREC>(row, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
                        w.slot + G::Q + w.lane_off + a_cols8(PREC) * c / 8);
@@ -795,13 +830,20 @@ __device__ __forceinline__ void stage_rows_half(const PRun &P, const WG &w, int 
   const int hi = q >> SH, lo = q & ((1 << SH) - 1);
   const int base = (ul << G::LOG2L) + (hi << (SH + G::LOG2R)) + lo;
   const uint32_t tabv = (uint32_t)(P.swz_tab >> (4 * (ul & 15))) & 15u;
+#ifndef TCU_DFT_CHECKED
+  const uint32_t a = smem_u32(w.buf) + 8u * (uint32_t)gswz<(G::LOG2L > 8)>(base, tabv);
+#endif
 #pragma unroll
   for (int c = 0; c < H; c += 8) {
     float2 row[8];
 #pragma unroll
     for (int jj = 0; jj < 8; ++jj) {
+#ifdef TCU_DFT_CHECKED
       const int bi = gswz<(G::LOG2L > 8)>(base + ((h * H + c + jj) << SH), tabv);
       row[jj] = in_range(w, bi, G::GPTS) ? w.buf[bi] : make_float2(0.f, 0.f);
+#else
+      row[jj] = ld_shared_f2(swz_addr<(G::LOG2L > 8), SH>(a, h * H + c + jj));
+#endif
     }
     split_store8<PREC>(row, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
                        w.slot + G::QA + w.lane_off + a_cols8(PREC) * c / 8);
@@ -1077,7 +1119,9 @@ __device__ __forceinline__ void init_wg(WG &w, uint32_t tbase, unsigned char *sm
   w.tws = reinterpret_cast<float2 *>(smem + SM::OFF_TWS) + (SM::TWS_BYTES ? team * SM::PTS : 0);
   w.twb = reinterpret_cast<float2 *>(smem + SM::OFF_TWB) + team * SM::TWB_PER_WG;
   w.ph_mma = w.ph_stg = w.ph_tws = 0;
-  w.fail = false;
+  // the transpose addressing needs the 1024-byte alignment the dynamic
+  // shared memory is declared with; a base without it fails the launch
+  w.fail = (smem_u32(smem) & 1023u) != 0;
   w.tws_inflight = false;
 }
 
