@@ -338,6 +338,12 @@ __host__ __device__ constexpr bool is_split(int PREC) { return PREC == 3 || PREC
 // TMEM columns of the A operand for 8 complex values, and bytes of one F_r
 // image (2r x 2r elements).
 __host__ __device__ constexpr int a_cols8(int PREC) { return is_bf16(PREC) ? 8 : 16; }
+// Values per register chunk of the loops that load operands (twiddles, rows,
+// spectra) ahead of the asm stores that consume them: 16, or 8 where five
+// warpgroups share the registers (at most 102 a thread).
+__host__ __device__ constexpr int load_chunk(int R, int NWG) {
+  return (R < 16 || NWG >= 5) ? 8 : 16;
+}
 __host__ __device__ constexpr int img_bytes(int R, int PREC) {
   return (is_bf16(PREC) ? 8 : 16) * R * R;
 }
@@ -562,22 +568,41 @@ __device__ __forceinline__ void stage_epilogue(const PRun &P, const float2 *tws,
   const int base = (ul << G::LOG2L) + (hi << (SH + G::LOG2R)) + lo;
   const uint32_t tabv = (uint32_t)(P.swz_tab >> (4 * (ul & 15))) & 15u;
   const float2 *twrow = tws + TWOFF + lo;  // [j][lo], row length R^(S-T)
-  float d[2 * R];
-  load_d_row<G, PREC>(w, d);
 #ifndef TCU_DFT_CHECKED
   const uint32_t a = smem_u32(w.buf) + 8u * (uint32_t)gswz<(G::LOG2L > 8)>(base, tabv);
 #endif
+  // The twiddles of a chunk are loaded before its stores (and the first
+  // chunk's before the TMEM load): the stores and the TMEM load are asm
+  // statements with a memory clobber, so a load written after one of them
+  // would be issued only after it, one shared-memory round trip per value.
+  constexpr int CH = load_chunk(R, G::NWG);
+  float2 t[CH];
 #pragma unroll
-  for (int j = 0; j < R; ++j) {
-    const float2 t = in_range(w, TWOFF + lo + (j << SH), G::TW_ENTRIES) ? twrow[j << SH]
-                                                                         : make_float2(1.f, 0.f);
-    const float2 y = cmul(make_float2(d[2 * j], d[2 * j + 1]), t);
+  for (int jj = 0; jj < CH; ++jj)
+    t[jj] = in_range(w, TWOFF + lo + (jj << SH), G::TW_ENTRIES) ? twrow[jj << SH]
+                                                                 : make_float2(1.f, 0.f);
+  float d[2 * R];
+  load_d_row<G, PREC>(w, d);
+#pragma unroll
+  for (int c = 0; c < R; c += CH) {
+    if (c > 0) {
+#pragma unroll
+      for (int jj = 0; jj < CH; ++jj)
+        t[jj] = in_range(w, TWOFF + lo + ((c + jj) << SH), G::TW_ENTRIES)
+                    ? twrow[(c + jj) << SH]
+                    : make_float2(1.f, 0.f);
+    }
+#pragma unroll
+    for (int jj = 0; jj < CH; ++jj) {
+      const int j = c + jj;
+      const float2 y = cmul(make_float2(d[2 * j], d[2 * j + 1]), t[jj]);
 #ifdef TCU_DFT_CHECKED
-    const int bi = gswz<(G::LOG2L > 8)>(base + (j << SH), tabv);
-    if (in_range(w, bi, G::GPTS)) w.buf[bi] = y;
+      const int bi = gswz<(G::LOG2L > 8)>(base + (j << SH), tabv);
+      if (in_range(w, bi, G::GPTS)) w.buf[bi] = y;
 #else
-    st_shared_f2(swz_addr<(G::LOG2L > 8), SH>(a, j), y);
+      st_shared_f2(swz_addr<(G::LOG2L > 8), SH>(a, j), y);
 #endif
+    }
   }
 }
 
@@ -595,11 +620,14 @@ __device__ __forceinline__ void stage_rows(const PRun &P, const WG &w) {
 #ifndef TCU_DFT_CHECKED
   const uint32_t a = smem_u32(w.buf) + 8u * (uint32_t)gswz<(G::LOG2L > 8)>(base, tabv);
 #endif
+  // a whole chunk is loaded before its TMEM stores (asm with a memory
+  // clobber, which a later load could not pass)
+  constexpr int CH = load_chunk(R, G::NWG);
 #pragma unroll
-  for (int c = 0; c < R; c += 8) {
-    float2 row[8];
+  for (int c = 0; c < R; c += CH) {
+    float2 row[CH];
 #pragma unroll
-    for (int jj = 0; jj < 8; ++jj) {
+    for (int jj = 0; jj < CH; ++jj) {
 #ifdef TCU_DFT_CHECKED
       const int bi = gswz<(G::LOG2L > 8)>(base + ((c + jj) << SH), tabv);
       row[jj] = in_range(w, bi, G::GPTS) ? w.buf[bi] : make_float2(0.f, 0.f);
@@ -607,8 +635,10 @@ __device__ __forceinline__ void stage_rows(const PRun &P, const WG &w) {
       row[jj] = ld_shared_f2(swz_addr<(G::LOG2L > 8), SH>(a, c + jj));
 #endif
     }
-    split_store8<PREC>(row, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
-                       w.slot + G::Q + w.lane_off + a_cols8(PREC) * c / 8);
+#pragma unroll
+    for (int c8 = 0; c8 < CH; c8 += 8)
+      split_store8<PREC>(row + c8, w.slot + w.lane_off + a_cols8(PREC) * (c + c8) / 8,
+                         w.slot + G::Q + w.lane_off + a_cols8(PREC) * (c + c8) / 8);
   }
 }
 
@@ -672,38 +702,43 @@ __device__ __forceinline__ void last_stage_store(const PRun &P, long long item, 
   const long long toff = klow * G::GG + ul, goff = ((long long)klow << G::LOG2VL) + vl;
   const long long gboff = (vh << G::LOG2L) + klow;
   const float2 one = make_float2(1.f, 0.f);
+  // The factors of a chunk of outputs (spectrum, twiddles) are loaded before
+  // its stores: the stores are asm with a memory clobber, so a load written
+  // after one of them would wait for it, a round trip per value.
+  constexpr int CH = (G::TW2L || G::MODE_LAST == kRQF) ? 8 : load_chunk(R, G::NWG);
 #pragma unroll
-  for (int j = 0; j < R; ++j) {
-    float2 y = make_float2(d[2 * j], d[2 * j + 1]);
-    if (G::MODE_LAST == kRQF && mul)
-      y = cmul(y, in_range(w, soff + j * JS, (P.spec_mask + 1) << G::LOG2L) ? __ldg(sp + j * JS)
-                                                                          : one);
-    if (G::TW_SMEM) {
-      const float2 ta = in_range(w, toff + j * TJS, G::GPTS) ? tws[j * TJS] : one;
-      if (G::TW2L) {
-        const float2 tb = in_range(w, klow + j * TBJ, G::L) ? twbs[j * TBJ] : one;
-        y = cmul(y, cmul(ta, tb));
-      } else {
-        y = cmul(y, ta);
-      }
-    } else if (G::TW_OUT) {
-      const float2 ta =
-          in_range(w, goff + j * TWG, (long long)G::L << G::LOG2VL) ? __ldg(twg + j * TWG) : one;
-      if (G::TW2L) {
-        const float2 tb =
-            in_range(w, gboff + j * TBJ, (1ll << (G::LOG2UPER - G::LOG2VL)) << G::LOG2L)
-                ? __ldg(twbg + j * TBJ)
-                : one;
-        y = cmul(y, cmul(ta, tb));
-      } else {
-        y = cmul(y, ta);
+  for (int c = 0; c < R; c += CH) {
+    float2 fs[CH], fa[CH], fb[CH];
+#pragma unroll
+    for (int jj = 0; jj < CH; ++jj) {
+      const int j = c + jj;
+      if (G::MODE_LAST == kRQF && mul)
+        fs[jj] = in_range(w, soff + j * JS, (P.spec_mask + 1) << G::LOG2L) ? __ldg(sp + j * JS)
+                                                                          : one;
+      if (G::TW_SMEM) {
+        fa[jj] = in_range(w, toff + j * TJS, G::GPTS) ? tws[j * TJS] : one;
+        if (G::TW2L) fb[jj] = in_range(w, klow + j * TBJ, G::L) ? twbs[j * TBJ] : one;
+      } else if (G::TW_OUT) {
+        fa[jj] = in_range(w, goff + j * TWG, (long long)G::L << G::LOG2VL) ? __ldg(twg + j * TWG)
+                                                                          : one;
+        if (G::TW2L)
+          fb[jj] = in_range(w, gboff + j * TBJ, (1ll << (G::LOG2UPER - G::LOG2VL)) << G::LOG2L)
+                       ? __ldg(twbg + j * TBJ)
+                       : one;
       }
     }
-    if (in_range(w, doff + j * JS, out_elems)) {
-      if (OUT_L2)
-        __stcg(dst + j * JS, y);
-      else
-        __stcs(dst + j * JS, y);
+#pragma unroll
+    for (int jj = 0; jj < CH; ++jj) {
+      const int j = c + jj;
+      float2 y = make_float2(d[2 * j], d[2 * j + 1]);
+      if (G::MODE_LAST == kRQF && mul) y = cmul(y, fs[jj]);
+      if (G::TW_SMEM || G::TW_OUT) y = G::TW2L ? cmul(y, cmul(fa[jj], fb[jj])) : cmul(y, fa[jj]);
+      if (in_range(w, doff + j * JS, out_elems)) {
+        if (OUT_L2)
+          __stcg(dst + j * JS, y);
+        else
+          __stcs(dst + j * JS, y);
+      }
     }
   }
 }
@@ -833,21 +868,22 @@ __device__ __forceinline__ void stage_rows_half(const PRun &P, const WG &w, int 
 #ifndef TCU_DFT_CHECKED
   const uint32_t a = smem_u32(w.buf) + 8u * (uint32_t)gswz<(G::LOG2L > 8)>(base, tabv);
 #endif
+  // the half row is loaded before its TMEM stores (asm with a memory
+  // clobber, which a later load could not pass)
+  float2 row[H];
 #pragma unroll
-  for (int c = 0; c < H; c += 8) {
-    float2 row[8];
-#pragma unroll
-    for (int jj = 0; jj < 8; ++jj) {
+  for (int jj = 0; jj < H; ++jj) {
 #ifdef TCU_DFT_CHECKED
-      const int bi = gswz<(G::LOG2L > 8)>(base + ((h * H + c + jj) << SH), tabv);
-      row[jj] = in_range(w, bi, G::GPTS) ? w.buf[bi] : make_float2(0.f, 0.f);
+    const int bi = gswz<(G::LOG2L > 8)>(base + ((h * H + jj) << SH), tabv);
+    row[jj] = in_range(w, bi, G::GPTS) ? w.buf[bi] : make_float2(0.f, 0.f);
 #else
-      row[jj] = ld_shared_f2(swz_addr<(G::LOG2L > 8), SH>(a, h * H + c + jj));
+    row[jj] = ld_shared_f2(swz_addr<(G::LOG2L > 8), SH>(a, h * H + jj));
 #endif
-    }
-    split_store8<PREC>(row, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
-                       w.slot + G::QA + w.lane_off + a_cols8(PREC) * c / 8);
   }
+#pragma unroll
+  for (int c = 0; c < H; c += 8)
+    split_store8<PREC>(row + c, w.slot + w.lane_off + a_cols8(PREC) * c / 8,
+                       w.slot + G::QA + w.lane_off + a_cols8(PREC) * c / 8);
 }
 
 template <class G, int PREC, class Mid>
@@ -1049,13 +1085,16 @@ __device__ __forceinline__ void process_item_conv(const PRun &P, const float2 *t
 // first item's input copy; wait_tables() before the first use.  Every size
 // is a multiple of 16 bytes (the images 64 r^2 bytes, the twiddle tables an
 // even number of complex values).
+// kernel_setup_start leaves the CTA unsynchronised, so that warp 0 can issue
+// its first input copy (its mbarriers are initialised by then, in program
+// order within warp 0) before kernel_setup_finish's CTA barrier.
 template <int NWG, int THREADS>
-__device__ __forceinline__ uint32_t kernel_setup(const float *bimg, int img_floats,
-                                                 float *img, const float2 *tw_src0,
-                                                 float2 *tw_dst0, int tw_n0,
-                                                 const float2 *tw_src1, float2 *tw_dst1,
-                                                 int tw_n1, uint64_t *mbar,
-                                                 uint32_t *tmem_slot) {
+__device__ __forceinline__ void kernel_setup_start(const float *bimg, int img_floats,
+                                                   float *img, const float2 *tw_src0,
+                                                   float2 *tw_dst0, int tw_n0,
+                                                   const float2 *tw_src1, float2 *tw_dst1,
+                                                   int tw_n1, uint64_t *mbar,
+                                                   uint32_t *tmem_slot) {
   const int tid = threadIdx.x;
   uint64_t *tbar = mbar + 3 * NWG + 1;
   if (tid == 0) {
@@ -1069,11 +1108,29 @@ __device__ __forceinline__ uint32_t kernel_setup(const float *bimg, int img_floa
     if (bytes1) tma_load_1d(smem_u32(tw_dst0), tw_src0, bytes1, smem_u32(tbar));
     if (bytes2) tma_load_1d(smem_u32(tw_dst1), tw_src1, bytes2, smem_u32(tbar));
   }
-  if ((tid >> 5) == 0) tmem_alloc(smem_u32(tmem_slot), 512);
+  if ((tid >> 5) == 0) {
+    __syncwarp();
+    tmem_alloc(smem_u32(tmem_slot), 512);
+  }
+}
+
+__device__ __forceinline__ uint32_t kernel_setup_finish(const uint32_t *tmem_slot) {
   fence_before_sync();
   __syncthreads();
   fence_after_sync();
   return *tmem_slot;
+}
+
+template <int NWG, int THREADS>
+__device__ __forceinline__ uint32_t kernel_setup(const float *bimg, int img_floats,
+                                                 float *img, const float2 *tw_src0,
+                                                 float2 *tw_dst0, int tw_n0,
+                                                 const float2 *tw_src1, float2 *tw_dst1,
+                                                 int tw_n1, uint64_t *mbar,
+                                                 uint32_t *tmem_slot) {
+  kernel_setup_start<NWG, THREADS>(bimg, img_floats, img, tw_src0, tw_dst0, tw_n0, tw_src1,
+                                   tw_dst1, tw_n1, mbar, tmem_slot);
+  return kernel_setup_finish(tmem_slot);
 }
 
 // Every thread, before the first use of the F images or stage twiddles.
@@ -1159,11 +1216,11 @@ __global__ void __launch_bounds__(
   uint32_t *tmem_slot = reinterpret_cast<uint32_t *>(mbar + 3 * G::NWG);
   const PRun &P = a.p[0];
   // a convolution row pass also holds the inverse stage twiddles (p[1])
-  const uint32_t tbase = kernel_setup<G::NWG, G::THREADS>(
+  kernel_setup_start<G::NWG, G::THREADS>(
       a.bimg, (int)(SM::IMG / 4), reinterpret_cast<float *>(smem), P.tw_stage, tw,
       G::TW_ENTRIES, a.p[1].tw_stage, tw_inv, CONV ? G::TW_ENTRIES : 0, mbar, tmem_slot);
   WG w;
-  init_wg<R, SM, G::GCOLS, TW>(w, tbase, smem);
+  init_wg<R, SM, G::GCOLS, TW>(w, 0, smem);  // TMEM slot set below
 #ifdef TCU_DFT_CHECKED
   w.err = a.err;
 #endif
@@ -1177,7 +1234,12 @@ __global__ void __launch_bounds__(
   // item: position in this CTA's sequence; phys: the item processed there
   // (team passes always run forward: no reversal code in them)
   auto phys = [&](long long i) { return TW == 1 && P.reverse ? nitems - 1 - i : i; };
-  if (w.team_lead && item < nitems) issue_input<G>(P, &a.tm_in, phys(item), w);
+  // the first input copy of team 0 leaves with the tables (warp 0 set up its
+  // mbarriers), the other teams' after the CTA barrier
+  if (team == 0 && w.team_lead && item < nitems) issue_input<G>(P, &a.tm_in, phys(item), w);
+  const uint32_t tbase = kernel_setup_finish(tmem_slot);
+  w.slot = tbase + (uint32_t)((threadIdx.x >> 7) * G::GCOLS);
+  if (team != 0 && w.team_lead && item < nitems) issue_input<G>(P, &a.tm_in, phys(item), w);
   // the tables have landed (the same answer in every thread of the team)
   if (named_bar_or(w.bar_id, w.bar_count, !wait_tables(mbar, G::NWG))) w.fail = true;
   while (item < nitems && !w.fail) {
