@@ -360,12 +360,14 @@ __device__ __forceinline__ void split_store8(const float2 *x, uint32_t col_hi,
     uint32_t ph[8], pl[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
-      const __nv_bfloat16 hx = __float2bfloat16_rn(x[j].x), hy = __float2bfloat16_rn(x[j].y);
-      ph[j] = (uint32_t)__bfloat16_as_ushort(hx) | ((uint32_t)__bfloat16_as_ushort(hy) << 16);
+      // both parts rounded to nearest by one packed conversion (re in the
+      // low half, im in the high half, as the B images expect)
+      const __nv_bfloat162 h = __floats2bfloat162_rn(x[j].x, x[j].y);
+      ph[j] = *reinterpret_cast<const uint32_t *>(&h);
       if (PREC == 5) {
-        const __nv_bfloat16 lx = __float2bfloat16_rn(x[j].x - __bfloat162float(hx));
-        const __nv_bfloat16 ly = __float2bfloat16_rn(x[j].y - __bfloat162float(hy));
-        pl[j] = (uint32_t)__bfloat16_as_ushort(lx) | ((uint32_t)__bfloat16_as_ushort(ly) << 16);
+        const __nv_bfloat162 l =
+            __floats2bfloat162_rn(x[j].x - __low2float(h), x[j].y - __high2float(h));
+        pl[j] = *reinterpret_cast<const uint32_t *>(&l);
       }
     }
     tmem_st8u(col_hi, ph);
