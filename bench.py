@@ -203,6 +203,33 @@ def profiled_traffic(batch, fused):
         return None
 
 
+def copy_floor_ms(h_in, h_out, d_in, d_out, stream, reps=3):
+    """Least time to copy h_in -> d_in and d_out -> h_out at once (one
+    cudaMemcpyAsync each, on two streams): the link's floor for a step of the
+    end-to-end path, which must move these bytes whatever the transform."""
+    import torch
+    s_in, s_out = torch.cuda.Stream(), torch.cuda.Stream()
+    f0 = torch.cuda.Event(enable_timing=True)
+    f1 = torch.cuda.Event(enable_timing=True)
+    best = None
+    for _ in range(reps):
+        torch.cuda.synchronize()
+        f0.record(stream)
+        s_in.wait_event(f0)
+        s_out.wait_event(f0)
+        with torch.cuda.stream(s_in):
+            d_in.copy_(h_in, non_blocking=True)
+        with torch.cuda.stream(s_out):
+            h_out.copy_(d_out, non_blocking=True)
+        stream.wait_stream(s_in)
+        stream.wait_stream(s_out)
+        f1.record(stream)
+        torch.cuda.synchronize()
+        t = f0.elapsed_time(f1)
+        best = t if best is None else min(best, t)
+    return best
+
+
 def rank_seed(wl, rank):
     """Each rank transforms its own batch (weak scaling): the workload's
     recipe with the seed offset by 1000 * rank."""
@@ -808,11 +835,17 @@ def main():
         torch.cuda.synchronize()
         e2e_ms = e0.elapsed_time(e1)
         e2e_ms = max_over_ranks(e2e_ms, dist, dev)
+        floor_ms = copy_floor_ms(h_in, h_out, work, x, stream)
         e2e = {"value": job_rate(dft_flops(n, batch), world, args.e2e_steps,
                                  e2e_ms),
                "unit": UNIT, "h2d_bytes_per_step": n * batch * 8,
                "d2h_bytes_per_step": n * batch * 8,
-               "steps": args.e2e_steps}
+               "steps": args.e2e_steps,
+               "ms_per_step": e2e_ms / args.e2e_steps,
+               # this machine's host<->device link, measured on the same pinned
+               # buffers: a step's bytes both ways at once, without the DFT
+               "copy_floor_ms_per_step": floor_ms,
+               "frac_of_copy_floor": floor_ms / (e2e_ms / args.e2e_steps)}
 
     # whole-step roofline: min HBM bytes vs tensor flops at the TF32 peak,
     # measured here (cuBLAS TF32 GEMM, after every timed region) or, if that
