@@ -247,7 +247,9 @@ struct WG {
   int bar_count;      // threads of the team
   int rho;            // this thread's row within the item (0 .. 128 TW - 1)
   bool wg_lead;       // warp 0 of its warpgroup: issues the warpgroup's products
-  bool team_lead;     // warp 0 of the team: issues copies, runs the schedule
+  bool team_lead;     // warp 0 of the team: runs the schedule
+  bool copy_lead;     // issues the team's copies: warp 0 of the team, or warp 1
+                      // in the strided passes of two or more stages
   float2 *buf;        // SMEM transpose buffer
   float2 *stg;        // SMEM input staging (one item)
   float2 *tws;        // SMEM twiddle staging (one item)
@@ -776,7 +778,7 @@ __device__ __forceinline__ void process_item(const PRun &P, const CUtensorMap *t
     fence_after_sync();
     issue_stage<R, PREC>(w.slot, w.img_addr + (S == 1 ? P.last_img : 0), w.bar_mma);
   }
-  if (w.team_lead) {
+  if (w.copy_lead) {
     if (G::TW_SMEM) {
       issue_twiddles<G>(P, tm_tw, item, w);
       w.tws_inflight = true;
@@ -1144,7 +1146,8 @@ __device__ __forceinline__ bool wait_tables(uint64_t *mbar, int nwg) {
 // staging, then free TMEM.
 __device__ __forceinline__ void kernel_teardown(uint32_t tbase, const WG &w, bool stg_pending,
                                                 bool tws_pending) {
-  if (w.rho == 0) {
+  // the first lane of the warp that issued the copies
+  if (w.copy_lead && (threadIdx.x & 31) == 0) {
     if (stg_pending) mbar_wait_bounded(w.bar_stg, w.ph_stg);
     if (tws_pending) mbar_wait_bounded(w.bar_tws, w.ph_tws);
   }
@@ -1164,6 +1167,7 @@ __device__ __forceinline__ void init_wg(WG &w, uint32_t tbase, unsigned char *sm
   w.rho = (wt * 4 + (warp & 3)) * 32 + lane;
   w.wg_lead = (warp & 3) == 0;
   w.team_lead = w.wg_lead && wt == 0;
+  w.copy_lead = w.team_lead;
   w.slot = tbase + wg * GCOLS;
   w.lane_off = (uint32_t)((warp & 3) * 32) << 16;
   w.img_addr = smem_u32(smem);
@@ -1223,6 +1227,13 @@ __global__ void __launch_bounds__(
       G::TW_ENTRIES, a.p[1].tw_stage, tw_inv, CONV ? G::TW_ENTRIES : 0, mbar, tmem_slot);
   WG w;
   init_wg<R, SM, G::GCOLS, TW>(w, 0, smem);  // TMEM slot set below
+  // In a strided pass of two or more stages warp 1 issues the copies after
+  // the first one (the inter-pass twiddles and the next input), beside warp
+  // 0's products, which the other warps otherwise wait for at the next
+  // barrier (measured: these passes 1 % faster; the others, and one-stage
+  // strided passes, slower)
+  if (ROLE == kFirst && S >= 2 && !G::KS && !CONV)
+    w.copy_lead = (threadIdx.x >> 5) % (4 * TW) == 1;
 #ifdef TCU_DFT_CHECKED
   w.err = a.err;
 #endif
